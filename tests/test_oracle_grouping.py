@@ -1,0 +1,78 @@
+"""Pins of the head-grouping rule (Sec. 4, Step 2)."""
+import math
+
+import numpy as np
+import pytest
+
+from oracle import headkv as O
+from synth import configs, gen
+
+
+def test_uniform_attention_count_is_ceil_tau_len():
+    # q = 0 makes every logit equal: the newest n tokens carry n/len
+    for n, tau in ((47, 0.9), (100, 0.85), (13, 0.95), (64, 0.9)):
+        K = np.random.default_rng(n).normal(size=(n, 8))
+        n_h, cum = O.grouping_count(np.zeros(8), K, tau)
+        expect = math.ceil(tau * n)
+        if abs(tau * n - round(tau * n)) < 1e-9:   # exact multiple: fp boundary
+            assert n_h in (expect, expect + 1)
+        else:
+            assert n_h == expect
+
+
+def test_dominant_newest_token_is_local():
+    D = 64
+    K = np.zeros((40, D)); K[-1, 0] = 30 * math.sqrt(D)
+    q = np.zeros(D); q[0] = 1.0
+    n_h, _ = O.grouping_count(q, K, 0.9)
+    assert n_h == 1 and O.classify(n_h, 32) == O.LOCAL
+
+
+def test_hand_worked_masses():
+    # D = 1, logits ln(p) give attention exactly proportional to p
+    p = np.array([0.04, 0.06, 0.1, 0.3, 0.5])          # oldest .. newest
+    K = np.log(p)[:, None]
+    q = np.array([1.0])
+    # backward masses 0.5, 0.8, 0.9, 0.96, 1.0
+    assert O.grouping_count(q, K, 0.85)[0] == 3
+    assert O.grouping_count(q, K, 0.75)[0] == 2
+    assert O.grouping_count(q, K, 0.95)[0] == 4
+    assert O.grouping_count(q, K, 0.45)[0] == 1
+    # w_loc = 3: n_h = 3 is not below it -> global; w_loc = 4 -> local
+    assert O.classify(3, 3) == O.GLOBAL and O.classify(3, 4) == O.LOCAL
+    _, cum = O.grouping_count(q, K, 0.85)
+    assert abs(O.label_margin(cum, 0.85, 4) - 0.05) < 1e-12   # mass of newest 3 = 0.9
+
+
+def test_backward_accumulation_starts_at_newest():
+    # a heavy OLD token must not make the head local
+    D = 64
+    K = np.zeros((50, D)); K[0, 0] = 30 * math.sqrt(D)
+    q = np.zeros(D); q[0] = 1.0
+    n_h, _ = O.grouping_count(q, K, 0.9)
+    assert n_h == 50 and O.classify(n_h, 32) == O.GLOBAL
+
+
+def test_hand_case_labels():
+    from _hand import load
+    case, heads = load()
+    c = case["config"]
+    for hd in heads:
+        t = c["group_at"] - 1
+        K = hd["k"][: c["n_cond"] + t + 1]
+        n_h, cum = O.grouping_count(hd["q"][t], K, c["tau"])
+        assert n_h == hd["expected"]["n_h"]
+        assert O.classify(n_h, c["local_w"]) == hd["expected"]["label"]
+
+
+def test_tiny_generator_gives_intended_head_types():
+    """Tiny workload: beta = 4 heads (0-3) local, beta = 0.3 heads (4-7) global."""
+    w = configs.TINY
+    hp = O.HeadParams.of(w)
+    labels = []
+    for h in range(w.n_heads):
+        hi = gen.HeadInputs(w, 0, 0, h)
+        tr = O.run_head(hp, hi.q, hi.k, hi.v, stop_after=w.group_at - 1)
+        labels.append(tr.label_computed)
+        assert tr.margin > 1e-3
+    assert labels == [0, 0, 0, 0, 1, 1, 1, 1]
