@@ -1,0 +1,388 @@
+"""Throughput of the HeadKV decode hot path on GB300.
+
+A bench "step" is one steady-state period of P decode steps of the whole
+model (all L layers): every layer appends its new token and attends over its
+ragged cache at each of the P steps, and runs its periodic head-aware update
+(STE + in-place compaction for global heads, window slide for local ones)
+once, at the start of the period. Inputs (synthetic Q/K/V of the Lumina-mGPT
+1024 shape) are resident in HBM before timing; the per-step KV working set
+(several GB) is far larger than L2.
+
+  value       image tokens/s = images x P x steps / device time
+  roofline    decode attention (the dominant kernel): retained K/V bytes +
+              q/out bytes per launch / measured launch time, vs measured HBM
+  e2e         the same metric through the C-ABI with pinned host buffers:
+              each step copies its inputs in and its outputs out
+  cpu_baseline the CPU oracle on a sample of heads (spawn pool), projected
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                       [--workload lumina1024] [--rho 1/4]
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import multiprocessing as mp
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+from fractions import Fraction
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from synth import configs  # noqa: E402
+
+METRIC = "image tokens/s per decode step on 1 GB300; decode-attn HBM GB/s vs peak"
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def workload(args) -> configs.Workload:
+    return configs.ALL[args.workload].with_(rho=Fraction(args.rho))
+
+
+def steady_start(w: configs.Workload) -> int:
+    """First step at whose start the update trims a full global history."""
+    B_g = math.floor(w.rho * w.n_image)
+    h_g = B_g - w.recent_w
+    hist0 = max(0, w.group_at - w.recent_w)
+    k = max(1, math.ceil(max(0, h_g - hist0) / w.period) + 1)
+    return w.group_at + k * w.period
+
+
+def describe(w, n_steps_window):
+    return (f"{w.name}: L{w.n_layers} H{w.n_heads} D{w.head_dim} {w.dtype}, {w.n_seqs} seqs, "
+            f"C={w.n_cond}, {w.rows}x{w.row_len} grid (N={w.n_image}), rho={w.rho}, "
+            f"w={w.recent_w}, P={w.period}, E={w.group_at}; one step = one steady-state "
+            f"period of P decode steps x L layers")
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (the baseline leg; runs in spawned processes)
+# ---------------------------------------------------------------------------
+def _oracle_period(args):
+    os.environ.setdefault("OPENBLAS_NUM_THREADS", "1")
+    os.environ.setdefault("OMP_NUM_THREADS", "1")
+    from oracle import headkv as O
+    from synth import gen
+    w, (s, l, h), t0 = args
+    hi = gen.HeadInputs(w, s, l, h)
+    hp = O.HeadParams.of(w)
+    # untimed: the head's cache at the start of the window
+    O.run_head(hp, hi.q, hi.k, hi.v, stop_after=t0 - 1)
+    tr0 = time.perf_counter()
+    O.run_head(hp, hi.q, hi.k, hi.v, stop_after=t0 + w.period - 1,
+               record=range(t0, t0 + w.period))
+    full = time.perf_counter() - tr0
+    tr1 = time.perf_counter()
+    O.run_head(hp, hi.q, hi.k, hi.v, stop_after=t0 - 1)
+    prefix = time.perf_counter() - tr1
+    return max(full - prefix, 1e-9)
+
+
+def oracle_rate(w, t0, n_heads, seed, workers):
+    """Projected image tokens/s of the CPU oracle from a sample of heads: the
+    oracle time of one period for each sampled head (its run up to the window
+    minus its run to the window start), averaged, times all L*S*H heads."""
+    import random
+    rnd = random.Random(seed)
+    heads = [(rnd.randrange(w.n_seqs), rnd.randrange(w.n_layers), rnd.randrange(w.n_heads))
+             for _ in range(n_heads)]
+    jobs = [(w, x, t0) for x in heads]
+    with mp.get_context("spawn").Pool(workers) as pool:
+        secs = pool.map(_oracle_period, jobs, chunksize=1)
+    per_head_period = statistics.mean(secs)
+    period_s = per_head_period * w.n_head_total / workers
+    images = w.n_seqs / w.cfg_rows
+    return images * w.period / period_s, per_head_period
+
+
+def run_reference(args):
+    """--impl reference: the CPU oracle as the reference arm."""
+    w = workload(args)
+    t0 = steady_start(w)
+    workers = min(16, os.cpu_count() or 1)
+    vals = []
+    for j in range(args.warmup + args.steps):
+        v, _ = oracle_rate(w, t0, workers, 1000 + j, workers)
+        if j >= args.warmup:
+            vals.append(v)
+    value = statistics.mean(vals)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "image tokens/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1000.0 * (w.n_seqs / w.cfg_rows) * w.period / value,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": {"workload": describe(w, w.period)},
+        "cpu_baseline": {"value": value, "unit": "image tokens/s", "cores": workers,
+                         "kind": "oracle",
+                         "sample": f"per step {workers} random heads, one period each after "
+                                   f"a simulated run to step {t0}, projected to all "
+                                   f"{w.n_head_total} heads"},
+        "e2e": {"value": value, "unit": "image tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index),
+                 "--query-gpu=clocks.sm,clocks.max.sm,clocks_event_reasons.hw_slowdown,"
+                 "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+                 "clocks_event_reasons.sw_power_cap",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        rows = []
+        try:
+            for line in open(self.path):
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 6 and parts[0].isdigit():
+                    rows.append(parts)
+        except Exception:
+            pass
+        finally:
+            if self.path:
+                os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm = [int(r[0]) for r in rows]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[2 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": int(rows[0][1]), "reasons": reasons,
+                "samples": len(rows)}
+
+
+def attn_bytes(cfg, lens):
+    """Algorithmic bytes of one decode-attention launch: every retained K and
+    V row once, the query row in, the fp32 output row out."""
+    es = 2 if cfg.dtype == 1 else 4
+    heads = cfg.n_seqs * cfg.n_heads
+    return int(lens.sum()) * cfg.head_dim * 2 * es + heads * cfg.head_dim * (es + 4)
+
+
+def run_ours(args):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    from paper_2605_20600_gb300 import hkv as H
+    from paper_2605_20600_gb300.engine import Engine, torch_dtype
+    from paper_2605_20600_gb300.runner import generate
+    from synth.gpu import DeviceSynth
+
+    w = workload(args)
+    L, S, Hh, D, P = w.n_layers, w.n_seqs, w.n_heads, w.head_dim, w.period
+    t0 = steady_start(w)
+    K, W = args.steps, args.warmup
+    n_periods = W + K + 2
+    assert t0 + n_periods * P <= w.n_image, "window past the end of the image"
+
+    # CPU baseline first (spawned workers, rank 0, one GPU)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        workers = min(16, os.cpu_count() or 1)
+        rate, per_head = oracle_rate(w, t0, 4 * workers, 7, workers)
+        cpu = {"value": rate, "unit": "image tokens/s", "cores": workers, "kind": "oracle",
+               "sample": f"{4 * workers} random heads of {w.n_head_total}, one period each "
+                         f"(P={P} steps incl. the update) after a simulated run to step {t0}; "
+                         f"mean {per_head * 1e3:.1f} ms per head-period, projected to all heads "
+                         f"on {workers} processes"}
+
+    cfg = H.make_config(n_layers=L, n_seqs=S, n_heads=Hh, head_dim=D, dtype=w.dtype,
+                        n_cond=w.n_cond, n_image=w.n_image, row_len=w.row_len,
+                        recent_w=w.recent_w, local_w=w.w_loc, period=P, group_at=w.group_at,
+                        rho=w.rho, tau=w.tau, r_s=w.r_s)
+    eng = Engine(cfg, dev)
+    synth = DeviceSynth(w, dev)
+    generate(eng, synth, last_step=t0 - 1)      # dense phase, grouping, compression, decode
+    eng.release_dense()
+    torch.cuda.synchronize()
+    eng.check()
+    labels = eng.labels.cpu().numpy()
+    dt = torch_dtype(cfg)
+
+    # resident inputs of every period of the window: [n][3][P][L][S][H][D]
+    pool = torch.empty(n_periods, 3, P, L, S, Hh, D, dtype=dt, device=dev)
+    for j in range(n_periods):
+        synth.image(pool[j, 0], pool[j, 1], pool[j, 2], 0, L, t0 + j * P, P)
+    staging = torch.empty(3, P, L, S, Hh, D, dtype=dt, device=dev)
+    out = torch.empty(P, L, S, Hh, D, dtype=torch.float32, device=dev)
+
+    def period_calls():
+        for p in range(P):
+            for layer in range(L):
+                eng.append(layer, staging[0, p, layer], staging[1, p, layer], staging[2, p, layer])
+                eng.attend(layer, staging[0, p, layer], out[p, layer])
+
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        period_calls()
+    stream = torch.cuda.current_stream()
+    launches_per_step = P * L * 2
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    j = 0
+    for _ in range(W):
+        staging.copy_(pool[j], non_blocking=True)
+        graph.replay()
+        j += 1
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        barrier()
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        for _ in range(K):
+            staging.copy_(pool[j], non_blocking=True)
+            graph.replay()
+            j += 1
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+    ms = ev0.elapsed_time(ev1)
+    clocks = clk.summary()
+    eng.check()
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    images = S / w.cfg_rows
+    value = world * images * P * K / (ms / 1e3)
+
+    # dominant kernel: decode attention of every layer, back to back, at the
+    # cache state the window reached (read-only, so it can be replayed)
+    lens = eng.cache.len.cpu().numpy().reshape(L, S * Hh)
+    bytes_per_launch = statistics.mean(attn_bytes(cfg, lens[layer]) for layer in range(L))
+    q_last = staging[0, P - 1]
+    attn_graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(attn_graph):
+        for layer in range(L):
+            eng.attend(layer, q_last[layer], out[0, layer])
+    reps = 20
+    attn_graph.replay()
+    torch.cuda.synchronize()
+    a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a0.record(stream)
+    for _ in range(reps):
+        attn_graph.replay()
+    a1.record(stream)
+    torch.cuda.synchronize()
+    attn_ms = a0.elapsed_time(a1) / (reps * L)
+    peak, peak_kind = load_peaks()
+    achieved = bytes_per_launch / (attn_ms / 1e3) / 1e9
+
+    # e2e through the C-ABI with pinned host buffers
+    host_in = torch.empty(staging.shape, dtype=dt, pin_memory=True)
+    host_out = torch.empty(out.shape, dtype=torch.float32, pin_memory=True)
+    host_in.copy_(pool[0])
+    e2e_steps = max(1, min(K, 5))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        staging.copy_(host_in, non_blocking=True)
+        graph.replay()
+        host_out.copy_(out, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+    eng.check()
+    e2e_value = world * images * P * e2e_steps / (e2e_ms / 1e3)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "image tokens/s", "n_gpus": world,
+            "steps": K, "warmup": W, "ms_per_step": ms / K, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
+            "config": {"workload": describe(w, P), "rho": str(w.rho),
+                       "decode_steps_per_step": P, "layers": L,
+                       "global_head_fraction": float((labels == 1).mean()),
+                       "window_start_step": t0,
+                       "l2": "no flush: inputs and the per-step KV working set exceed L2",
+                       "parallelism": "replicas" if world > 1 else "single GPU"},
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": None,
+                         "kernel": "attn_kernel (hkv_decode_attention)",
+                         "bytes_per_launch": bytes_per_launch, "launch_us": attn_ms * 1e3,
+                         "peak_kind": peak_kind},
+            "e2e": {"value": e2e_value, "unit": "image tokens/s",
+                    "h2d_bytes_per_step": staging.numel() * staging.element_size(),
+                    "d2h_bytes_per_step": out.numel() * out.element_size()},
+            "gpu_launches": launches_per_step * K,
+            "clocks": clocks,
+        }
+        if cpu is not None:
+            line["cpu_baseline"] = cpu
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="lumina1024", choices=sorted(configs.ALL))
+    ap.add_argument("--rho", default="1/4")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        if int(os.environ.get("RANK", "0")) == 0:
+            run_reference(args)
+        return
+    run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,212 @@
+/*
+ * hkv.h — C-ABI of the HeadKV decode hot path on one GB300 (sm_103a).
+ *
+ * HeadKV ("Head-Aware Key-Value Compression for Efficient Autoregressive
+ * Image Generation") labels every attention head local or global from the
+ * early attention (Sec. 4, Step 2), gives local heads a small budget and
+ * global heads rho*N tokens (Sec. 5.1), trims global heads with Stratified
+ * Token Eviction (Sec. 4, Eqs. 5-6) every P steps, and decodes over the
+ * resulting ragged per-head cache (Eq. 1).
+ *
+ * Conventions for every entry point
+ *  - All pointers to tensors are DEVICE pointers unless marked "host".
+ *    The caller owns every buffer and the stream; the library never
+ *    allocates, frees, or keeps state between calls (all state lives in the
+ *    caller's buffers).
+ *  - All calls are asynchronous on `stream` except hkv_allocate_budgets and
+ *    hkv_check, which synchronise it.
+ *  - Per-head arrays are indexed by the flat head index
+ *        i = (layer * n_seqs + seq) * n_heads + head      ([L][S][H] order),
+ *    so one layer's heads are contiguous.
+ *  - Per-step activations q, k, v are [n_seqs][n_heads][head_dim] in the
+ *    config's dtype (fp32 or bf16), contiguous.
+ *  - Errors: every call validates its arguments before launching anything
+ *    and returns a status; nothing aborts or throws across the ABI.
+ *    Failures detected on the device (capacity, bounds, a bounded wait that
+ *    ran out) set the cache's error word; hkv_check reports it.
+ *  - Fault injection for tests: if the environment variable
+ *    HKV_FAULT_INJECT is "<name>:<code>" (name without the hkv_ prefix, e.g.
+ *    "decode_attention:7"), that call returns <code> before touching the GPU.
+ */
+#ifndef HKV_H
+#define HKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* A CUDA stream (cudaStream_t); NULL selects the legacy default stream. */
+typedef struct CUstream_st *hkv_stream_t;
+
+typedef enum {
+  HKV_OK = 0,
+  HKV_ERR_INVALID_ARG = 1, /* null pointer, bad layer index, bad enum value */
+  HKV_ERR_SHAPE = 2,       /* unsupported head_dim / dtype / sizes */
+  HKV_ERR_CAPACITY = 3,    /* a segment or the workspace is too small */
+  HKV_ERR_STATE = 4,       /* the cache is not in the phase the call needs */
+  HKV_ERR_BOUNDS = 5,      /* a segment reaches outside the arena (device) */
+  HKV_ERR_TIMEOUT = 6,     /* a bounded device wait ran out (device) */
+  HKV_ERR_CUDA = 7,        /* a CUDA runtime call or launch failed */
+  HKV_ERR_ALIGN = 8        /* a pointer is not 16-byte aligned */
+} hkv_status;
+
+enum { HKV_FP32 = 0, HKV_BF16 = 1 };
+
+/* head labels (Sec. 4, Step 2); DENSE marks heads of the uncompressed
+ * prefill-phase cache (Step 1), which are never evicted from */
+enum { HKV_LOCAL = 0, HKV_GLOBAL = 1, HKV_DENSE = 255 };
+
+/*
+ * Model shape and method hyperparameters (plain data, host memory).
+ *  n_cond        C: conditioning tokens, always kept (Eqs. 2-4)
+ *  n_image       N: image tokens per sequence (grid rows x row_len)
+ *  row_len       tokens per grid row, end-of-row token included
+ *  recent_w      w: recent window, two grid rows (Sec. 5.1)
+ *  local_w       w_loc: a head is local iff fewer than w_loc tokens carry
+ *                tau of its attention (Sec. 4, Step 2)
+ *  period        P: tokens buffered between cache updates (Sec. 4,
+ *                Efficient Cache Update)
+ *  group_at      E: image tokens generated when heads are grouped
+ *                (Appendix, More Implementation Details)
+ *  global_budget B_g = floor(rho * N) image tokens kept by a global head
+ *                (Sec. 5.1); must be >= recent_w
+ *  tau           accumulation threshold, 0.9 in the paper (Step 2)
+ *  r_s           long/near split ratio, 0.5 in the paper (Eq. 5)
+ */
+typedef struct {
+  int32_t n_layers, n_seqs, n_heads, head_dim;
+  int32_t dtype; /* HKV_FP32 or HKV_BF16 */
+  int32_t n_cond, n_image, row_len;
+  int32_t recent_w, local_w, period, group_at;
+  int32_t global_budget;
+  int32_t reserved;
+  double tau, r_s;
+} hkv_config;
+
+/*
+ * A KV cache: one arena holding every head's segment back to back.
+ * Segment i spans tokens [off[i], off[i] + cap[i]) of the arena; its first
+ * len[i] tokens are live, oldest first: [conditioning | history | recent |
+ * buffered] (Eq. 2). All arrays are device memory owned by the caller.
+ *  k, v      arena, [capacity_tokens][head_dim] in the config dtype
+ *  pos       [capacity_tokens] int32: the original cache position of each
+ *            live token (conditioning j -> j, image token t -> C + t)
+ *  off       [L*S*H] int64 segment offsets (tokens)
+ *  cap       [L*S*H] int32 segment capacities (tokens)
+ *  len       [L*S*H] int32 live tokens
+ *  nbuf      [L*S*H] int32 tokens buffered since the last update
+ *  ntok      [L*S*H] int32 image tokens appended so far
+ *  label     [L*S*H] uint8 HKV_LOCAL / HKV_GLOBAL / HKV_DENSE
+ *  qbuf      [L*S*H][P][head_dim] ring of the P latest image-token queries
+ *            (Q_past of Eq. 6); image token t goes to slot t mod P
+ *  err       one uint32 error word (0 = none), first error wins
+ *  capacity_tokens  arena size in tokens (host value), used for checks
+ */
+typedef struct {
+  void *k;
+  void *v;
+  int32_t *pos;
+  int64_t *off;
+  int32_t *cap;
+  int32_t *len;
+  int32_t *nbuf;
+  int32_t *ntok;
+  uint8_t *label;
+  void *qbuf;
+  uint32_t *err;
+  int64_t capacity_tokens;
+} hkv_cache;
+
+/* Human-readable name of a status code (static string). */
+const char *hkv_status_str(hkv_status s);
+
+/* Checks a config: sizes positive, head_dim in {64, 128}, dtype known,
+ * recent_w <= global_budget <= n_image, period <= group_at <= n_image,
+ * 0 < tau <= 1, 0 <= r_s <= 1. Host only. */
+hkv_status hkv_validate_config(const hkv_config *cfg);
+
+/* Bytes of device workspace hkv_decode_attention needs for this config
+ * (split-K partial results and per-head arrival counters). The workspace
+ * must be zero-filled before its first use; every call leaves its counters
+ * at zero again. Concurrent calls must not share a workspace. Host only. */
+size_t hkv_workspace_size(const hkv_config *cfg);
+
+/* Sets up the uncompressed cache of Step 1 (cache prefilling): every head
+ * gets a segment of cap = C + E tokens at off = i * (C + E), len = nbuf =
+ * ntok = 0, label = HKV_DENSE, and the error word is cleared. The arena
+ * must hold L*S*H*(C+E) tokens. */
+hkv_status hkv_init_dense(const hkv_config *cfg, const hkv_cache *cache, hkv_stream_t stream);
+
+/* Step 1: writes the C conditioning tokens of one layer (kc, vc:
+ * [S][H][C][head_dim]) at the start of every head's segment and sets
+ * len = C. Only for an HKV_DENSE cache of a fresh layer. */
+hkv_status hkv_prefill(const hkv_config *cfg, const hkv_cache *cache, int layer,
+                       const void *kc, const void *vc, hkv_stream_t stream);
+
+/* One decode step of one layer, before its attention (KV cache update,
+ * Sec. 3; periodic update, Sec. 4):
+ *  1. for a compressed head whose buffer holds P tokens, run the update
+ *     first: a local head keeps its conditioning and newest w tokens
+ *     (Eq. 3); a global head whose history exceeds B_g - w evicts the excess
+ *     by STE (Eqs. 4-6: long/near split by r_s, scores from the P buffered
+ *     queries, the lowest floor(M/2) / M - floor(M/2) of each subset
+ *     evicted, older first on equal score) and compacts K, V and pos in
+ *     place (survivors keep their order);
+ *  2. append k, v of the new image token at the tail (pos = C + ntok), push
+ *     q into the Q_past ring, len += 1.
+ * q, k, v: [S][H][head_dim]. A full segment sets HKV_ERR_CAPACITY in the
+ * error word and leaves that head unchanged. */
+hkv_status hkv_append_evict(const hkv_config *cfg, const hkv_cache *cache, int layer,
+                            const void *q, const void *k, const void *v, hkv_stream_t stream);
+
+/* Eq. 1 for one new query per head over that head's live tokens (any mix
+ * of lengths): out[s][h][:] = softmax(q k^T / sqrt(d)) V, fp32 accumulation,
+ * written in fp32 ([S][H][head_dim]). Split-K over the layer's total token
+ * count with a per-head combine; workspace of hkv_workspace_size bytes.
+ * A head with len = 0 yields zeros. */
+hkv_status hkv_decode_attention(const hkv_config *cfg, const hkv_cache *cache, int layer,
+                                const void *q, float *out, void *workspace, size_t ws_bytes,
+                                hkv_stream_t stream);
+
+/* Sec. 4, Step 2 for one layer of an HKV_DENSE cache: for each head, the
+ * attention of q over the live keys is accumulated backward from the newest
+ * token until tau is reached; n_h is the number of tokens needed and the
+ * head is HKV_LOCAL iff n_h < w_loc. Writes label_out[i] and, if non-null,
+ * nh_out[i] for the layer's heads (i = flat head index; both arrays are
+ * [L*S*H]). */
+hkv_status hkv_identify_heads(const hkv_config *cfg, const hkv_cache *cache, int layer,
+                              const void *q, uint8_t *label_out, int32_t *nh_out,
+                              hkv_stream_t stream);
+
+/* Sec. 5.1 budgets for all L*S*H heads from their labels: budget = B_g
+ * (global) or w (local) image tokens, cap = C + budget + P, off = exclusive
+ * prefix sum of cap (tokens). Writes budget, cap, off (device) and the
+ * arena size in tokens to *total_tokens (host); synchronises the stream.
+ * A label other than HKV_LOCAL / HKV_GLOBAL yields HKV_ERR_STATE. */
+hkv_status hkv_allocate_budgets(const hkv_config *cfg, const uint8_t *label, int32_t *budget,
+                                int32_t *cap, int64_t *off, int64_t *total_tokens,
+                                hkv_stream_t stream);
+
+/* Head-aware compression of one layer after grouping (Step 3): copies
+ * every head of the dense cache into its segment of the ragged cache (whose
+ * off, cap and label arrays the caller filled from hkv_allocate_budgets and
+ * hkv_identify_heads) and applies the first update there: local heads keep
+ * the conditioning and newest w tokens; global heads keep a history of at
+ * most B_g - w tokens chosen by STE with the P latest queries. Sets len,
+ * nbuf = 0 and ntok on the ragged side. The two caches share the qbuf ring
+ * layout; the ragged cache's qbuf must be the dense cache's qbuf. */
+hkv_status hkv_repack(const hkv_config *cfg, const hkv_cache *dense, const hkv_cache *ragged,
+                      int layer, hkv_stream_t stream);
+
+/* Synchronises the stream and returns the status recorded in the cache's
+ * error word (HKV_OK if none), or HKV_ERR_CUDA if the stream failed. */
+hkv_status hkv_check(const hkv_cache *cache, hkv_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HKV_H */

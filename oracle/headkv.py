@@ -268,23 +268,25 @@ class HeadTrace:
     n_h: int = -1
     margin: float = float("nan")
     outputs: dict = field(default_factory=dict)   # t -> o_t (fp64 [D])
+    pos_at: dict = field(default_factory=dict)    # t -> positions attended at step t
     updates: list = field(default_factory=list)   # UpdateRecord per update
     final_pos: np.ndarray | None = None
     nbuf: int = 0
 
 
 def run_head(hp: HeadParams, q, k, v, *, label: int | None = None, record=(),
-             stop_after: int | None = None, scores: str = "fp32") -> HeadTrace:
+             record_pos=(), stop_after: int | None = None, scores: str = "fp32") -> HeadTrace:
     """Generate image tokens 0..N-1 for one head (Steps 1-3).
 
     q [N, d] holds the image-token queries; k, v [C+N, d] the keys and values
     indexed by cache position. `label` overrides the grouping result (used to
     continue from the label the device chose on a declared near-tie). The
-    attention output is kept for the steps in `record`. `stop_after` ends the
-    run after that image token's attention.
+    attention output is kept for the steps in `record`, the positions the
+    attention saw for those in `record_pos`. `stop_after` ends the run after
+    that image token's attention.
     """
     C, N, P, E = hp.n_cond, hp.n_image, hp.period, hp.group_at
-    record = set(record)
+    record, record_pos = set(record), set(record_pos)
     tr = HeadTrace()
     pos = np.arange(C, dtype=np.int64)       # Step 1: cache of the condition
     compressed = False
@@ -300,6 +302,8 @@ def run_head(hp: HeadParams, q, k, v, *, label: int | None = None, record=(),
             nbuf += 1
         if t in record:
             tr.outputs[t] = attention(q[t], k[pos], v[pos])
+        if t in record_pos:
+            tr.pos_at[t] = pos.copy()
         if t == E - 1:                        # Step 2: head grouping
             n_h, cum = grouping_count(q[t], k[pos], hp.tau)
             tr.n_h = n_h

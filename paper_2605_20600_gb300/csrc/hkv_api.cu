@@ -1,0 +1,340 @@
+// Host side of the HeadKV C-ABI (include/hkv.h): argument validation, fault
+// injection for tests, per-device launch setup, and the kernel launches.
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <mutex>
+
+#include "hkv.h"
+#include "hkv_kernels.h"
+
+namespace {
+
+using namespace hkv;
+
+constexpr int kMaxDevices = 64;
+constexpr size_t kMaxSmem = 227 * 1024;
+
+struct DeviceState {
+  bool init = false;
+  int sms = 0;
+  int attn_ctas[2][2] = {{0, 0}, {0, 0}};   // [dtype][D == 128]
+  size_t update_smem[2][2] = {{0, 0}, {0, 0}};
+};
+
+DeviceState g_dev[kMaxDevices];
+std::mutex g_mu;
+
+hkv_status injected(const char *name) {
+  const char *s = getenv("HKV_FAULT_INJECT");
+  if (!s) return HKV_OK;
+  const size_t n = strlen(name);
+  if (strncmp(s, name, n) == 0 && s[n] == ':') return (hkv_status)atoi(s + n + 1);
+  return HKV_OK;
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int dt_index(int dtype) { return dtype == HKV_BF16 ? 1 : 0; }
+int d_index(int D) { return D == 128 ? 1 : 0; }
+
+hkv_status cuda_status(cudaError_t e) { return e == cudaSuccess ? HKV_OK : HKV_ERR_CUDA; }
+
+// Per-device, per-(D, dtype) launch setup (shared memory limits, occupancy);
+// done on the first call that needs it, outside any stream capture.
+hkv_status device_state(DeviceState **out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return HKV_ERR_CUDA;
+  DeviceState &st = g_dev[dev];
+  if (!st.init) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (!st.init) {
+      if (cudaDeviceGetAttribute(&st.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return HKV_ERR_CUDA;
+      st.init = true;
+    }
+  }
+  *out = &st;
+  return HKV_OK;
+}
+
+hkv_status attention_ctas(DeviceState *st, int D, int dtype, int *ctas) {
+  int &c = st->attn_ctas[dt_index(dtype)][d_index(D)];
+  if (c == 0) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (c == 0) {
+      int n = 0;
+      if (attention_prepare(D, dtype, &n) != cudaSuccess || n <= 0) return HKV_ERR_CUDA;
+      c = n;
+    }
+  }
+  *ctas = c;
+  return HKV_OK;
+}
+
+hkv_status update_ready(DeviceState *st, int D, int dtype, size_t smem) {
+  size_t &have = st->update_smem[dt_index(dtype)][d_index(D)];
+  if (smem > kMaxSmem) return HKV_ERR_CAPACITY;
+  if (have < smem) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (have < smem) {
+      if (update_prepare(D, dtype, smem) != cudaSuccess) return HKV_ERR_CUDA;
+      have = smem;
+    }
+  }
+  return HKV_OK;
+}
+
+hkv_status check_cache(const hkv_cache *c) {
+  if (!c || !c->k || !c->v || !c->pos || !c->off || !c->cap || !c->len || !c->nbuf || !c->ntok ||
+      !c->label || !c->qbuf || !c->err)
+    return HKV_ERR_INVALID_ARG;
+  if (!aligned16(c->k) || !aligned16(c->v) || !aligned16(c->qbuf)) return HKV_ERR_ALIGN;
+  if (c->capacity_tokens <= 0) return HKV_ERR_CAPACITY;
+  return HKV_OK;
+}
+
+CacheArgs cache_args(const hkv_cache *c) {
+  CacheArgs a;
+  a.K = c->k;
+  a.V = c->v;
+  a.pos = c->pos;
+  a.off = c->off;
+  a.cap = c->cap;
+  a.len = c->len;
+  a.nbuf = c->nbuf;
+  a.ntok = c->ntok;
+  a.label = c->label;
+  a.qbuf = c->qbuf;
+  a.err = c->err;
+  a.arena_tokens = c->capacity_tokens;
+  return a;
+}
+
+MethodArgs method_args(const hkv_config *cfg) {
+  MethodArgs m;
+  m.C = cfg->n_cond;
+  m.w = cfg->recent_w;
+  m.w_loc = cfg->local_w;
+  m.P = cfg->period;
+  m.hist_budget = cfg->global_budget - cfg->recent_w;
+  m.r_s = cfg->r_s;
+  m.tau = (float)cfg->tau;
+  return m;
+}
+
+int heads_per_layer(const hkv_config *c) { return c->n_seqs * c->n_heads; }
+
+// longest segment any call may see: a dense head (C + E) or a compressed
+// global head right before its update (C + B_g + P)
+int max_segment(const hkv_config *c) {
+  const int a = c->n_cond + c->group_at;
+  const int b = c->n_cond + c->global_budget + c->period;
+  return a > b ? a : b;
+}
+
+size_t part_bytes(const hkv_config *c) {
+  const size_t b = (size_t)kAttnMaxGrid * 2 * (size_t)(c->head_dim + 2) * sizeof(float);
+  return (b + 255) & ~(size_t)255;
+}
+
+#define HKV_TRY(x)                 \
+  do {                             \
+    hkv_status s_ = (x);           \
+    if (s_ != HKV_OK) return s_;   \
+  } while (0)
+
+}  // namespace
+
+extern "C" {
+
+const char *hkv_status_str(hkv_status s) {
+  switch (s) {
+    case HKV_OK: return "ok";
+    case HKV_ERR_INVALID_ARG: return "invalid argument";
+    case HKV_ERR_SHAPE: return "unsupported shape";
+    case HKV_ERR_CAPACITY: return "capacity exceeded";
+    case HKV_ERR_STATE: return "cache in the wrong state";
+    case HKV_ERR_BOUNDS: return "segment outside the arena";
+    case HKV_ERR_TIMEOUT: return "device wait timed out";
+    case HKV_ERR_CUDA: return "CUDA error";
+    case HKV_ERR_ALIGN: return "pointer not 16-byte aligned";
+  }
+  return "unknown status";
+}
+
+hkv_status hkv_validate_config(const hkv_config *c) {
+  HKV_TRY(injected("validate_config"));
+  if (!c) return HKV_ERR_INVALID_ARG;
+  if (c->dtype != HKV_FP32 && c->dtype != HKV_BF16) return HKV_ERR_INVALID_ARG;
+  if (c->head_dim != 64 && c->head_dim != 128) return HKV_ERR_SHAPE;
+  if (c->n_layers <= 0 || c->n_seqs <= 0 || c->n_heads <= 0 || c->n_cond < 0 ||
+      c->n_image <= 0 || c->row_len <= 0 || c->recent_w <= 0 || c->local_w <= 0 ||
+      c->period <= 0 || c->group_at <= 0)
+    return HKV_ERR_SHAPE;
+  if (c->period > c->group_at || c->group_at > c->n_image) return HKV_ERR_SHAPE;
+  if (c->global_budget < c->recent_w || c->global_budget > c->n_image) return HKV_ERR_SHAPE;
+  if ((long long)c->n_layers * c->n_seqs * c->n_heads > (1ll << 30)) return HKV_ERR_SHAPE;
+  if ((long long)c->n_cond + c->n_image + c->period > (1ll << 24)) return HKV_ERR_SHAPE;
+  if (!(c->tau > 0.0 && c->tau <= 1.0) || !(c->r_s >= 0.0 && c->r_s <= 1.0))
+    return HKV_ERR_INVALID_ARG;
+  return HKV_OK;
+}
+
+size_t hkv_workspace_size(const hkv_config *c) {
+  if (!c || hkv_validate_config(c) != HKV_OK) return 0;
+  return part_bytes(c) + (size_t)heads_per_layer(c) * sizeof(int32_t);
+}
+
+hkv_status hkv_init_dense(const hkv_config *cfg, const hkv_cache *cache, hkv_stream_t stream) {
+  HKV_TRY(injected("init_dense"));
+  HKV_TRY(hkv_validate_config(cfg));
+  HKV_TRY(check_cache(cache));
+  const int seg = cfg->n_cond + cfg->group_at;
+  const long long n = (long long)cfg->n_layers * heads_per_layer(cfg);
+  if (cache->capacity_tokens < n * seg) return HKV_ERR_CAPACITY;
+  return cuda_status(launch_init_dense(cache_args(cache), (int)n, seg, (cudaStream_t)stream));
+}
+
+hkv_status hkv_prefill(const hkv_config *cfg, const hkv_cache *cache, int layer, const void *kc,
+                       const void *vc, hkv_stream_t stream) {
+  HKV_TRY(injected("prefill"));
+  HKV_TRY(hkv_validate_config(cfg));
+  HKV_TRY(check_cache(cache));
+  if (layer < 0 || layer >= cfg->n_layers) return HKV_ERR_INVALID_ARG;
+  if (cfg->n_cond > 0 && (!kc || !vc)) return HKV_ERR_INVALID_ARG;
+  if (cfg->n_cond > 0 && (!aligned16(kc) || !aligned16(vc))) return HKV_ERR_ALIGN;
+  const int hpl = heads_per_layer(cfg);
+  return cuda_status(launch_prefill(cache_args(cache), layer * hpl, hpl, cfg->n_cond, kc, vc,
+                                    cfg->head_dim, cfg->dtype, (cudaStream_t)stream));
+}
+
+hkv_status hkv_append_evict(const hkv_config *cfg, const hkv_cache *cache, int layer,
+                            const void *q, const void *k, const void *v, hkv_stream_t stream) {
+  HKV_TRY(injected("append_evict"));
+  HKV_TRY(hkv_validate_config(cfg));
+  HKV_TRY(check_cache(cache));
+  if (layer < 0 || layer >= cfg->n_layers) return HKV_ERR_INVALID_ARG;
+  if (!q || !k || !v) return HKV_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v)) return HKV_ERR_ALIGN;
+  DeviceState *st;
+  HKV_TRY(device_state(&st));
+  const size_t smem = update_smem_bytes(max_segment(cfg), cfg->head_dim);
+  HKV_TRY(update_ready(st, cfg->head_dim, cfg->dtype, smem));
+  const int hpl = heads_per_layer(cfg);
+  return cuda_status(launch_append_evict(cache_args(cache), method_args(cfg), layer * hpl, hpl, q,
+                                         k, v, cfg->head_dim, cfg->dtype, smem,
+                                         (cudaStream_t)stream));
+}
+
+hkv_status hkv_decode_attention(const hkv_config *cfg, const hkv_cache *cache, int layer,
+                                const void *q, float *out, void *workspace, size_t ws_bytes,
+                                hkv_stream_t stream) {
+  HKV_TRY(injected("decode_attention"));
+  HKV_TRY(hkv_validate_config(cfg));
+  HKV_TRY(check_cache(cache));
+  if (layer < 0 || layer >= cfg->n_layers) return HKV_ERR_INVALID_ARG;
+  if (!q || !out || !workspace) return HKV_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(out) || !aligned16(workspace)) return HKV_ERR_ALIGN;
+  if (ws_bytes < hkv_workspace_size(cfg)) return HKV_ERR_CAPACITY;
+  DeviceState *st;
+  HKV_TRY(device_state(&st));
+  int ctas = 0;
+  HKV_TRY(attention_ctas(st, cfg->head_dim, cfg->dtype, &ctas));
+  int grid = st->sms * ctas;
+  if (grid > kAttnMaxGrid) grid = kAttnMaxGrid;
+  const int hpl = heads_per_layer(cfg);
+  AttnArgs a;
+  a.K = cache->k;
+  a.V = cache->v;
+  a.off = cache->off + (size_t)layer * hpl;
+  a.len = cache->len + (size_t)layer * hpl;
+  a.q = q;
+  a.out = out;
+  a.part = static_cast<float *>(workspace);
+  a.cnt = reinterpret_cast<int32_t *>(static_cast<unsigned char *>(workspace) + part_bytes(cfg));
+  a.err = cache->err;
+  a.arena_tokens = cache->capacity_tokens;
+  a.nheads = hpl;
+  a.qscale = (float)(1.4426950408889634 / sqrt((double)cfg->head_dim));
+  return cuda_status(
+      launch_attention(a, cfg->head_dim, cfg->dtype, grid, (cudaStream_t)stream));
+}
+
+hkv_status hkv_identify_heads(const hkv_config *cfg, const hkv_cache *cache, int layer,
+                              const void *q, uint8_t *label_out, int32_t *nh_out,
+                              hkv_stream_t stream) {
+  HKV_TRY(injected("identify_heads"));
+  HKV_TRY(hkv_validate_config(cfg));
+  HKV_TRY(check_cache(cache));
+  if (layer < 0 || layer >= cfg->n_layers) return HKV_ERR_INVALID_ARG;
+  if (!q || !label_out) return HKV_ERR_INVALID_ARG;
+  if (!aligned16(q)) return HKV_ERR_ALIGN;
+  DeviceState *st;
+  HKV_TRY(device_state(&st));
+  const int max_len = cfg->n_cond + cfg->group_at;
+  HKV_TRY(update_ready(st, cfg->head_dim, cfg->dtype,
+                       update_smem_bytes(max_segment(cfg), cfg->head_dim)));
+  const int hpl = heads_per_layer(cfg);
+  return cuda_status(launch_identify(cache_args(cache), method_args(cfg), layer * hpl, hpl, q,
+                                     label_out, nh_out, cfg->head_dim, cfg->dtype, max_len,
+                                     (cudaStream_t)stream));
+}
+
+hkv_status hkv_allocate_budgets(const hkv_config *cfg, const uint8_t *label, int32_t *budget,
+                                int32_t *cap, int64_t *off, int64_t *total_tokens,
+                                hkv_stream_t stream) {
+  HKV_TRY(injected("allocate_budgets"));
+  HKV_TRY(hkv_validate_config(cfg));
+  if (!label || !budget || !cap || !off || !total_tokens) return HKV_ERR_INVALID_ARG;
+  const int n = cfg->n_layers * heads_per_layer(cfg);
+  cudaStream_t s = (cudaStream_t)stream;
+  if (launch_budgets(label, budget, cap, off, n, cfg->n_cond, cfg->global_budget, cfg->recent_w,
+                     cfg->period, s) != cudaSuccess)
+    return HKV_ERR_CUDA;
+  int64_t last_off = 0;
+  int32_t last_cap = 0;
+  if (cudaMemcpyAsync(&last_off, off + (n - 1), sizeof(last_off), cudaMemcpyDeviceToHost, s) !=
+          cudaSuccess ||
+      cudaMemcpyAsync(&last_cap, cap + (n - 1), sizeof(last_cap), cudaMemcpyDeviceToHost, s) !=
+          cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return HKV_ERR_CUDA;
+  if (last_off < 0) return HKV_ERR_STATE;
+  *total_tokens = last_off + last_cap;
+  return HKV_OK;
+}
+
+hkv_status hkv_repack(const hkv_config *cfg, const hkv_cache *dense, const hkv_cache *ragged,
+                      int layer, hkv_stream_t stream) {
+  HKV_TRY(injected("repack"));
+  HKV_TRY(hkv_validate_config(cfg));
+  HKV_TRY(check_cache(dense));
+  HKV_TRY(check_cache(ragged));
+  if (layer < 0 || layer >= cfg->n_layers) return HKV_ERR_INVALID_ARG;
+  if (dense->qbuf != ragged->qbuf) return HKV_ERR_INVALID_ARG;
+  DeviceState *st;
+  HKV_TRY(device_state(&st));
+  const size_t smem = update_smem_bytes(max_segment(cfg), cfg->head_dim);
+  HKV_TRY(update_ready(st, cfg->head_dim, cfg->dtype, smem));
+  const int hpl = heads_per_layer(cfg);
+  return cuda_status(launch_repack(cache_args(dense), cache_args(ragged), method_args(cfg),
+                                   layer * hpl, hpl, cfg->head_dim, cfg->dtype, smem,
+                                   (cudaStream_t)stream));
+}
+
+hkv_status hkv_check(const hkv_cache *cache, hkv_stream_t stream) {
+  HKV_TRY(injected("check"));
+  if (!cache || !cache->err) return HKV_ERR_INVALID_ARG;
+  cudaStream_t s = (cudaStream_t)stream;
+  uint32_t word = 0;
+  if (cudaMemcpyAsync(&word, cache->err, sizeof(word), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return HKV_ERR_CUDA;
+  return (hkv_status)word;
+}
+
+}  // extern "C"

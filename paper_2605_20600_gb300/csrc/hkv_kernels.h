@@ -1,0 +1,75 @@
+// Host-side launchers of the HeadKV kernels (internal to libheadkv.so).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "hkv.h"
+
+namespace hkv {
+
+// split-K decode attention over one layer of a ragged cache
+struct AttnArgs {
+  const void *K, *V;          // arena
+  const int64_t *off;         // layer slice of segment offsets
+  const int32_t *len;         // layer slice of live lengths
+  const void *q;              // [nheads][D]
+  float *out;                 // [nheads][D]
+  float *part;                // [grid][2][D + 2] partial results
+  int32_t *cnt;               // [nheads] arrival counters (zero between calls)
+  uint32_t *err;
+  int64_t arena_tokens;
+  int nheads;
+  float qscale;               // log2(e) / sqrt(D)
+};
+
+constexpr int kAttnThreads = 128;
+constexpr int kAttnMaxGrid = 4096;
+
+size_t attention_smem_bytes(int D, int dtype);
+cudaError_t attention_prepare(int D, int dtype, int *ctas_per_sm);
+cudaError_t launch_attention(const AttnArgs &a, int D, int dtype, int grid, cudaStream_t s);
+
+// per-head cache maintenance (append / update / repack / prefill / identify)
+struct CacheArgs {
+  void *K, *V;
+  int32_t *pos;
+  const int64_t *off;
+  const int32_t *cap;
+  int32_t *len, *nbuf, *ntok;
+  const uint8_t *label;
+  void *qbuf;
+  uint32_t *err;
+  int64_t arena_tokens;
+};
+
+struct MethodArgs {
+  int C, w, w_loc, P, hist_budget;  // hist_budget = B_g - w
+  double r_s;
+  float tau;
+};
+
+constexpr int kCacheThreads = 256;
+
+// dynamic shared memory of the update paths for segments of up to max_len tokens
+size_t update_smem_bytes(int max_len, int D);
+cudaError_t update_prepare(int D, int dtype, size_t smem);
+
+cudaError_t launch_append_evict(const CacheArgs &c, const MethodArgs &m, int layer_base,
+                                int nheads, const void *q, const void *k, const void *v, int D,
+                                int dtype, size_t smem, cudaStream_t s);
+cudaError_t launch_repack(const CacheArgs &dense, const CacheArgs &ragged, const MethodArgs &m,
+                          int layer_base, int nheads, int D, int dtype, size_t smem,
+                          cudaStream_t s);
+cudaError_t launch_prefill(const CacheArgs &c, int layer_base, int nheads, int C, const void *kc,
+                           const void *vc, int D, int dtype, cudaStream_t s);
+cudaError_t launch_init_dense(const CacheArgs &c, int nheads_total, int seg_tokens,
+                              cudaStream_t s);
+cudaError_t launch_identify(const CacheArgs &c, const MethodArgs &m, int layer_base, int nheads,
+                            const void *q, uint8_t *label_out, int32_t *nh_out, int D, int dtype,
+                            int max_len, cudaStream_t s);
+cudaError_t launch_budgets(const uint8_t *label, int32_t *budget, int32_t *cap, int64_t *off,
+                           int n, int C, int B_g, int w, int P, cudaStream_t s);
+
+}  // namespace hkv

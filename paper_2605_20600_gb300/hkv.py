@@ -1,0 +1,167 @@
+"""ctypes binding of the HeadKV C-ABI (include/hkv.h).
+
+Argument marshalling only: every function has the name of the C entry point
+it forwards to, accepts integers (device addresses) or objects with a
+`data_ptr()` method for pointer arguments, and raises HkvError on a status
+other than HKV_OK. There is no fallback: if libheadkv.so is missing the
+import of a function fails loudly.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+from ctypes import POINTER, Structure, c_char_p, c_double, c_int, c_int32, c_int64, c_size_t, c_void_p
+from fractions import Fraction
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libheadkv.so")
+
+HKV_OK = 0
+HKV_ERR_INVALID_ARG = 1
+HKV_ERR_SHAPE = 2
+HKV_ERR_CAPACITY = 3
+HKV_ERR_STATE = 4
+HKV_ERR_BOUNDS = 5
+HKV_ERR_TIMEOUT = 6
+HKV_ERR_CUDA = 7
+HKV_ERR_ALIGN = 8
+
+HKV_FP32, HKV_BF16 = 0, 1
+HKV_LOCAL, HKV_GLOBAL, HKV_DENSE = 0, 1, 255
+
+
+class hkv_config(Structure):
+    _fields_ = [
+        ("n_layers", c_int32), ("n_seqs", c_int32), ("n_heads", c_int32), ("head_dim", c_int32),
+        ("dtype", c_int32), ("n_cond", c_int32), ("n_image", c_int32), ("row_len", c_int32),
+        ("recent_w", c_int32), ("local_w", c_int32), ("period", c_int32), ("group_at", c_int32),
+        ("global_budget", c_int32), ("reserved", c_int32), ("tau", c_double), ("r_s", c_double),
+    ]
+
+
+class hkv_cache(Structure):
+    _fields_ = [
+        ("k", c_void_p), ("v", c_void_p), ("pos", c_void_p), ("off", c_void_p), ("cap", c_void_p),
+        ("len", c_void_p), ("nbuf", c_void_p), ("ntok", c_void_p), ("label", c_void_p),
+        ("qbuf", c_void_p), ("err", c_void_p), ("capacity_tokens", c_int64),
+    ]
+
+
+class HkvError(RuntimeError):
+    def __init__(self, name: str, status: int):
+        self.status = status
+        super().__init__(f"hkv_{name}: {hkv_status_str(status)} ({status})")
+
+
+_lib = None
+
+# (name, argtypes, restype)
+_SIGNATURES = {
+    "hkv_status_str": ([c_int], c_char_p),
+    "hkv_validate_config": ([POINTER(hkv_config)], c_int),
+    "hkv_workspace_size": ([POINTER(hkv_config)], c_size_t),
+    "hkv_init_dense": ([POINTER(hkv_config), POINTER(hkv_cache), c_void_p], c_int),
+    "hkv_prefill": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p, c_void_p, c_void_p], c_int),
+    "hkv_append_evict": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p, c_void_p, c_void_p,
+                          c_void_p], c_int),
+    "hkv_decode_attention": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p, c_void_p, c_void_p,
+                              c_size_t, c_void_p], c_int),
+    "hkv_identify_heads": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p, c_void_p, c_void_p,
+                            c_void_p], c_int),
+    "hkv_allocate_budgets": ([POINTER(hkv_config), c_void_p, c_void_p, c_void_p, c_void_p,
+                              POINTER(c_int64), c_void_p], c_int),
+    "hkv_repack": ([POINTER(hkv_config), POINTER(hkv_cache), POINTER(hkv_cache), c_int, c_void_p], c_int),
+    "hkv_check": ([POINTER(hkv_cache), c_void_p], c_int),
+}
+
+
+def lib():
+    """The loaded libheadkv.so (raises if it was not built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is missing: build it with __graft_entry__.build()")
+        l = ctypes.CDLL(LIB_PATH)
+        for name, (args, res) in _SIGNATURES.items():
+            f = getattr(l, name)
+            f.argtypes = args
+            f.restype = res
+        _lib = l
+    return _lib
+
+
+def _p(x) -> int | None:
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    return x.data_ptr()
+
+
+def _call(name: str, *args) -> None:
+    st = getattr(lib(), "hkv_" + name)(*args)
+    if st != HKV_OK:
+        raise HkvError(name, st)
+
+
+def hkv_status_str(status: int) -> str:
+    return lib().hkv_status_str(status).decode()
+
+
+def make_config(*, n_layers, n_seqs, n_heads, head_dim, dtype, n_cond, n_image, row_len,
+                recent_w, local_w, period, group_at, rho=None, global_budget=None,
+                tau=0.9, r_s=0.5) -> hkv_config:
+    """Builds an hkv_config; the global budget is floor(rho * N) (Sec. 5.1)
+    unless given explicitly."""
+    if global_budget is None:
+        global_budget = math.floor(Fraction(rho) * n_image)
+    return hkv_config(n_layers, n_seqs, n_heads, head_dim,
+                      HKV_BF16 if dtype in ("bf16", HKV_BF16) else HKV_FP32,
+                      n_cond, n_image, row_len, recent_w, local_w, period, group_at,
+                      int(global_budget), 0, float(tau), float(r_s))
+
+
+def hkv_validate_config(cfg: hkv_config) -> None:
+    _call("validate_config", ctypes.byref(cfg))
+
+
+def hkv_workspace_size(cfg: hkv_config) -> int:
+    return int(lib().hkv_workspace_size(ctypes.byref(cfg)))
+
+
+def hkv_init_dense(cfg, cache, stream=0) -> None:
+    _call("init_dense", ctypes.byref(cfg), ctypes.byref(cache), stream)
+
+
+def hkv_prefill(cfg, cache, layer, kc, vc, stream=0) -> None:
+    _call("prefill", ctypes.byref(cfg), ctypes.byref(cache), layer, _p(kc), _p(vc), stream)
+
+
+def hkv_append_evict(cfg, cache, layer, q, k, v, stream=0) -> None:
+    _call("append_evict", ctypes.byref(cfg), ctypes.byref(cache), layer, _p(q), _p(k), _p(v), stream)
+
+
+def hkv_decode_attention(cfg, cache, layer, q, out, workspace, ws_bytes, stream=0) -> None:
+    _call("decode_attention", ctypes.byref(cfg), ctypes.byref(cache), layer, _p(q), _p(out),
+          _p(workspace), ws_bytes, stream)
+
+
+def hkv_identify_heads(cfg, cache, layer, q, label_out, nh_out=None, stream=0) -> None:
+    _call("identify_heads", ctypes.byref(cfg), ctypes.byref(cache), layer, _p(q), _p(label_out),
+          _p(nh_out), stream)
+
+
+def hkv_allocate_budgets(cfg, label, budget, cap, off, stream=0) -> int:
+    total = c_int64(0)
+    _call("allocate_budgets", ctypes.byref(cfg), _p(label), _p(budget), _p(cap), _p(off),
+          ctypes.byref(total), stream)
+    return int(total.value)
+
+
+def hkv_repack(cfg, dense, ragged, layer, stream=0) -> None:
+    _call("repack", ctypes.byref(cfg), ctypes.byref(dense), ctypes.byref(ragged), layer, stream)
+
+
+def hkv_check(cache, stream=0) -> None:
+    _call("check", ctypes.byref(cache), stream)

@@ -1,0 +1,50 @@
+"""Drives one full image generation through the Engine (Sec. 4 Steps 1-3 and
+the decode loop), taking per-step inputs from a provider object with
+
+    provider.cond(kc, vc, layer, stream)                 # kc/vc [S][H][C][D]
+    provider.image(q, k, v, l0, nl, t0, nt, stream)     # [nt][nl][S][H][D]
+
+and handing each step's attention outputs to an optional callback.
+"""
+from __future__ import annotations
+
+import torch
+
+from .engine import Engine, torch_dtype
+
+
+def generate(engine: Engine, provider, *, last_step: int | None = None, on_step=None,
+             before_compress=None) -> None:
+    """Runs image tokens 0..last_step (default N-1) for every layer.
+
+    on_step(t, out) receives out [L][S][H][D] (fp32, device) after step t.
+    before_compress(engine) runs after grouping, before budgets and repack.
+    """
+    cfg = engine.cfg
+    L, S, H, D, C = cfg.n_layers, cfg.n_seqs, cfg.n_heads, cfg.head_dim, cfg.n_cond
+    E = cfg.group_at
+    dev, dt = engine.device, torch_dtype(cfg)
+    st = engine.stream()
+    if C > 0:
+        kc = torch.empty(S, H, C, D, dtype=dt, device=dev)
+        vc = torch.empty_like(kc)
+        for layer in range(L):
+            provider.cond(kc, vc, layer, st)
+            engine.prefill(layer, kc, vc)
+    q = torch.empty(L, S, H, D, dtype=dt, device=dev)
+    k, v = torch.empty_like(q), torch.empty_like(q)
+    out = torch.empty(L, S, H, D, dtype=torch.float32, device=dev)
+    last = cfg.n_image - 1 if last_step is None else last_step
+    for t in range(last + 1):
+        provider.image(q, k, v, 0, L, t, 1, st)
+        for layer in range(L):
+            engine.append(layer, q[layer], k[layer], v[layer])
+            engine.attend(layer, q[layer], out[layer])
+            if t == E - 1:
+                engine.identify(layer, q[layer])
+        if on_step is not None:
+            on_step(t, out)
+        if t == E - 1:
+            if before_compress is not None:
+                before_compress(engine)
+            engine.compress()

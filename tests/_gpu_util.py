@@ -1,0 +1,111 @@
+"""Helpers of the GPU parity tests: workload -> config, one generation through
+the C-ABI with snapshots, oracle runs of sampled heads in a spawn pool."""
+from __future__ import annotations
+
+import multiprocessing as mp
+import os
+
+import numpy as np
+
+from oracle import headkv as O
+from synth import configs, gen
+
+
+def cfg_of(H, w: configs.Workload):
+    return H.make_config(n_layers=w.n_layers, n_seqs=w.n_seqs, n_heads=w.n_heads,
+                         head_dim=w.head_dim, dtype=w.dtype, n_cond=w.n_cond, n_image=w.n_image,
+                         row_len=w.row_len, recent_w=w.recent_w, local_w=w.w_loc,
+                         period=w.period, group_at=w.group_at, rho=w.rho, tau=w.tau, r_s=w.r_s)
+
+
+def flat(w, s, l, h):
+    return (l * w.n_seqs + s) * w.n_heads + h
+
+
+def run_gpu(w, *, out_steps=(), pos_steps=(), pos_heads=(), last_step=None):
+    """One generation on the GPU. Returns outputs {t: [L,S,H,D] fp32},
+    positions {t: {flat head: positions}}, labels, n_h and the engine."""
+    import torch
+    from paper_2605_20600_gb300 import hkv as H
+    from paper_2605_20600_gb300.engine import Engine
+    from paper_2605_20600_gb300.runner import generate
+    from synth.gpu import DeviceSynth
+
+    eng = Engine(cfg_of(H, w), "cuda")
+    out_steps, pos_steps = set(out_steps), set(pos_steps)
+    outs, poss = {}, {}
+
+    def on_step(t, out):
+        if t in out_steps:
+            outs[t] = out.cpu().numpy()
+        if t in pos_steps:
+            c = eng.cache
+            off, ln = c.off.cpu().numpy(), c.len.cpu().numpy()
+            allpos = c.pos
+            poss[t] = {i: allpos[int(off[i]): int(off[i]) + int(ln[i])].cpu().numpy()
+                       for i in pos_heads}
+
+    generate(eng, DeviceSynth(w, "cuda"), on_step=on_step, last_step=last_step)
+    torch.cuda.synchronize()
+    eng.check()
+    return outs, poss, eng.labels.cpu().numpy(), eng.n_h.cpu().numpy(), eng
+
+
+def _oracle_job(args):
+    w, s, l, h, label, record, record_pos = args
+    pe, cq = gen.pe_table(w), gen.q_coef(w)
+    hi = gen.HeadInputs(w, s, l, h, pe, cq)
+    hp = O.HeadParams.of(w)
+    tr = O.run_head(hp, hi.q, hi.k, hi.v, label=label, record=record, record_pos=record_pos)
+    return (s, l, h), tr
+
+
+def oracle_heads(w, heads, labels=None, record=(), record_pos=()):
+    """Oracle traces of the given (s, l, h) heads; labels (flat array) are
+    injected when given. Runs in a spawn pool (safe after CUDA init)."""
+    jobs = [(w, s, l, h, None if labels is None else int(labels[flat(w, s, l, h)]),
+             tuple(record), tuple(record_pos)) for (s, l, h) in heads]
+    if len(jobs) <= 2:
+        return dict(map(_oracle_job, jobs))
+    n = min(len(jobs), os.cpu_count() or 1, 16)
+    with mp.get_context("spawn").Pool(n) as pool:
+        return dict(pool.map(_oracle_job, jobs, chunksize=1))
+
+
+def label_job(args):
+    """Oracle grouping for heads of one (s, l): (label, n_h, margin) per head."""
+    w, s, l, heads = args
+    pe, cq = gen.pe_table(w), gen.q_coef(w)
+    hp = O.HeadParams.of(w)
+    res = []
+    for h in heads:
+        hi = gen.HeadInputs(w, s, l, h, pe, cq)
+        t = w.group_at - 1
+        K = hi.k[: w.n_cond + t + 1]
+        n_h, cum = O.grouping_count(hi.q[t], K, w.tau)
+        res.append((O.classify(n_h, w.w_loc), n_h, O.label_margin(cum, w.tau, w.w_loc)))
+    return (s, l), res
+
+
+def oracle_labels(w, layers, seqs):
+    jobs = [(w, s, l, tuple(range(w.n_heads))) for l in layers for s in seqs]
+    n = min(len(jobs), os.cpu_count() or 1, 16)
+    with mp.get_context("spawn").Pool(n) as pool:
+        return dict(pool.map(label_job, jobs, chunksize=1))
+
+
+LABEL_TIE = 1e-4   # |fp64 mass of the newest w_loc-1 tokens - tau| below this: either label
+
+
+def check_labels(w, gpu_labels, gpu_nh, oracle_lab, where):
+    """Bit-exact labels except declared near-ties; returns the tied heads."""
+    ties = []
+    for (s, l), res in oracle_lab.items():
+        for h, (lab, n_h, margin) in enumerate(res):
+            i = flat(w, s, l, h)
+            if int(gpu_labels[i]) != lab:
+                assert margin < LABEL_TIE, (where, s, l, h, lab, int(gpu_labels[i]), margin)
+                ties.append((s, l, h, margin))
+            elif margin >= LABEL_TIE:
+                assert int(gpu_nh[i]) == n_h or abs(n_h - int(gpu_nh[i])) <= 1, (where, s, l, h)
+    return ties

@@ -1,0 +1,155 @@
+"""The C-ABI library without a GPU: it loads, exports every entry point the
+header declares, and its host-side validation and fault injection answer
+before any CUDA call."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from conftest import ROOT
+
+HEADER = os.path.join(ROOT, "include", "hkv.h")
+
+
+@pytest.fixture(scope="module")
+def H():
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2605_20600_gb300 import hkv
+    hkv.lib()
+    return hkv
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(hkv_[a-z_]+)\s*\(", text)))
+
+
+def tiny_cfg(H, **kw):
+    base = dict(n_layers=2, n_seqs=2, n_heads=4, head_dim=64, dtype="bf16", n_cond=8, n_image=64,
+                row_len=8, recent_w=16, local_w=16, period=8, group_at=16, global_budget=24)
+    base.update(kw)
+    return H.make_config(**base)
+
+
+def fake_cache(H, **kw):
+    # aligned, non-null host addresses: never dereferenced by the checks tested here
+    buf = ctypes.create_string_buffer(4096)
+    a = (ctypes.addressof(buf) + 255) & ~255
+    c = H.hkv_cache(a, a + 256, a, a, a, a, a, a, a, a + 512, a, 1000)
+    for k, v in kw.items():
+        setattr(c, k, v)
+    c._keep = buf
+    return c
+
+
+def test_every_declared_symbol_is_exported(H):
+    names = declared_functions()
+    assert len(names) == 11
+    for n in names:
+        assert hasattr(H.lib(), n), n
+    assert set(names) >= {"hkv_identify_heads", "hkv_allocate_budgets", "hkv_append_evict",
+                          "hkv_decode_attention"}
+
+
+def test_struct_sizes(H):
+    assert ctypes.sizeof(H.hkv_config) == 14 * 4 + 2 * 8
+    assert ctypes.sizeof(H.hkv_cache) == 11 * 8 + 8
+
+
+def test_status_strings(H):
+    assert H.hkv_status_str(0) == "ok"
+    assert "capacity" in H.hkv_status_str(3)
+    assert H.hkv_status_str(99) == "unknown status"
+
+
+@pytest.mark.parametrize("change,code", [
+    (dict(head_dim=96), 2), (dict(dtype=5), 1), (dict(period=32), 2), (dict(global_budget=8), 2),
+    (dict(global_budget=65), 2), (dict(group_at=65), 2), (dict(n_seqs=0), 2), (dict(tau=0.0), 1),
+    (dict(r_s=1.5), 1),
+])
+def test_validate_config_rejects(H, change, code):
+    cfg = tiny_cfg(H)
+    for k, v in change.items():
+        setattr(cfg, k, v)
+    with pytest.raises(H.HkvError) as e:
+        H.hkv_validate_config(cfg)
+    assert e.value.status == code
+
+
+def test_validate_config_accepts_paper_shapes(H):
+    from fractions import Fraction
+    from synth import configs
+    for w in configs.ALL.values():
+        cfg = H.make_config(n_layers=w.n_layers, n_seqs=w.n_seqs, n_heads=w.n_heads,
+                            head_dim=w.head_dim, dtype=w.dtype, n_cond=w.n_cond,
+                            n_image=w.n_image, row_len=w.row_len, recent_w=w.recent_w,
+                            local_w=w.w_loc, period=w.period, group_at=w.group_at, rho=w.rho)
+        H.hkv_validate_config(cfg)
+        assert H.hkv_workspace_size(cfg) > 0
+    assert H.make_config(**{**dict(n_layers=1, n_seqs=1, n_heads=1, head_dim=128, dtype="bf16",
+                                   n_cond=128, n_image=4160, row_len=65, recent_w=130,
+                                   local_w=130, period=65, group_at=500)},
+                         rho=Fraction(1, 6)).global_budget == 693
+
+
+def test_workspace_size_zero_for_bad_config(H):
+    assert H.hkv_workspace_size(tiny_cfg(H, head_dim=32)) == 0
+
+
+def test_null_and_misaligned_arguments(H):
+    cfg = tiny_cfg(H)
+    c = fake_cache(H)
+    lib = H.lib()
+    assert lib.hkv_decode_attention(ctypes.byref(cfg), None, 0, 16, 16, 16, 1 << 30, None) == 1
+    assert lib.hkv_decode_attention(ctypes.byref(cfg), ctypes.byref(c), 0, None, 16, 16, 1 << 30, None) == 1
+    assert lib.hkv_decode_attention(ctypes.byref(cfg), ctypes.byref(c), 0, 24, 16, 16, 1 << 30, None) == 8
+    assert lib.hkv_decode_attention(ctypes.byref(cfg), ctypes.byref(c), 2, 16, 16, 16, 1 << 30, None) == 1
+    assert lib.hkv_decode_attention(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, 16, 8, None) == 3
+    assert lib.hkv_append_evict(ctypes.byref(cfg), ctypes.byref(c), -1, 16, 16, 16, None) == 1
+    assert lib.hkv_append_evict(ctypes.byref(cfg), ctypes.byref(c), 0, 16, None, 16, None) == 1
+    bad = fake_cache(H, qbuf=c.qbuf + 8)
+    assert lib.hkv_append_evict(ctypes.byref(cfg), ctypes.byref(bad), 0, 16, 16, 16, None) == 8
+    nul = fake_cache(H, err=None)
+    assert lib.hkv_identify_heads(ctypes.byref(cfg), ctypes.byref(nul), 0, 16, 16, None, None) == 1
+    small = fake_cache(H, capacity_tokens=10)
+    assert lib.hkv_init_dense(ctypes.byref(cfg), ctypes.byref(small), None) == 3
+    other = fake_cache(H, qbuf=c.qbuf + 256)
+    assert lib.hkv_repack(ctypes.byref(cfg), ctypes.byref(c), ctypes.byref(other), 0, None) == 1
+    assert lib.hkv_allocate_budgets(ctypes.byref(cfg), None, 16, 16, 16, None, None) == 1
+    assert lib.hkv_check(None, None) == 1
+
+
+@pytest.mark.parametrize("name", ["decode_attention", "append_evict", "identify_heads",
+                                  "allocate_budgets", "repack", "prefill", "init_dense", "check"])
+def test_fault_injection_returns_the_code(H, name, monkeypatch):
+    cfg = tiny_cfg(H)
+    c = fake_cache(H)
+    monkeypatch.setenv("HKV_FAULT_INJECT", f"{name}:6")
+    lib = H.lib()
+    calls = {
+        "decode_attention": lambda: lib.hkv_decode_attention(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, 16, 1 << 30, None),
+        "append_evict": lambda: lib.hkv_append_evict(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, 16, None),
+        "identify_heads": lambda: lib.hkv_identify_heads(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, None, None),
+        "allocate_budgets": lambda: lib.hkv_allocate_budgets(ctypes.byref(cfg), 16, 16, 16, 16, None, None),
+        "repack": lambda: lib.hkv_repack(ctypes.byref(cfg), ctypes.byref(c), ctypes.byref(c), 0, None),
+        "prefill": lambda: lib.hkv_prefill(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, None),
+        "init_dense": lambda: lib.hkv_init_dense(ctypes.byref(cfg), ctypes.byref(c), None),
+        "check": lambda: lib.hkv_check(ctypes.byref(c), None),
+    }
+    assert calls[name]() == 6
+
+
+def test_fault_injection_raises_through_binding(H, monkeypatch):
+    c = fake_cache(H)
+    monkeypatch.setenv("HKV_FAULT_INJECT", "check:6")
+    with pytest.raises(H.HkvError) as e:
+        H.hkv_check(c)
+    assert e.value.status == 6 and "timed out" in str(e.value)
+
+
+def test_fault_injection_other_name_does_not_fire(H, monkeypatch):
+    monkeypatch.setenv("HKV_FAULT_INJECT", "repack:6")
+    H.hkv_validate_config(tiny_cfg(H))

@@ -1,0 +1,144 @@
+"""The whole decode path through the C-ABI against the oracle: identification,
+budgets, STE with in-place compaction, and decode attention, step by step.
+
+* the hand-worked 4x4 grid (labels, n_h, positions after every update);
+* Tiny, every step and every head (outputs within 1e-5, positions exact);
+* each model shape cut to 2 layers x 2 sequences, every head (positions
+  exact at every update, outputs within 2e-3 at sampled steps)."""
+import numpy as np
+import pytest
+
+from oracle import headkv as O
+from synth import configs, gen
+
+from _gpu_util import (LABEL_TIE, check_labels, flat, oracle_heads, oracle_labels, run_gpu)
+from _hand import load as load_hand
+
+pytestmark = pytest.mark.gpu
+
+TOL = {"fp32": 1e-5, "bf16": 2e-3}
+
+
+class HandProvider:
+    def __init__(self, heads, C, device):
+        import torch
+        self.torch = torch
+        self.q = torch.from_numpy(np.stack([h["q"] for h in heads], 1)).to(device)   # [N][H][D]
+        self.k = torch.from_numpy(np.stack([h["k"] for h in heads], 0)).to(device)   # [H][C+N][D]
+        self.v = torch.from_numpy(np.stack([h["v"] for h in heads], 0)).to(device)
+        self.C = C
+
+    def cond(self, kc, vc, layer, stream=0):
+        kc[0].copy_(self.k[:, : self.C])
+        vc[0].copy_(self.v[:, : self.C])
+
+    def image(self, q, k, v, l0, nl, t0, nt, stream=0):
+        for tt in range(nt):
+            t = t0 + tt
+            q[tt, 0, 0].copy_(self.q[t]) if q.dim() == 5 else q[0, 0].copy_(self.q[t])
+            k[0, 0].copy_(self.k[:, self.C + t])
+            v[0, 0].copy_(self.v[:, self.C + t])
+
+
+def test_hand_worked_grid_on_gpu():
+    import torch
+    from paper_2605_20600_gb300 import hkv as H
+    from paper_2605_20600_gb300.engine import Engine
+    from paper_2605_20600_gb300.runner import generate
+    case, heads = load_hand()
+    c = case["config"]
+    cfg = H.make_config(n_layers=1, n_seqs=1, n_heads=2, head_dim=c["head_dim"], dtype="fp32",
+                        n_cond=c["n_cond"], n_image=c["n_image"], row_len=c["row_len"],
+                        recent_w=c["recent_w"], local_w=c["local_w"], period=c["period"],
+                        group_at=c["group_at"], global_budget=c["global_budget"], tau=c["tau"],
+                        r_s=c["r_s"])
+    eng = Engine(cfg, "cuda")
+    pos_at, outs = {}, {}
+
+    def on_step(t, out):
+        cc = eng.cache
+        off, ln = cc.off.cpu().numpy(), cc.len.cpu().numpy()
+        pos_at[t] = [cc.pos[int(off[h]): int(off[h]) + int(ln[h])].cpu().numpy() for h in range(2)]
+        outs[t] = out.cpu().numpy()[0, 0]
+
+    generate(eng, HandProvider(heads, c["n_cond"], "cuda"), on_step=on_step)
+    eng.check()
+    labels, nh = eng.labels.cpu().numpy(), eng.n_h.cpu().numpy()
+    hp = O.HeadParams(n_cond=c["n_cond"], n_image=c["n_image"], recent_w=c["recent_w"],
+                      local_w=c["local_w"], period=c["period"], group_at=c["group_at"],
+                      global_budget=c["global_budget"], tau=c["tau"], r_s=c["r_s"])
+    for h, hd in enumerate(heads):
+        exp = hd["expected"]
+        assert int(labels[h]) == exp["label"] and int(nh[h]) == exp["n_h"], hd["name"]
+        # after the update that ran at the start of step t_last+1 the cache
+        # holds the survivors plus the new token t_last+1
+        for u in exp["updates"][1:]:
+            t = u["t_last"] + 1
+            assert not set(u["evicted"]) & set(pos_at[t][h].tolist()), (hd["name"], t)
+        final = np.concatenate([pos_at[c["n_image"] - 1][h]])
+        assert final.tolist() == exp["final_pos"], hd["name"]
+        tr = O.run_head(hp, hd["q"], hd["k"], hd["v"], record=range(c["n_image"]),
+                        record_pos=range(c["n_image"]))
+        for t in range(c["n_image"]):
+            assert np.array_equal(pos_at[t][h], tr.pos_at[t]), (hd["name"], t)
+            assert np.abs(outs[t][h] - tr.outputs[t]).max() < 1e-5, (hd["name"], t)
+
+
+def test_tiny_every_step_every_head():
+    w = configs.TINY
+    N = w.n_image
+    heads = [(0, 0, h) for h in range(w.n_heads)]
+    outs, poss, labels, nh, eng = run_gpu(w, out_steps=range(N), pos_steps=range(N),
+                                          pos_heads=[flat(w, *x) for x in heads])
+    lab = oracle_labels(w, [0], [0])
+    ties = check_labels(w, labels, nh, lab, "tiny")
+    assert not ties
+    assert labels.tolist() == [0, 0, 0, 0, 1, 1, 1, 1]
+    tr = oracle_heads(w, heads, labels, record=range(N), record_pos=range(N))
+    worst = 0.0
+    for (s, l, h) in heads:
+        t_r = tr[(s, l, h)]
+        i = flat(w, s, l, h)
+        for t in range(N):
+            assert np.array_equal(poss[t][i], t_r.pos_at[t]), (h, t)
+            worst = max(worst, float(np.abs(outs[t][l, s, h] - t_r.outputs[t]).max()))
+    assert worst <= TOL["fp32"], worst
+
+
+def sampled_steps(w, rng, extra=12):
+    E, P, N = w.group_at, w.period, w.n_image
+    s = {0, E - 2, E - 1, E, E + 1, N - 1}
+    s |= {t for t in range(E, N, P)} | {t for t in range(E + P - 1, N, P)}
+    s |= set(rng.integers(0, N, size=extra).tolist())
+    return sorted(x for x in s if 0 <= x < N)
+
+
+REDUCED = [("lumina768", "1/4"), ("lumina1024", "1/4"), ("lumina1024", "1/6"),
+           ("lumina1024", "1/8"), ("llamagen_xl", "1/6"), ("janus_pro_7b", "1/8")]
+
+
+@pytest.mark.parametrize("name,rho", REDUCED)
+def test_model_shapes_two_layers_two_seqs(name, rho):
+    from fractions import Fraction
+    w = configs.ALL[name].with_(n_layers=2, n_seqs=2, rho=Fraction(rho))
+    rng = np.random.default_rng(42)
+    steps = sampled_steps(w, rng)
+    heads = [(s, l, h) for l in range(w.n_layers) for s in range(w.n_seqs) for h in range(w.n_heads)]
+    outs, poss, labels, nh, eng = run_gpu(w, out_steps=steps, pos_steps=steps,
+                                          pos_heads=[flat(w, *x) for x in heads])
+    lab = oracle_labels(w, range(w.n_layers), range(w.n_seqs))
+    ties = check_labels(w, labels, nh, lab, name)
+    assert len(ties) <= 2, ties
+    g = float((labels == 1).mean())
+    assert 0.2 < g < 0.8, g                       # both head types present
+    tr = oracle_heads(w, heads, labels, record=steps, record_pos=steps)
+    worst = 0.0
+    for (s, l, h) in heads:
+        t_r, i = tr[(s, l, h)], flat(w, s, l, h)
+        for t in steps:
+            assert np.array_equal(poss[t][i], t_r.pos_at[t]), (name, s, l, h, t)
+            worst = max(worst, float(np.abs(outs[t][l, s, h] - t_r.outputs[t]).max()))
+        # retained budget after the last update
+        budget = O.global_budget(w.rho, w.n_image) if labels[i] == 1 else w.recent_w
+        assert poss[w.n_image - 1][i].size == w.n_cond + budget + t_r.nbuf
+    assert worst <= TOL[w.dtype], worst
