@@ -22,7 +22,7 @@ def lib():
         l = ctypes.CDLL(LIB_PATH)
         l.hkv_synth_image.argtypes = [c_void_p, c_void_p, c_void_p, c_int, c_void_p, c_void_p,
                                       c_uint64, c_int, c_int, c_int, c_int, c_int, c_int, c_int,
-                                      c_int, c_int, c_int, c_float, c_float, c_void_p]
+                                      c_int, c_int, c_int, c_int, c_float, c_float, c_void_p]
         l.hkv_synth_image.restype = c_int
         l.hkv_synth_cond.argtypes = [c_void_p, c_void_p, c_int, c_uint64, c_int, c_int, c_int,
                                      c_int, c_int, c_float, c_float, c_void_p]
@@ -46,8 +46,9 @@ class DeviceSynth:
         w = self.w
         st = lib().hkv_synth_image(q.data_ptr(), k.data_ptr(), v.data_ptr(), self.bf16,
                                    self.pe.data_ptr(), self.cq.data_ptr(), w.seed, w.n_seqs,
-                                   w.n_heads, w.head_dim, w.n_cond, w.row_len, w.n_layers, l0, nl,
-                                   t0, nt, float(gen.KS), float(gen.VS), stream)
+                                   w.n_heads, w.head_dim, w.n_cond, w.row_len, w.n_image,
+                                   w.n_layers, l0, nl, t0, nt, float(gen.KS), float(gen.VS),
+                                   stream)
         if st != 0:
             raise RuntimeError(f"hkv_synth_image failed ({st})")
 

@@ -88,12 +88,14 @@ int grid_for(size_t total) {
 
 }  // namespace
 
+// n_image: tokens of the embedding table (rows * row_len); t0 + nt must not
+// exceed it
 extern "C" int hkv_synth_image(void* q, void* k, void* v, int bf16, const float* pe,
                                const float* cq, unsigned long long seed, int S, int H, int D,
-                               int C, int row_len, int L, int l0, int nl, int t0, int nt,
-                               float ks, float vs, cudaStream_t stream) {
+                               int C, int row_len, int n_image, int L, int l0, int nl, int t0,
+                               int nt, float ks, float vs, cudaStream_t stream) {
   if (!q || !k || !v || !pe || !cq || S <= 0 || H <= 0 || D <= 0 || nl <= 0 || nt <= 0 ||
-      l0 < 0 || l0 + nl > L || t0 < 0 || row_len <= 0)
+      l0 < 0 || l0 + nl > L || t0 < 0 || row_len <= 0 || t0 + nt > n_image)
     return 1;
   const size_t total = (size_t)nt * nl * S * H * D;
   synth_image_kernel<<<grid_for(total), 256, 0, stream>>>(q, k, v, bf16, pe, cq, seed, S, H, D,
