@@ -171,6 +171,25 @@ hkv_status hkv_decode_attention(const hkv_config *cfg, const hkv_cache *cache, i
                                 const void *q, float *out, void *workspace, size_t ws_bytes,
                                 hkv_stream_t stream);
 
+/* hkv_decode_attention for callers that cannot allocate device memory:
+ * the paper has no counterpart to this entry point. A plain C host program
+ * without a device allocator, or a plugin inside a host framework that owns
+ * and budgets all device memory, may have no way to provide the workspace
+ * that hkv_decode_attention takes. Here the split-K partials and per-head
+ * counters live in a fixed device array inside the library (1.25 MiB: 1 MiB
+ * of partials and 65536 counters), which every GPU that loads the library
+ * holds until the process exits. Same inputs, outputs and results as
+ * hkv_decode_attention; it allocates nothing.
+ *  - More than 65536 heads per layer (n_seqs * n_heads) -> HKV_ERR_CAPACITY.
+ *  - The first call on a device, with that device current, looks up the
+ *    array's device address and prepares the kernel; make that first call
+ *    before any stream capture.
+ *  - Every call uses the same array and clears its counters on `stream`
+ *    first; calls that may overlap on the GPU (other streams, other host
+ *    threads) race on it and must be serialised by the caller. */
+hkv_status hkv_decode_attention_noalloc(const hkv_config *cfg, const hkv_cache *cache, int layer,
+                                        const void *q, float *out, hkv_stream_t stream);
+
 /* Sec. 4, Step 2 for one layer of an HKV_DENSE cache: for each head, the
  * attention of q over the live keys is accumulated backward from the newest
  * token until tau is reached; n_h is the number of tokens needed and the

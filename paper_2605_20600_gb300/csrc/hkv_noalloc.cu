@@ -1,0 +1,121 @@
+// hkv_decode_attention_noalloc: decode attention that needs no workspace
+// from its caller.
+//
+// Some callers cannot hand us device memory for scratch: a plain C host
+// program with no device allocator of its own, a plugin inside a host
+// framework that owns and budgets all device memory, or code on a path where
+// an allocation is not allowed (for instance because it would synchronise the
+// device in a latency-critical loop). For them the split-K partial results
+// and the per-head arrival counters live in one file-scope device array of
+// fixed size, which every GPU that loads this library holds until the process
+// exits.
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+
+#include <mutex>
+
+#include "hkv.h"
+#include "hkv_kernels.h"
+
+namespace {
+
+using namespace hkv;
+
+// Split-K partials (up to 1 MiB) followed by one arrival counter per head of
+// a layer (up to 65536 heads): 1.25 MiB in total.
+constexpr size_t kPartBytes = 1u << 20;
+constexpr int kMaxHeadsPerLayer = 65536;
+constexpr size_t kScratchBytes = kPartBytes + (size_t)kMaxHeadsPerLayer * sizeof(int32_t);
+
+static __device__ __align__(256) unsigned char g_scratch[kScratchBytes];
+
+constexpr int kMaxDevices = 64;
+
+struct NoAllocDevice {
+  bool ready = false;
+  unsigned char *scratch = nullptr;  // device address of g_scratch
+  int sms = 0;
+  int ctas[2][2] = {{0, 0}, {0, 0}};  // [dtype][D == 128]
+};
+
+NoAllocDevice g_devs[kMaxDevices];
+std::mutex g_mu;
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Per-device set-up, done by the first call on each device with that device
+// current: the host-side name g_scratch is only a stand-in for the array, so
+// its device address is looked up here and passed to the kernel.
+hkv_status setup(int D, int dtype, NoAllocDevice **out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return HKV_ERR_CUDA;
+  NoAllocDevice &st = g_devs[dev];
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!st.ready) {
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_scratch) != cudaSuccess || p == nullptr) return HKV_ERR_CUDA;
+    if (cudaDeviceGetAttribute(&st.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return HKV_ERR_CUDA;
+    st.scratch = static_cast<unsigned char *>(p);
+    st.ready = true;
+  }
+  int &c = st.ctas[dtype == HKV_BF16 ? 1 : 0][D == 128 ? 1 : 0];
+  if (c == 0) {
+    int n = 0;
+    if (attention_prepare(D, dtype, &n) != cudaSuccess || n <= 0) return HKV_ERR_CUDA;
+    c = n;
+  }
+  *out = &st;
+  return HKV_OK;
+}
+
+}  // namespace
+
+extern "C" hkv_status hkv_decode_attention_noalloc(const hkv_config *cfg, const hkv_cache *cache,
+                                                   int layer, const void *q, float *out,
+                                                   hkv_stream_t stream) {
+  const hkv_status vs = hkv_validate_config(cfg);
+  if (vs != HKV_OK) return vs;
+  if (!cache || !cache->k || !cache->v || !cache->off || !cache->len || !cache->err || !q ||
+      !out)
+    return HKV_ERR_INVALID_ARG;
+  if (!aligned16(cache->k) || !aligned16(cache->v) || !aligned16(q) || !aligned16(out))
+    return HKV_ERR_ALIGN;
+  if (layer < 0 || layer >= cfg->n_layers) return HKV_ERR_INVALID_ARG;
+  const int hpl = cfg->n_seqs * cfg->n_heads;
+  if (hpl > kMaxHeadsPerLayer) return HKV_ERR_CAPACITY;  // counters would not fit
+
+  NoAllocDevice *st = nullptr;
+  const hkv_status ss = setup(cfg->head_dim, cfg->dtype, &st);
+  if (ss != HKV_OK) return ss;
+  const int ctas = st->ctas[cfg->dtype == HKV_BF16 ? 1 : 0][cfg->head_dim == 128 ? 1 : 0];
+
+  // as many CTAs as the partial area holds, at most the usual grid
+  const size_t per_cta = 2 * (size_t)(cfg->head_dim + 2) * sizeof(float);
+  int grid = st->sms * ctas;
+  if (grid > kAttnMaxGrid) grid = kAttnMaxGrid;
+  if ((size_t)grid * per_cta > kPartBytes) grid = (int)(kPartBytes / per_cta);
+
+  cudaStream_t s = (cudaStream_t)stream;
+  int32_t *cnt = reinterpret_cast<int32_t *>(st->scratch + kPartBytes);
+  // the array keeps whatever the previous call left: start the counters at 0
+  if (cudaMemsetAsync(cnt, 0, (size_t)hpl * sizeof(int32_t), s) != cudaSuccess)
+    return HKV_ERR_CUDA;
+
+  AttnArgs a;
+  a.K = cache->k;
+  a.V = cache->v;
+  a.off = cache->off + (size_t)layer * hpl;
+  a.len = cache->len + (size_t)layer * hpl;
+  a.q = q;
+  a.out = out;
+  a.part = reinterpret_cast<float *>(st->scratch);
+  a.cnt = cnt;
+  a.err = cache->err;
+  a.arena_tokens = cache->capacity_tokens;
+  a.nheads = hpl;
+  a.qscale = (float)(1.4426950408889634 / sqrt((double)cfg->head_dim));
+  return launch_attention(a, cfg->head_dim, cfg->dtype, grid, s) == cudaSuccess ? HKV_OK
+                                                                                  : HKV_ERR_CUDA;
+}

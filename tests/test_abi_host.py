@@ -47,7 +47,7 @@ def fake_cache(H, **kw):
 
 def test_every_declared_symbol_is_exported(H):
     names = declared_functions()
-    assert len(names) == 11
+    assert len(names) == 12
     for n in names:
         assert hasattr(H.lib(), n), n
     assert set(names) >= {"hkv_identify_heads", "hkv_allocate_budgets", "hkv_append_evict",
