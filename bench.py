@@ -193,14 +193,6 @@ class ClockSampler:
                 "samples": len(rows)}
 
 
-def attn_bytes(cfg, lens):
-    """Algorithmic bytes of one decode-attention launch: every retained K and
-    V row once, the query row in, the fp32 output row out."""
-    es = 2 if cfg.dtype == 1 else 4
-    heads = cfg.n_seqs * cfg.n_heads
-    return int(lens.sum()) * cfg.head_dim * 2 * es + heads * cfg.head_dim * (es + 4)
-
-
 def run_ours(args):
     import numpy as np
     import torch
@@ -258,17 +250,30 @@ def run_ours(args):
     staging = torch.empty(3, P, L, S, Hh, D, dtype=dt, device=dev)
     out = torch.empty(P, L, S, Hh, D, dtype=torch.float32, device=dev)
 
-    def period_calls():
+    def period_calls(events=None):
+        # the period starts with the update of every layer (its buffer is full);
+        # events (instrumented copy only): [step_begin, step_end] per decode
+        # step, then [evict_begin, evict_end] per layer
         for p in range(P):
             for layer in range(L):
-                eng.append(layer, staging[0, p, layer], staging[1, p, layer], staging[2, p, layer])
-                eng.attend(layer, staging[0, p, layer], out[p, layer])
+                if p == 0:
+                    if events is not None:
+                        events[P * L + layer][0].record()
+                    eng.evict(layer)
+                    if events is not None:
+                        events[P * L + layer][1].record()
+                if events is not None:
+                    events[p * L + layer][0].record()
+                eng.step(layer, staging[0, p, layer], staging[1, p, layer], staging[2, p, layer],
+                         out[p, layer])
+                if events is not None:
+                    events[p * L + layer][1].record()
 
     graph = torch.cuda.CUDAGraph()
     with torch.cuda.graph(graph):
         period_calls()
     stream = torch.cuda.current_stream()
-    launches_per_step = P * L * 2
+    launches_per_step = P * L + L
 
     def barrier():
         if world > 1:
@@ -304,29 +309,38 @@ def run_ours(args):
     images = S / w.cfg_rows
     value = world * images * P * K / (ms / 1e3)
 
-    # dominant kernel: decode attention of every layer, back to back, at the
-    # cache state the window reached (read-only, so it can be replayed)
-    lens = eng.cache.len.cpu().numpy().reshape(L, S * Hh)
-    bytes_per_launch = statistics.mean(attn_bytes(cfg, lens[layer]) for layer in range(L))
-    q_last = staging[0, P - 1]
-    attn_graph = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(attn_graph):
-        for layer in range(L):
-            eng.attend(layer, q_last[layer], out[0, layer])
-    reps = 20
-    attn_graph.replay()
-    torch.cuda.synchronize()
-    a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    torch.cuda.nvtx.range_push("hkv_attn_only")
-    a0.record(stream)
-    for _ in range(reps):
-        attn_graph.replay()
-    a1.record(stream)
+    # dominant kernel: the fused decode step (append + attention). One more
+    # period is replayed from a copy of the graph with an event pair around
+    # every decode-step launch; bytes per launch follow from the lengths at
+    # the period boundary (old rows at step p = boundary length - P + p).
+    lens = eng.cache.len.cpu().numpy().reshape(L, S * Hh).astype(np.int64)
+    es = 2 if cfg.dtype == 1 else 4
+    per_launch = [int((lens[layer] - P + p).sum()) * D * 2 * es + S * Hh * D * (6 * es + 4)
+                  for p in range(P) for layer in range(L)]
+    bytes_per_launch = statistics.mean(per_launch)
+    events = [(torch.cuda.Event(enable_timing=True, external=True),
+               torch.cuda.Event(enable_timing=True, external=True)) for _ in range(P * L + L)]
+    igraph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(igraph):
+        period_calls(events)
+    c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    c0.record(stream)
+    staging.copy_(pool[j % n_pool], non_blocking=True)
+    c1.record(stream)
+    j += 1
+    torch.cuda.nvtx.range_push("hkv_instrumented")
+    igraph.replay()
     torch.cuda.nvtx.range_pop()
     torch.cuda.synchronize()
-    attn_ms = a0.elapsed_time(a1) / (reps * L)
+    eng.check()
+    step_us = [e0.elapsed_time(e1) * 1e3 for e0, e1 in events[:P * L]]
+    evict_us = [e0.elapsed_time(e1) * 1e3 for e0, e1 in events[P * L:]]
+    copy_us = c0.elapsed_time(c1) * 1e3
+    # average decode-step launch in the timed graph: the period's device time
+    # minus the updates and the input copy (timed above), per launch
+    attn_us = (ms * 1e3 / K - sum(evict_us) - copy_us) / (P * L)
     peak, peak_kind = load_peaks()
-    achieved = bytes_per_launch / (attn_ms / 1e3) / 1e9
+    achieved = bytes_per_launch / (attn_us / 1e6) / 1e9
 
     # e2e through the C-ABI with pinned host buffers
     host_in = torch.empty(staging.shape, dtype=dt, pin_memory=True)
@@ -359,8 +373,10 @@ def run_ours(args):
                        "parallelism": "replicas" if world > 1 else "single GPU"},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": None,
-                         "kernel": "attn_kernel (hkv_decode_attention)",
-                         "bytes_per_launch": bytes_per_launch, "launch_us": attn_ms * 1e3,
+                         "kernel": "attn_kernel<fused> (hkv_decode_step: append + attention)",
+                         "bytes_per_launch": bytes_per_launch, "launch_us": attn_us,
+                         "launch_us_isolated": statistics.mean(step_us),
+                         "evict_us_per_period": sum(evict_us), "copy_us_per_period": copy_us,
                          "peak_kind": peak_kind},
             "e2e": {"value": e2e_value, "unit": "image tokens/s",
                     "h2d_bytes_per_step": staging.numel() * staging.element_size(),

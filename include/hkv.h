@@ -55,6 +55,19 @@ typedef enum {
 
 enum { HKV_FP32 = 0, HKV_BF16 = 1 };
 
+/* flags of hkv_decode_step */
+enum {
+  /* The kernel launched just before this call on the same stream does not
+   * write this layer's cache (its K/V rows, off/cap/len, label, nbuf).
+   * The step then reads the layer's lengths and starts streaming old K/V
+   * rows while that kernel is still finishing (programmatic dependent
+   * launch), and waits for it only before touching q, k, v. True when the
+   * previous kernel is the decode step or attention of another layer, or
+   * any call of this library other than a decode step or append of the same
+   * layer (hkv_evict never lets the next kernel start early). */
+  HKV_STEP_PREFETCH = 1
+};
+
 /* head labels (Sec. 4, Step 2); DENSE marks heads of the uncompressed
  * prefill-phase cache (Step 1), which are never evicted from */
 enum { HKV_LOCAL = 0, HKV_GLOBAL = 1, HKV_DENSE = 255 };
@@ -89,8 +102,13 @@ typedef struct {
 /*
  * A KV cache: one arena holding every head's segment back to back.
  * Segment i spans tokens [off[i], off[i] + cap[i]) of the arena; its first
- * len[i] tokens are live, oldest first: [conditioning | history | recent |
- * buffered] (Eq. 2). All arrays are device memory owned by the caller.
+ * len[i] rows are live: the conditioning tokens, the history, the recent
+ * window and the buffered tokens of Eq. 2. Attention does not depend on row
+ * order, so the periodic update refills evicted rows with surviving rows
+ * from the end of the segment instead of shifting everything: rows are in
+ * position order only in an uncompressed (HKV_DENSE) cache and among the
+ * tokens appended since the last update; pos[] identifies every row.
+ * All arrays are device memory owned by the caller.
  *  k, v      arena, [capacity_tokens][head_dim] in the config dtype
  *  pos       [capacity_tokens] int32: the original cache position of each
  *            live token (conditioning j -> j, image token t -> C + t)
@@ -128,10 +146,12 @@ const char *hkv_status_str(hkv_status s);
  * 0 < tau <= 1, 0 <= r_s <= 1. Host only. */
 hkv_status hkv_validate_config(const hkv_config *cfg);
 
-/* Bytes of device workspace hkv_decode_attention needs for this config
- * (split-K partial results and per-head arrival counters). The workspace
- * must be zero-filled before its first use; every call leaves its counters
- * at zero again. Concurrent calls must not share a workspace. Host only. */
+/* Bytes of device workspace hkv_decode_attention and hkv_decode_step need
+ * for this config (split-K partial results, per-head and grid arrival
+ * counters). The workspace must be zero-filled before its first use; every
+ * call leaves its counters at zero again (after a call that reported an
+ * error, zero it again). Concurrent calls must not share a workspace.
+ * Host only. */
 size_t hkv_workspace_size(const hkv_config *cfg);
 
 /* Sets up the uncompressed cache of Step 1 (cache prefilling): every head
@@ -153,14 +173,38 @@ hkv_status hkv_prefill(const hkv_config *cfg, const hkv_cache *cache, int layer,
  *     (Eq. 3); a global head whose history exceeds B_g - w evicts the excess
  *     by STE (Eqs. 4-6: long/near split by r_s, scores from the P buffered
  *     queries, the lowest floor(M/2) / M - floor(M/2) of each subset
- *     evicted, older first on equal score) and compacts K, V and pos in
- *     place (survivors keep their order);
+ *     evicted, older first on equal score); the segment shrinks in place by
+ *     moving the surviving rows above the new length into the evicted rows
+ *     below it;
  *  2. append k, v of the new image token at the tail (pos = C + ntok), push
  *     q into the Q_past ring, len += 1.
  * q, k, v: [S][H][head_dim]. A full segment sets HKV_ERR_CAPACITY in the
  * error word and leaves that head unchanged. */
 hkv_status hkv_append_evict(const hkv_config *cfg, const hkv_cache *cache, int layer,
                             const void *q, const void *k, const void *v, hkv_stream_t stream);
+
+/* The periodic head-aware update alone (Sec. 4, Efficient Cache Update;
+ * Eqs. 3-6), for every head of the layer whose buffer holds P tokens: the
+ * same update hkv_append_evict runs before its append, without the append.
+ * Heads whose buffer is not full are left as they are, so the call is
+ * harmless when no update is due; with hkv_decode_step it must run before
+ * the step that follows the P-th buffered token. */
+hkv_status hkv_evict(const hkv_config *cfg, const hkv_cache *cache, int layer, hkv_stream_t stream);
+
+/* One decode step of one layer in a single launch: the append of the new
+ * token (Sec. 3, KV Cache) fused with the attention of Eq. 1 over the cache
+ * including that token. out[s][h][:] = softmax(q k^T / sqrt(d)) V over the
+ * head's len live tokens and the new one (whose K/V are read straight from
+ * k and v), fp32; then k, v join the arena at row len, q joins the Q_past
+ * ring, and len, ntok (and nbuf for compressed heads) advance by one.
+ * q, k, v: [S][H][head_dim] in the config dtype; workspace of
+ * hkv_workspace_size bytes. A compressed head whose buffer already holds P
+ * tokens (hkv_evict not run) sets HKV_ERR_STATE, a full segment
+ * HKV_ERR_CAPACITY, in the error word; the step is then not taken.
+ * flags: 0 or HKV_STEP_PREFETCH (see above). */
+hkv_status hkv_decode_step(const hkv_config *cfg, const hkv_cache *cache, int layer,
+                           const void *q, const void *k, const void *v, float *out,
+                           void *workspace, size_t ws_bytes, int flags, hkv_stream_t stream);
 
 /* Eq. 1 for one new query per head over that head's live tokens (any mix
  * of lengths): out[s][h][:] = softmax(q k^T / sqrt(d)) V, fp32 accumulation,
@@ -190,7 +234,8 @@ hkv_status hkv_decode_attention(const hkv_config *cfg, const hkv_cache *cache, i
 hkv_status hkv_decode_attention_noalloc(const hkv_config *cfg, const hkv_cache *cache, int layer,
                                         const void *q, float *out, hkv_stream_t stream);
 
-/* Sec. 4, Step 2 for one layer of an HKV_DENSE cache: for each head, the
+/* Sec. 4, Step 2 for one layer of an HKV_DENSE cache (heads of any other
+ * label set HKV_ERR_STATE in the error word): for each head, the
  * attention of q over the live keys is accumulated backward from the newest
  * token until tau is reached; n_h is the number of tokens needed and the
  * head is HKV_LOCAL iff n_h < w_loc. Writes label_out[i] and, if non-null,

@@ -53,25 +53,31 @@ def _stale(target, deps):
     return any(os.path.getmtime(d) > t for d in deps)
 
 
-def build(force: bool = False, extra_flags=()) -> None:
-    os.makedirs(BUILD, exist_ok=True)
+def build(force: bool = False, extra_flags=(), lib_path: str | None = None,
+          build_dir: str | None = None) -> None:
+    """Compiles the sources into lib_path (default: the package's
+    libheadkv.so, objects in _build/); extra_flags (e.g. -D tuning macros) go
+    to every nvcc call of the library."""
+    lib = lib_path or LIB
+    bdir = build_dir or (BUILD if lib_path is None else os.path.join(os.path.dirname(lib), "_build"))
+    os.makedirs(bdir, exist_ok=True)
     cc = nvcc()
     headers = [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".h", ".cuh"))]
     headers.append(os.path.join(ROOT, "include", "hkv.h"))
     objs, cmds = [], []
     for src in SOURCES:
         s = os.path.join(CSRC, src)
-        o = os.path.join(BUILD, src.replace(".cu", ".o"))
+        o = os.path.join(bdir, src.replace(".cu", ".o"))
         objs.append(o)
         if force or _stale(o, [s] + headers):
             cmds.append([cc, *ARCH, *FLAGS, *extra_flags, "-c", s, "-o", o])
     synth_cmd = None
-    if force or _stale(SYNTH_LIB, [SYNTH_SRC]):
+    if lib_path is None and (force or _stale(SYNTH_LIB, [SYNTH_SRC])):
         synth_cmd = [cc, *ARCH, "-O3", "-std=c++17", "-Xcompiler", "-fPIC", "-shared",
                      SYNTH_SRC, "-o", SYNTH_LIB]
     _run_all(cmds + ([synth_cmd] if synth_cmd else []))
-    if force or cmds or _stale(LIB, objs):
-        _run_all([[cc, *ARCH, "-shared", *objs, "-o", LIB]])
+    if force or cmds or _stale(lib, objs):
+        _run_all([[cc, *ARCH, "-shared", *objs, "-o", lib]])
 
 
 if __name__ == "__main__":

@@ -141,6 +141,54 @@ size_t part_bytes(const hkv_config *c) {
   return (b + 255) & ~(size_t)255;
 }
 
+size_t cnt_bytes(const hkv_config *c) {
+  return ((size_t)c->n_seqs * c->n_heads * sizeof(int32_t) + 15) & ~(size_t)15;
+}
+
+// Fills the attention launch arguments for one layer; the workspace holds
+// the split-K partials, the per-head counters and the grid counter.
+AttnArgs attn_args(const hkv_config *cfg, const hkv_cache *cache, int layer, const void *q,
+                   float *out, void *workspace) {
+  const int hpl = cfg->n_seqs * cfg->n_heads;
+  AttnArgs a = {};
+  a.K = cache->k;
+  a.V = cache->v;
+  a.off = cache->off + (size_t)layer * hpl;
+  a.len = cache->len + (size_t)layer * hpl;
+  a.cap = cache->cap + (size_t)layer * hpl;
+  a.q = q;
+  a.out = out;
+  unsigned char *ws = static_cast<unsigned char *>(workspace);
+  a.part = reinterpret_cast<float *>(ws);
+  a.cnt = reinterpret_cast<int32_t *>(ws + part_bytes(cfg));
+  a.gcnt = reinterpret_cast<int32_t *>(ws + part_bytes(cfg) + cnt_bytes(cfg));
+  a.err = cache->err;
+  a.pos = cache->pos;
+  a.nbuf = cache->nbuf;
+  a.ntok = cache->ntok;
+  a.label = cache->label;
+  a.qbuf = cache->qbuf;
+  a.layer_base = layer * hpl;
+  a.period = cfg->period;
+  a.n_cond = cfg->n_cond;
+  a.arena_tokens = cache->capacity_tokens;
+  a.nheads = hpl;
+  a.qscale = (float)(1.4426950408889634 / sqrt((double)cfg->head_dim));
+  return a;
+}
+
+hkv_status attn_grid(const hkv_config *cfg, int *grid) {
+  DeviceState *st;
+  hkv_status s = device_state(&st);
+  if (s != HKV_OK) return s;
+  int ctas = 0;
+  s = attention_ctas(st, cfg->head_dim, cfg->dtype, &ctas);
+  if (s != HKV_OK) return s;
+  int g = st->sms * ctas;
+  *grid = g > kAttnMaxGrid ? kAttnMaxGrid : g;
+  return HKV_OK;
+}
+
 #define HKV_TRY(x)                 \
   do {                             \
     hkv_status s_ = (x);           \
@@ -186,7 +234,7 @@ hkv_status hkv_validate_config(const hkv_config *c) {
 
 size_t hkv_workspace_size(const hkv_config *c) {
   if (!c || hkv_validate_config(c) != HKV_OK) return 0;
-  return part_bytes(c) + (size_t)heads_per_layer(c) * sizeof(int32_t);
+  return part_bytes(c) + cnt_bytes(c) + 16;
 }
 
 hkv_status hkv_init_dense(const hkv_config *cfg, const hkv_cache *cache, hkv_stream_t stream) {
@@ -240,28 +288,48 @@ hkv_status hkv_decode_attention(const hkv_config *cfg, const hkv_cache *cache, i
   if (!q || !out || !workspace) return HKV_ERR_INVALID_ARG;
   if (!aligned16(q) || !aligned16(out) || !aligned16(workspace)) return HKV_ERR_ALIGN;
   if (ws_bytes < hkv_workspace_size(cfg)) return HKV_ERR_CAPACITY;
+  int grid = 0;
+  HKV_TRY(attn_grid(cfg, &grid));
+  const AttnArgs a = attn_args(cfg, cache, layer, q, out, workspace);
+  return cuda_status(
+      launch_attention(a, cfg->head_dim, cfg->dtype, grid, false, (cudaStream_t)stream));
+}
+
+hkv_status hkv_decode_step(const hkv_config *cfg, const hkv_cache *cache, int layer,
+                           const void *q, const void *k, const void *v, float *out,
+                           void *workspace, size_t ws_bytes, int flags, hkv_stream_t stream) {
+  HKV_TRY(injected("decode_step"));
+  HKV_TRY(hkv_validate_config(cfg));
+  HKV_TRY(check_cache(cache));
+  if (layer < 0 || layer >= cfg->n_layers) return HKV_ERR_INVALID_ARG;
+  if (!q || !k || !v || !out || !workspace) return HKV_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out) || !aligned16(workspace))
+    return HKV_ERR_ALIGN;
+  if (ws_bytes < hkv_workspace_size(cfg)) return HKV_ERR_CAPACITY;
+  if (flags & ~HKV_STEP_PREFETCH) return HKV_ERR_INVALID_ARG;
+  int grid = 0;
+  HKV_TRY(attn_grid(cfg, &grid));
+  AttnArgs a = attn_args(cfg, cache, layer, q, out, workspace);
+  a.k_new = k;
+  a.v_new = v;
+  a.prefetch = (flags & HKV_STEP_PREFETCH) ? 1 : 0;
+  return cuda_status(
+      launch_attention(a, cfg->head_dim, cfg->dtype, grid, true, (cudaStream_t)stream));
+}
+
+hkv_status hkv_evict(const hkv_config *cfg, const hkv_cache *cache, int layer,
+                     hkv_stream_t stream) {
+  HKV_TRY(injected("evict"));
+  HKV_TRY(hkv_validate_config(cfg));
+  HKV_TRY(check_cache(cache));
+  if (layer < 0 || layer >= cfg->n_layers) return HKV_ERR_INVALID_ARG;
   DeviceState *st;
   HKV_TRY(device_state(&st));
-  int ctas = 0;
-  HKV_TRY(attention_ctas(st, cfg->head_dim, cfg->dtype, &ctas));
-  int grid = st->sms * ctas;
-  if (grid > kAttnMaxGrid) grid = kAttnMaxGrid;
+  const size_t smem = update_smem_bytes(max_segment(cfg), cfg->head_dim);
+  HKV_TRY(update_ready(st, cfg->head_dim, cfg->dtype, smem));
   const int hpl = heads_per_layer(cfg);
-  AttnArgs a;
-  a.K = cache->k;
-  a.V = cache->v;
-  a.off = cache->off + (size_t)layer * hpl;
-  a.len = cache->len + (size_t)layer * hpl;
-  a.q = q;
-  a.out = out;
-  a.part = static_cast<float *>(workspace);
-  a.cnt = reinterpret_cast<int32_t *>(static_cast<unsigned char *>(workspace) + part_bytes(cfg));
-  a.err = cache->err;
-  a.arena_tokens = cache->capacity_tokens;
-  a.nheads = hpl;
-  a.qscale = (float)(1.4426950408889634 / sqrt((double)cfg->head_dim));
-  return cuda_status(
-      launch_attention(a, cfg->head_dim, cfg->dtype, grid, (cudaStream_t)stream));
+  return cuda_status(launch_evict(cache_args(cache), method_args(cfg), layer * hpl, hpl,
+                                  cfg->head_dim, cfg->dtype, smem, (cudaStream_t)stream));
 }
 
 hkv_status hkv_identify_heads(const hkv_config *cfg, const hkv_cache *cache, int layer,

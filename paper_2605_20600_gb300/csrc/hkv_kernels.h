@@ -9,27 +9,45 @@
 
 namespace hkv {
 
-// split-K decode attention over one layer of a ragged cache
+// split-K decode attention over one layer of a ragged cache, optionally
+// fused with the append of the step's new token
 struct AttnArgs {
-  const void *K, *V;          // arena
+  void *K, *V;                // arena
   const int64_t *off;         // layer slice of segment offsets
-  const int32_t *len;         // layer slice of live lengths
+  int32_t *len;               // layer slice of live lengths
+  const int32_t *cap;         // layer slice of capacities (fused)
   const void *q;              // [nheads][D]
+  const void *k_new, *v_new;  // [nheads][D] new token (fused)
   float *out;                 // [nheads][D]
   float *part;                // [grid][2][D + 2] partial results
   int32_t *cnt;               // [nheads] arrival counters (zero between calls)
+  int32_t *gcnt;              // grid arrival counter (fused; zero between calls)
   uint32_t *err;
+  // fused append: full [L*S*H] arrays and the layer's first flat head
+  int32_t *pos, *nbuf, *ntok;
+  const uint8_t *label;
+  void *qbuf;
+  int layer_base;
+  int period, n_cond;
   int64_t arena_tokens;
   int nheads;
   float qscale;               // log2(e) / sqrt(D)
+  int prefetch;               // read the layer's cache before waiting for the
+                              // previous kernel (its writes do not touch it)
 };
 
-constexpr int kAttnThreads = 128;
+// decode attention CTA: one producer warp (TMA) + consumer warps
+#ifndef HKV_ATTN_CONSUMER_WARPS
+#define HKV_ATTN_CONSUMER_WARPS 8
+#endif
+constexpr int kAttnConsumerWarps = HKV_ATTN_CONSUMER_WARPS;
+constexpr int kAttnThreads = 32 * (kAttnConsumerWarps + 1);
 constexpr int kAttnMaxGrid = 4096;
 
 size_t attention_smem_bytes(int D, int dtype);
 cudaError_t attention_prepare(int D, int dtype, int *ctas_per_sm);
-cudaError_t launch_attention(const AttnArgs &a, int D, int dtype, int grid, cudaStream_t s);
+cudaError_t launch_attention(const AttnArgs &a, int D, int dtype, int grid, bool fused,
+                             cudaStream_t s);
 
 // per-head cache maintenance (append / update / repack / prefill / identify)
 struct CacheArgs {
@@ -59,6 +77,8 @@ cudaError_t update_prepare(int D, int dtype, size_t smem);
 cudaError_t launch_append_evict(const CacheArgs &c, const MethodArgs &m, int layer_base,
                                 int nheads, const void *q, const void *k, const void *v, int D,
                                 int dtype, size_t smem, cudaStream_t s);
+cudaError_t launch_evict(const CacheArgs &c, const MethodArgs &m, int layer_base, int nheads,
+                         int D, int dtype, size_t smem, cudaStream_t s);
 cudaError_t launch_repack(const CacheArgs &dense, const CacheArgs &ragged, const MethodArgs &m,
                           int layer_base, int nheads, int D, int dtype, size_t smem,
                           cudaStream_t s);

@@ -103,7 +103,7 @@ extern "C" hkv_status hkv_decode_attention_noalloc(const hkv_config *cfg, const 
   if (cudaMemsetAsync(cnt, 0, (size_t)hpl * sizeof(int32_t), s) != cudaSuccess)
     return HKV_ERR_CUDA;
 
-  AttnArgs a;
+  AttnArgs a = {};
   a.K = cache->k;
   a.V = cache->v;
   a.off = cache->off + (size_t)layer * hpl;
@@ -116,6 +116,7 @@ extern "C" hkv_status hkv_decode_attention_noalloc(const hkv_config *cfg, const 
   a.arena_tokens = cache->capacity_tokens;
   a.nheads = hpl;
   a.qscale = (float)(1.4426950408889634 / sqrt((double)cfg->head_dim));
-  return launch_attention(a, cfg->head_dim, cfg->dtype, grid, s) == cudaSuccess ? HKV_OK
-                                                                                  : HKV_ERR_CUDA;
+  return launch_attention(a, cfg->head_dim, cfg->dtype, grid, false, s) == cudaSuccess
+             ? HKV_OK
+             : HKV_ERR_CUDA;
 }

@@ -1,23 +1,28 @@
 // Per-head cache maintenance of HeadKV, one CTA per head:
-//  * append_evict: the periodic head-aware update when the buffer is full
-//    (Sec. 4: local heads drop their history, Eq. 3; global heads trim it
-//    by Stratified Token Eviction, Eqs. 4-6), then the append of the new
-//    token (Sec. 3, KV Cache);
+//  * evict / append_evict: the periodic head-aware update when a head's
+//    buffer holds P tokens (Sec. 4: local heads drop their history, Eq. 3;
+//    global heads trim it by Stratified Token Eviction, Eqs. 4-6), and for
+//    append_evict the append of the new token after it (Sec. 3, KV Cache);
 //  * repack: the first update at grouping, out of place from the dense
 //    cache into the ragged one (Step 3);
 //  * prefill / init_dense: the uncompressed cache of Step 1;
 //  * identify: threshold-based attention accumulation (Step 2);
 //  * budgets: per-head budgets and the arena layout (Sec. 5.1).
 //
-// STE on the device: the P buffered queries are summed (q-bar), each
-// history key is scored q-bar . k in a fixed fp32 order, a (score, position)
-// 64-bit key is formed (unique, ascending = evict first), an 8-pass radix
-// select finds the quota-th smallest key of the long- and near-range
-// subsets at once, and a block prefix sum over the keep flags gives every
-// survivor its new row; rows move in ascending chunks (destination <=
-// source), each chunk fully loaded before any of it is stored, so the
-// compaction is safe in place.
+// The update works on token POSITIONS, not on storage order, so a segment
+// may hold its live tokens in any order:
+//  * conditioning tokens have positions < C; the recent window is the newest
+//    w image tokens, positions >= C + ntok - w; everything else is history;
+//  * Eq. 5's long-range subset is the floor(T * r_s) history tokens with the
+//    smallest positions (a rank select on positions);
+//  * scores q-bar . k in a fixed fp32 order, keys (order-preserving score
+//    bits, position) unique and ascending in eviction priority, one 8-pass
+//    MSD radix select finds the quota-th key of both subsets at once;
+//  * in place, the holes below the new length are refilled with the
+//    surviving rows above it: at most M rows move and no move depends on
+//    another, instead of shifting every row after the first eviction.
 #include <math.h>
+#include <stdlib.h>
 
 #include "hkv_device.cuh"
 #include "hkv_kernels.h"
@@ -26,6 +31,13 @@ namespace hkv {
 namespace {
 
 constexpr int NT = kCacheThreads;
+
+__device__ __forceinline__ void pdl_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
 
 struct SegRef {
   const unsigned char *sk, *sv;  // source rows, row 0 = segment start
@@ -37,19 +49,37 @@ struct SegRef {
   bool in_place;
 };
 
-struct SelectShared {
+struct UpdShared {
   unsigned long long prefix[2];
   int rem[2];
-  int scan[33];
-  int first;
-  int bad;
+  int iscan[33];
 };
 
-// The k0-th smallest key among keys[0, n_long) and the k1-th among
-// keys[n_long, T) (1-based; 0 = not needed), by MSD radix select on bytes.
-// Keys are unique, so the result identifies exactly k keys at or below it.
-__device__ void radix_select2(const unsigned long long *keys, int T, int n_long, int k0, int k1,
-                              int *hist, SelectShared &sh) {
+// Shared-memory work area of one update (dynamic).
+struct UpdSmem {
+  unsigned long long *keys;  // [max_len]
+  int *ps;                   // [max_len] positions of the source rows
+  int *aux;                  // [max_len] class, then keep flag, then rank
+  float *qbar;               // [D]
+  int *hist;                 // [512]
+};
+
+__device__ __forceinline__ UpdSmem carve(unsigned char *dyn, int max_len, int D) {
+  UpdSmem u;
+  u.keys = reinterpret_cast<unsigned long long *>(dyn);
+  u.ps = reinterpret_cast<int *>(u.keys + max_len);
+  u.aux = u.ps + max_len;
+  u.qbar = reinterpret_cast<float *>(u.aux + max_len);
+  u.hist = reinterpret_cast<int *>(u.qbar + D);
+  return u;
+}
+
+// The k0-th smallest key among rows of class 0 and the k1-th among rows of
+// class 1 (1-based; 0 = not needed; other classes ignored), by MSD radix
+// select on bytes from `top_shift` down. Keys are unique within a class, so
+// each result bounds exactly k keys of its class from above.
+__device__ void radix_select2(const unsigned long long *keys, const int *cls, int n, int k0,
+                              int k1, int top_shift, int *hist, UpdShared &sh) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   if (tid == 0) {
     sh.prefix[0] = sh.prefix[1] = 0ull;
@@ -57,14 +87,15 @@ __device__ void radix_select2(const unsigned long long *keys, int T, int n_long,
     sh.rem[1] = k1;
   }
   __syncthreads();
-  for (int shift = 56; shift >= 0; shift -= 8) {
+  for (int shift = top_shift; shift >= 0; shift -= 8) {
     for (int i = tid; i < 512; i += NT) hist[i] = 0;
     __syncthreads();
-    const unsigned long long hi = shift == 56 ? 0ull : (~0ull << (shift + 8));
+    const unsigned long long hi = shift >= 56 ? 0ull : (~0ull << (shift + 8));
     const unsigned long long p0 = sh.prefix[0], p1 = sh.prefix[1];
     const int r0 = sh.rem[0], r1 = sh.rem[1];
-    for (int j = tid; j < T; j += NT) {
-      const int s = j < n_long ? 0 : 1;
+    for (int j = tid; j < n; j += NT) {
+      const int s = cls[j];
+      if (s != 0 && s != 1) continue;
       const unsigned long long key = keys[j];
       if ((s ? r1 : r0) > 0 && (key & hi) == (s ? p1 : p0))
         atomicAdd(&hist[s * 256 + (int)((key >> shift) & 255ull)], 1);
@@ -101,44 +132,53 @@ __device__ void radix_select2(const unsigned long long *keys, int T, int n_long,
   }
 }
 
-// One head-aware update of a segment (Eqs. 2-6). Returns the new length,
-// or -1 if the destination is too small (error word set). Block-uniform.
+__device__ __forceinline__ int block_sum(int x, UpdShared &sh) {
+  int tot;
+  block_excl_scan<int>(x, sh.iscan, &tot);
+  return tot;
+}
+
+// Decides which rows of a segment the update evicts (Eqs. 2-6). On return
+// u.aux[r] is 1 for a kept row and 0 for an evicted one (r < len), u.ps
+// holds the rows' positions, and the number of evicted rows is returned.
+// Block-uniform.
 template <int D, typename T>
-__device__ int update_segment(const SegRef &sg, int label, const MethodArgs &m,
-                              const unsigned char *qring, int ntok, unsigned char *dyn,
-                              int max_len, uint32_t *err) {
+__device__ int select_evictions(const SegRef &sg, int label, const MethodArgs &m,
+                                const unsigned char *qring, int ntok, const UpdSmem &u,
+                                UpdShared &sh) {
   constexpr int RB = D * (int)sizeof(T);
   constexpr int EPL = Elem<T>::kPerPiece;
   constexpr int LPR = RB / 16;
-  constexpr int U = 4;                 // 16-byte pieces per thread per chunk
-  constexpr int CH = NT * U / LPR;     // rows per move chunk
-  static_assert(CH <= NT, "one pos per thread per chunk");
-  __shared__ SelectShared sh;
-
   const int tid = threadIdx.x;
   const int C = m.C;
-  const int n_img = sg.len - C;
-  const int n_recent = n_img < m.w ? n_img : m.w;
-  const int NH = n_img - n_recent;  // history candidates (Eq. 2)
-  int M = 0;
-  if (label == HKV_LOCAL) M = NH;   // Eq. 3: no history
-  else if (NH > m.hist_budget) M = NH - m.hist_budget;
-  if (M == 0 && sg.in_place) return sg.len;
-  if (sg.len - M > sg.dst_cap) {
-    if (tid == 0) set_err(err, HKV_ERR_CAPACITY);
-    return -1;
+  const int recent_from = C + (ntok > m.w ? ntok - m.w : 0);   // newest w image tokens
+  int nh = 0;
+  for (int r = tid; r < sg.len; r += NT) {
+    const int ps = sg.spos[r];
+    u.ps[r] = ps;
+    const bool hist = ps >= C && ps < recent_from;
+    u.aux[r] = hist ? 0 : -1;   // class: history (0) or always kept (-1)
+    nh += hist ? 1 : 0;
   }
-
-  unsigned long long *keys = reinterpret_cast<unsigned long long *>(dyn);
-  int *dst = reinterpret_cast<int *>(keys + max_len);
-  float *qbar = reinterpret_cast<float *>(dst + max_len);
-  int *hist = reinterpret_cast<int *>(qbar + D);
-
-  // dst[] first holds the keep flags
-  for (int r = tid; r < sg.len; r += NT) dst[r] = (r >= C && r < C + NH && label == HKV_LOCAL) ? 0 : 1;
+  const int NH = block_sum(nh, sh);  // history candidates (Eq. 2)
+  int M = 0;
+  if (label == HKV_LOCAL) M = NH;    // Eq. 3: no history
+  else if (NH > m.hist_budget) M = NH - m.hist_budget;
 
   if (label == HKV_GLOBAL && M > 0) {
-    // q-bar: the P buffered queries, oldest first (Eq. 6, reading R8/R10)
+    // Eq. 5: the floor(NH r_s) oldest history tokens are long-range
+    const int n_long = (int)floor((double)NH * m.r_s);
+    if (n_long > 0 && n_long < NH) {
+      for (int r = tid; r < sg.len; r += NT) u.keys[r] = (unsigned long long)(uint32_t)u.ps[r];
+      radix_select2(u.keys, u.aux, sg.len, n_long, 0, 24, u.hist, sh);
+      const int p_long = (int)sh.prefix[0];
+      for (int r = tid; r < sg.len; r += NT)
+        if (u.aux[r] == 0) u.aux[r] = u.ps[r] <= p_long ? 0 : 1;
+    } else {
+      for (int r = tid; r < sg.len; r += NT)
+        if (u.aux[r] == 0) u.aux[r] = n_long == NH ? 0 : 1;
+    }
+    // Eq. 6 scores: q-bar = the P buffered queries, oldest first
     const int P = m.P;
     for (int d = tid; d < D; d += NT) {
       float acc = 0.f;
@@ -147,28 +187,27 @@ __device__ int update_segment(const SegRef &sg, int label, const MethodArgs &m,
         if (slot < 0) slot += P;
         acc = __fadd_rn(acc, Elem<T>::load1(qring, (size_t)slot * D + d));
       }
-      qbar[d] = acc;
+      u.qbar[d] = acc;
     }
     __syncthreads();
-    // scores s_j = q-bar . k_j, d ascending, each product and sum rounded
-    for (int j = tid; j < NH; j += NT) {
-      const unsigned char *krow = sg.sk + (size_t)(C + j) * RB;
+    for (int r = tid; r < sg.len; r += NT) {
+      if (u.aux[r] < 0) continue;
+      const unsigned char *krow = sg.sk + (size_t)r * RB;
       float s = 0.f;
 #pragma unroll 4
       for (int pc = 0; pc < LPR; ++pc) {
         float kf[EPL];
         Elem<T>::unpack(*reinterpret_cast<const uint4 *>(krow + pc * 16), kf);
 #pragma unroll
-        for (int e = 0; e < EPL; ++e) s = __fadd_rn(s, __fmul_rn(qbar[pc * EPL + e], kf[e]));
+        for (int e = 0; e < EPL; ++e) s = __fadd_rn(s, __fmul_rn(u.qbar[pc * EPL + e], kf[e]));
       }
       s = __fadd_rn(s, 0.f);  // -0 reads as +0
-      uint32_t u = __float_as_uint(s);
-      u = (u & 0x80000000u) ? ~u : (u | 0x80000000u);  // order-preserving
-      keys[j] = ((unsigned long long)u << 32) | (uint32_t)sg.spos[C + j];
+      uint32_t bits = __float_as_uint(s);
+      bits = (bits & 0x80000000u) ? ~bits : (bits | 0x80000000u);  // order-preserving
+      u.keys[r] = ((unsigned long long)bits << 32) | (uint32_t)u.ps[r];
     }
     __syncthreads();
-    // Eq. 5 split and the M/2 quotas, excess of a short subset to the other
-    const int n_long = (int)floor((double)NH * m.r_s);
+    // M/2 from each subset; a short subset hands its excess to the other
     int m_long = M / 2, m_near = M - M / 2;
     if (m_long > n_long) {
       m_near += m_long - n_long;
@@ -178,65 +217,145 @@ __device__ int update_segment(const SegRef &sg, int label, const MethodArgs &m,
       m_long += m_near - (NH - n_long);
       m_near = NH - n_long;
     }
-    radix_select2(keys, NH, n_long, m_long, m_near, hist, sh);
+    radix_select2(u.keys, u.aux, sg.len, m_long, m_near, 56, u.hist, sh);
     const unsigned long long thr0 = sh.prefix[0], thr1 = sh.prefix[1];
-    for (int j = tid; j < NH; j += NT) {
-      const bool ev = j < n_long ? (m_long > 0 && keys[j] <= thr0) : (m_near > 0 && keys[j] <= thr1);
-      if (ev) dst[C + j] = 0;
+    for (int r = tid; r < sg.len; r += NT) {
+      const int c = u.aux[r];
+      const bool ev = c == 0 ? (m_long > 0 && u.keys[r] <= thr0)
+                             : c == 1 ? (m_near > 0 && u.keys[r] <= thr1) : false;
+      u.aux[r] = ev ? 0 : 1;
     }
+  } else {
+    for (int r = tid; r < sg.len; r += NT) u.aux[r] = (u.aux[r] == 0 && M > 0) ? 0 : 1;
   }
-  if (tid == 0) sh.first = sg.len;
   __syncthreads();
+  return M;
+}
 
-  // prefix sum of keep flags -> destination rows; first row that moves
-  int running = 0;
+template <int D, typename T>
+__device__ __forceinline__ void copy_piece(unsigned char *dk, unsigned char *dv,
+                                           const unsigned char *sk, const unsigned char *sv,
+                                           int piece) {
+  *reinterpret_cast<uint4 *>(dk + piece * 16) =
+      __ldcg(reinterpret_cast<const uint4 *>(sk + piece * 16));
+  *reinterpret_cast<uint4 *>(dv + piece * 16) =
+      __ldcg(reinterpret_cast<const uint4 *>(sv + piece * 16));
+}
+
+// In place: the new length is len - M; every evicted row below it takes a
+// surviving row from above it (the i-th hole the i-th survivor). Sources
+// are all >= new_len and destinations < new_len, so the moves are
+// independent. Returns the new length.
+template <int D, typename T>
+__device__ int fill_holes(const SegRef &sg, int M, const UpdSmem &u, UpdShared &sh) {
+  constexpr int RB = D * (int)sizeof(T);
+  constexpr int LPR = RB / 16;
+  const int tid = threadIdx.x;
+  const int new_len = sg.len - M;
+  if (M == 0) return sg.len;
+  // rank holes (evicted, r < new_len) and fills (kept, r >= new_len); the
+  // keys area is free now and holds the two index lists
+  int *hole = reinterpret_cast<int *>(u.keys);  // [<= M]
+  int *fill = hole + M;                          // [<= M]
+  int hrun = 0, frun = 0;
   for (int base = 0; base < sg.len; base += NT) {
     const int r = base + tid;
-    const int k = r < sg.len ? dst[r] : 0;
-    int tot;
-    const int ex = block_excl_scan<int>(k, sh.scan, &tot);
-    if (r < sg.len) {
-      const int d = k ? running + ex : -1;
-      dst[r] = d;
-      if (d != r) atomicMin(&sh.first, r);
-    }
-    running += tot;
+    const int keep = r < sg.len ? u.aux[r] : 1;
+    const int is_hole = (r < new_len && !keep) ? 1 : 0;
+    const int is_fill = (r >= new_len && r < sg.len && keep) ? 1 : 0;
+    int ht, ft;
+    const int hx = block_excl_scan<int>(is_hole, sh.iscan, &ht);
+    const int fx = block_excl_scan<int>(is_fill, sh.iscan, &ft);
+    if (is_hole) hole[hrun + hx] = r;
+    if (is_fill) fill[frun + fx] = r;
+    hrun += ht;
+    frun += ft;
   }
   __syncthreads();
-  const int new_len = running;
-  const int first = sg.in_place ? sh.first : 0;
-
-  // move rows in ascending chunks: load the whole chunk, then store it
-  for (int c0 = first; c0 < sg.len; c0 += CH) {
-    uint4 kr[U], vr[U];
-    int drow[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int piece = u * NT + tid;
-      const int r = c0 + piece / LPR, col = piece % LPR;
-      drow[u] = r < sg.len ? dst[r] : -1;
-      if (drow[u] >= 0) {
-        kr[u] = __ldcg(reinterpret_cast<const uint4 *>(sg.sk + (size_t)r * RB + col * 16));
-        vr[u] = __ldcg(reinterpret_cast<const uint4 *>(sg.sv + (size_t)r * RB + col * 16));
-      }
-    }
-    const int pr = c0 + tid;
-    const int pd = (tid < CH && pr < sg.len) ? dst[pr] : -1;
-    const int pv = pd >= 0 ? __ldcg(sg.spos + pr) : 0;
-    __syncthreads();
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int piece = u * NT + tid;
-      const int col = piece % LPR;
-      if (drow[u] >= 0) {
-        *reinterpret_cast<uint4 *>(sg.dk + (size_t)drow[u] * RB + col * 16) = kr[u];
-        *reinterpret_cast<uint4 *>(sg.dv + (size_t)drow[u] * RB + col * 16) = vr[u];
-      }
-    }
-    if (pd >= 0) sg.dpos[pd] = pv;
-    __syncthreads();
+  const int k = hrun < frun ? hrun : frun;  // equal by construction
+  for (int w = tid; w < k * LPR; w += NT) {
+    const int j = w / LPR, pc = w % LPR;
+    const int dr = hole[j], sr = fill[j];
+    copy_piece<D, T>(sg.dk + (size_t)dr * RB, sg.dv + (size_t)dr * RB, sg.sk + (size_t)sr * RB,
+                     sg.sv + (size_t)sr * RB, pc);
   }
+  for (int j = tid; j < k; j += NT) sg.dpos[hole[j]] = u.ps[fill[j]];
+  __syncthreads();
   return new_len;
+}
+
+// Out of place, keeping the source order: survivors are packed by a prefix
+// sum of the keep flags. Returns the new length.
+template <int D, typename T>
+__device__ int copy_kept(const SegRef &sg, const UpdSmem &u, UpdShared &sh) {
+  constexpr int RB = D * (int)sizeof(T);
+  constexpr int LPR = RB / 16;
+  const int tid = threadIdx.x;
+  int run = 0;
+  for (int base = 0; base < sg.len; base += NT) {
+    const int r = base + tid;
+    const int keep = r < sg.len ? u.aux[r] : 0;
+    int tot;
+    const int ex = block_excl_scan<int>(keep, sh.iscan, &tot);
+    if (r < sg.len) u.aux[r] = keep ? run + ex : -1;
+    run += tot;
+  }
+  __syncthreads();
+  for (int w = tid; w < sg.len * LPR; w += NT) {
+    const int r = w / LPR, pc = w % LPR;
+    const int d = u.aux[r];
+    if (d >= 0)
+      copy_piece<D, T>(sg.dk + (size_t)d * RB, sg.dv + (size_t)d * RB, sg.sk + (size_t)r * RB,
+                       sg.sv + (size_t)r * RB, pc);
+  }
+  for (int r = tid; r < sg.len; r += NT)
+    if (u.aux[r] >= 0) sg.dpos[u.aux[r]] = u.ps[r];
+  __syncthreads();
+  return run;
+}
+
+// The update of one head in place (local: window slide; global: STE).
+template <int D, typename T>
+__device__ int update_in_place(const SegRef &sg, int label, const MethodArgs &m,
+                               const unsigned char *qring, int ntok, const UpdSmem &u,
+                               UpdShared &sh) {
+  const int M = select_evictions<D, T>(sg, label, m, qring, ntok, u, sh);
+  return fill_holes<D, T>(sg, M, u, sh);
+}
+
+template <int D, typename T>
+__global__ void __launch_bounds__(NT)
+    evict_kernel(const CacheArgs c, const MethodArgs m, int layer_base, int max_len) {
+  constexpr int RB = D * (int)sizeof(T);
+  extern __shared__ __align__(16) unsigned char dyn[];
+  __shared__ UpdShared sh;
+  // no early launch of the next kernel: a decode step that prefetches this
+  // layer's cache before its own wait must start after the update is done
+  pdl_wait();
+  const int tid = threadIdx.x, i = layer_base + blockIdx.x;
+  const uint8_t lab = c.label[i];
+  const int nbuf = c.nbuf[i];
+  if (lab == HKV_DENSE || nbuf < m.P) return;  // not due
+  const int len = c.len[i], cp = c.cap[i];
+  const long long off = c.off[i];
+  if (off < 0 || cp < 0 || off + cp > c.arena_tokens || len < 0 || len > cp) {
+    if (tid == 0) set_err(c.err, HKV_ERR_BOUNDS);
+    return;
+  }
+  if (len > max_len) {
+    if (tid == 0) set_err(c.err, HKV_ERR_CAPACITY);
+    return;
+  }
+  unsigned char *K = static_cast<unsigned char *>(c.K) + off * RB;
+  unsigned char *V = static_cast<unsigned char *>(c.V) + off * RB;
+  int32_t *pos = c.pos + off;
+  const unsigned char *qring = static_cast<const unsigned char *>(c.qbuf) + (size_t)i * m.P * RB;
+  SegRef sg{K, V, pos, K, V, pos, len, cp, true};
+  const int nl = update_in_place<D, T>(sg, lab, m, qring, c.ntok[i], carve(dyn, max_len, D), sh);
+  if (tid == 0) {
+    c.len[i] = nl;
+    c.nbuf[i] = 0;
+  }
 }
 
 template <int D, typename T>
@@ -245,6 +364,9 @@ __global__ void __launch_bounds__(NT)
                         const void *k, const void *v, int max_len) {
   constexpr int RB = D * (int)sizeof(T);
   extern __shared__ __align__(16) unsigned char dyn[];
+  __shared__ UpdShared sh;
+  pdl_wait();
+  pdl_launch_dependents();
   const int tid = threadIdx.x, hl = blockIdx.x, i = layer_base + hl;
   int len = c.len[i];
   const int cp = c.cap[i];
@@ -267,9 +389,7 @@ __global__ void __launch_bounds__(NT)
       return;
     }
     SegRef sg{K, V, pos, K, V, pos, len, cp, true};
-    const int nl = update_segment<D, T>(sg, lab, m, qring, ntok, dyn, max_len, c.err);
-    if (nl < 0) return;
-    len = nl;
+    len = update_in_place<D, T>(sg, lab, m, qring, ntok, carve(dyn, max_len, D), sh);
     nbuf = 0;
   }
   if (len >= cp) {
@@ -306,6 +426,9 @@ __global__ void __launch_bounds__(NT)
                   int max_len) {
   constexpr int RB = D * (int)sizeof(T);
   extern __shared__ __align__(16) unsigned char dyn[];
+  __shared__ UpdShared sh;
+  pdl_wait();
+  pdl_launch_dependents();
   const int tid = threadIdx.x, i = layer_base + blockIdx.x;
   const int slen = dn.len[i];
   const long long soff = dn.off[i];
@@ -335,8 +458,13 @@ __global__ void __launch_bounds__(NT)
             dcap,
             false};
   const unsigned char *qring = static_cast<const unsigned char *>(dn.qbuf) + (size_t)i * m.P * RB;
-  const int nl = update_segment<D, T>(sg, lab, m, qring, dn.ntok[i], dyn, max_len, rg.err);
-  if (nl < 0) return;
+  const UpdSmem u = carve(dyn, max_len, D);
+  const int M = select_evictions<D, T>(sg, lab, m, qring, dn.ntok[i], u, sh);
+  if (slen - M > dcap) {
+    if (tid == 0) set_err(rg.err, HKV_ERR_CAPACITY);
+    return;
+  }
+  const int nl = copy_kept<D, T>(sg, u, sh);
   if (tid == 0) {
     rg.len[i] = nl;
     rg.nbuf[i] = 0;
@@ -348,6 +476,8 @@ template <int D, typename T>
 __global__ void prefill_kernel(const CacheArgs c, int layer_base, int C, const void *kc,
                                const void *vc) {
   constexpr int RB = D * (int)sizeof(T);
+  pdl_wait();
+  pdl_launch_dependents();
   const int hl = blockIdx.x, i = layer_base + hl, tid = threadIdx.x;
   const long long off = c.off[i];
   const int cp = c.cap[i];
@@ -377,6 +507,8 @@ __global__ void prefill_kernel(const CacheArgs c, int layer_base, int C, const v
 }
 
 __global__ void init_dense_kernel(const CacheArgs c, int n, int seg) {
+  pdl_wait();
+  pdl_launch_dependents();
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) {
     const_cast<int64_t *>(c.off)[i] = (int64_t)i * seg;
     const_cast<int32_t *>(c.cap)[i] = seg;
@@ -390,7 +522,7 @@ __global__ void init_dense_kernel(const CacheArgs c, int n, int seg) {
 
 // Step 2: attention of the current query over the key cache, accumulated
 // backward from the newest token until tau; local iff fewer than w_loc
-// tokens were needed.
+// tokens were needed. The dense cache holds its tokens in position order.
 template <int D, typename T>
 __global__ void __launch_bounds__(NT)
     identify_kernel(const CacheArgs c, const MethodArgs m, int layer_base, const void *q,
@@ -405,10 +537,16 @@ __global__ void __launch_bounds__(NT)
   __shared__ float s_bcast;
   __shared__ float fscan[33];
   __shared__ int s_nh;
+  pdl_wait();
+  pdl_launch_dependents();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int hl = blockIdx.x, i = layer_base + hl;
   const int len = c.len[i];
   const long long off = c.off[i];
+  if (c.label[i] != HKV_DENSE) {  // only the uncompressed cache is in order
+    if (tid == 0) set_err(c.err, HKV_ERR_STATE);
+    return;
+  }
   if (off < 0 || len <= 0 || off + len > c.arena_tokens) {
     if (tid == 0) set_err(c.err, HKV_ERR_BOUNDS);
     return;
@@ -425,8 +563,7 @@ __global__ void __launch_bounds__(NT)
 #pragma unroll
   for (int x = 0; x < EPL; ++x) qf[x] *= qscale;
   const unsigned char *K = static_cast<const unsigned char *>(c.K) + off * RB;
-  // logits (log2 units)
-  for (int r0 = warp * RPW; r0 < len; r0 += NW * RPW) {
+  for (int r0 = warp * RPW; r0 < len; r0 += NW * RPW) {  // logits (log2 units)
     const int r = r0 + grp;
     float dot = 0.f;
     if (r < len) {
@@ -472,8 +609,7 @@ __global__ void __launch_bounds__(NT)
   }
   __syncthreads();
   const float thr = s_bcast;
-  // backward cumulative mass from the newest token
-  float running = 0.f;
+  float running = 0.f;  // backward cumulative mass from the newest token
   for (int base = 0; base < len; base += NT) {
     const int jb = base + tid;  // jb-th newest token (0 = current)
     const float x = jb < len ? e[len - 1 - jb] : 0.f;
@@ -492,6 +628,8 @@ __global__ void __launch_bounds__(NT)
 __global__ void budgets_kernel(const uint8_t *label, int32_t *budget, int32_t *cap, int64_t *off,
                                int n, int C, int B_g, int w, int P) {
   __shared__ long long scratch[33];
+  pdl_wait();
+  pdl_launch_dependents();
   long long running = 0;
   int bad = 0;
   for (int base = 0; base < n; base += blockDim.x) {
@@ -519,12 +657,16 @@ template <int D, typename T>
 cudaError_t prepare_t(size_t smem) {
   cudaError_t e = cudaFuncSetAttribute(append_evict_kernel<D, T>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(repack_kernel<D, T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           (int)smem);
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(identify_kernel<D, T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(evict_kernel<D, T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(repack_kernel<D, T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(identify_kernel<D, T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+  return e;
 }
 
 #define HKV_DISPATCH(D_, DT_, ...)                  \
@@ -552,11 +694,35 @@ cudaError_t prepare_t(size_t smem) {
     }                                               \
   } while (0)
 
+// launch with programmatic stream serialisation (the kernels wait for their
+// predecessor with griddepcontrol.wait before touching memory)
+template <typename... KArgs, typename... Args>
+cudaError_t pdl_launch(void (*kernel)(KArgs...), int grid, int block, size_t smem, cudaStream_t s,
+                       Args... args) {
+  static const bool pdl = getenv("HKV_NO_PDL") == nullptr;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(block);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
+int max_len_of(size_t smem, int D) {
+  return (int)((smem - (size_t)D * 4 - 512 * 4 - 64) / 16);
+}
+
 }  // namespace
 
 size_t update_smem_bytes(int max_len, int D) {
-  // keys (8 B) + destinations (4 B) per row, q-bar, two 256-bin histograms
-  return (size_t)max_len * 12 + (size_t)D * 4 + 512 * 4 + 64;
+  // keys (8 B), positions (4 B), class/flag/rank (4 B) per row; q-bar; two
+  // 256-bin histograms
+  return (size_t)max_len * 16 + (size_t)D * 4 + 512 * 4 + 64;
 }
 
 cudaError_t update_prepare(int D, int dtype, size_t smem) {
@@ -567,35 +733,45 @@ cudaError_t update_prepare(int D, int dtype, size_t smem) {
 cudaError_t launch_append_evict(const CacheArgs &c, const MethodArgs &m, int layer_base,
                                 int nheads, const void *q, const void *k, const void *v, int D,
                                 int dtype, size_t smem, cudaStream_t s) {
-  const int max_len = (int)((smem - (size_t)D * 4 - 512 * 4 - 64) / 12);
+  const int max_len = max_len_of(smem, D);
   HKV_DISPATCH(D, dtype,
-               (append_evict_kernel<kD, kT><<<nheads, NT, smem, s>>>(c, m, layer_base, q, k, v,
-                                                                    max_len)));
-  return cudaGetLastError();
+               return pdl_launch(append_evict_kernel<kD, kT>, nheads, NT, smem, s, c, m,
+                                 layer_base, q, k, v, max_len));
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_evict(const CacheArgs &c, const MethodArgs &m, int layer_base, int nheads,
+                         int D, int dtype, size_t smem, cudaStream_t s) {
+  const int max_len = max_len_of(smem, D);
+  HKV_DISPATCH(D, dtype,
+               return pdl_launch(evict_kernel<kD, kT>, nheads, NT, smem, s, c, m, layer_base,
+                                 max_len));
+  return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_repack(const CacheArgs &dense, const CacheArgs &ragged, const MethodArgs &m,
                           int layer_base, int nheads, int D, int dtype, size_t smem,
                           cudaStream_t s) {
-  const int max_len = (int)((smem - (size_t)D * 4 - 512 * 4 - 64) / 12);
+  const int max_len = max_len_of(smem, D);
   HKV_DISPATCH(D, dtype,
-               (repack_kernel<kD, kT><<<nheads, NT, smem, s>>>(dense, ragged, m, layer_base,
-                                                              max_len)));
-  return cudaGetLastError();
+               return pdl_launch(repack_kernel<kD, kT>, nheads, NT, smem, s, dense, ragged, m,
+                                 layer_base, max_len));
+  return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_prefill(const CacheArgs &c, int layer_base, int nheads, int C, const void *kc,
                            const void *vc, int D, int dtype, cudaStream_t s) {
-  HKV_DISPATCH(D, dtype, (prefill_kernel<kD, kT><<<nheads, 128, 0, s>>>(c, layer_base, C, kc, vc)));
-  return cudaGetLastError();
+  HKV_DISPATCH(D, dtype,
+               return pdl_launch(prefill_kernel<kD, kT>, nheads, 128, 0, s, c, layer_base, C, kc,
+                                 vc));
+  return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_init_dense(const CacheArgs &c, int n, int seg, cudaStream_t s) {
   int grid = (n + 255) / 256;
   if (grid > 4096) grid = 4096;
   if (grid < 1) grid = 1;
-  init_dense_kernel<<<grid, 256, 0, s>>>(c, n, seg);
-  return cudaGetLastError();
+  return pdl_launch(init_dense_kernel, grid, 256, 0, s, c, n, seg);
 }
 
 cudaError_t launch_identify(const CacheArgs &c, const MethodArgs &m, int layer_base, int nheads,
@@ -604,15 +780,14 @@ cudaError_t launch_identify(const CacheArgs &c, const MethodArgs &m, int layer_b
   const float qscale = (float)(1.4426950408889634 / sqrt((double)D));
   const size_t smem = (size_t)max_len * 4;
   HKV_DISPATCH(D, dtype,
-               (identify_kernel<kD, kT><<<nheads, NT, smem, s>>>(c, m, layer_base, q, label_out,
-                                                                nh_out, qscale, max_len)));
-  return cudaGetLastError();
+               return pdl_launch(identify_kernel<kD, kT>, nheads, NT, smem, s, c, m, layer_base,
+                                 q, label_out, nh_out, qscale, max_len));
+  return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_budgets(const uint8_t *label, int32_t *budget, int32_t *cap, int64_t *off,
                            int n, int C, int B_g, int w, int P, cudaStream_t s) {
-  budgets_kernel<<<1, 1024, 0, s>>>(label, budget, cap, off, n, C, B_g, w, P);
-  return cudaGetLastError();
+  return pdl_launch(budgets_kernel, 1, 1024, 0, s, label, budget, cap, off, n, C, B_g, w, P);
 }
 
 }  // namespace hkv

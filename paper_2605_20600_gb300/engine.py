@@ -82,6 +82,25 @@ class Engine:
         H.hkv_decode_attention(self.cfg, self.cache.c, layer, q, out, self.ws, self.ws_bytes,
                                self.stream())
 
+    # fused path: the update when due, then append + attention in one launch
+    def evict(self, layer: int) -> None:
+        H.hkv_evict(self.cfg, self.cache.c, layer, self.stream())
+
+    def step(self, layer: int, q, k, v, out) -> None:
+        # layers run in order, so with two or more layers the kernel before a
+        # decode step belongs to another layer (or is hkv_evict, which never
+        # lets its successor start early): the step may prefetch
+        flags = H.HKV_STEP_PREFETCH if self.cfg.n_layers >= 2 else 0
+        H.hkv_decode_step(self.cfg, self.cache.c, layer, q, k, v, out, self.ws, self.ws_bytes,
+                          flags, self.stream())
+
+    def update_due(self, t: int) -> bool:
+        """Whether image token t's step starts with the periodic update: the
+        buffer filled P steps after grouping (image token E-1) and every P
+        steps since."""
+        E, P = self.cfg.group_at, self.cfg.period
+        return t > E and (t - E) % P == 0
+
     # Step 2
     def identify(self, layer: int, q) -> None:
         H.hkv_identify_heads(self.cfg, self.dense.c, layer, q, self.labels, self.n_h, self.stream())

@@ -28,6 +28,7 @@ HKV_ERR_CUDA = 7
 HKV_ERR_ALIGN = 8
 
 HKV_FP32, HKV_BF16 = 0, 1
+HKV_STEP_PREFETCH = 1
 HKV_LOCAL, HKV_GLOBAL, HKV_DENSE = 0, 1, 255
 
 
@@ -67,6 +68,9 @@ _SIGNATURES = {
                           c_void_p], c_int),
     "hkv_decode_attention": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p, c_void_p, c_void_p,
                               c_size_t, c_void_p], c_int),
+    "hkv_decode_step": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p, c_void_p, c_void_p,
+                         c_void_p, c_void_p, c_size_t, c_int, c_void_p], c_int),
+    "hkv_evict": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p], c_int),
     "hkv_identify_heads": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p, c_void_p, c_void_p,
                             c_void_p], c_int),
     "hkv_allocate_budgets": ([POINTER(hkv_config), c_void_p, c_void_p, c_void_p, c_void_p,
@@ -145,6 +149,16 @@ def hkv_append_evict(cfg, cache, layer, q, k, v, stream=0) -> None:
 def hkv_decode_attention(cfg, cache, layer, q, out, workspace, ws_bytes, stream=0) -> None:
     _call("decode_attention", ctypes.byref(cfg), ctypes.byref(cache), layer, _p(q), _p(out),
           _p(workspace), ws_bytes, stream)
+
+
+def hkv_decode_step(cfg, cache, layer, q, k, v, out, workspace, ws_bytes, flags=0,
+                    stream=0) -> None:
+    _call("decode_step", ctypes.byref(cfg), ctypes.byref(cache), layer, _p(q), _p(k), _p(v), _p(out),
+          _p(workspace), ws_bytes, flags, stream)
+
+
+def hkv_evict(cfg, cache, layer, stream=0) -> None:
+    _call("evict", ctypes.byref(cfg), ctypes.byref(cache), layer, stream)
 
 
 def hkv_identify_heads(cfg, cache, layer, q, label_out, nh_out=None, stream=0) -> None:

@@ -14,18 +14,21 @@ from .engine import Engine, torch_dtype
 
 
 def generate(engine: Engine, provider, *, last_step: int | None = None, on_step=None,
-             before_compress=None) -> None:
-    """Runs image tokens 0..last_step (default N-1) for every layer.
+             before_compress=None, fused: bool = True, first_step: int = 0) -> None:
+    """Runs image tokens first_step..last_step (default N-1) for every layer.
 
+    fused: per layer and step, hkv_evict when the update is due and then
+    hkv_decode_step; otherwise hkv_append_evict then hkv_decode_attention.
     on_step(t, out) receives out [L][S][H][D] (fp32, device) after step t.
     before_compress(engine) runs after grouping, before budgets and repack.
+    first_step > 0 continues a generation (the prefill is skipped).
     """
     cfg = engine.cfg
     L, S, H, D, C = cfg.n_layers, cfg.n_seqs, cfg.n_heads, cfg.head_dim, cfg.n_cond
     E = cfg.group_at
     dev, dt = engine.device, torch_dtype(cfg)
     st = engine.stream()
-    if C > 0:
+    if C > 0 and first_step == 0:
         kc = torch.empty(S, H, C, D, dtype=dt, device=dev)
         vc = torch.empty_like(kc)
         for layer in range(L):
@@ -35,11 +38,17 @@ def generate(engine: Engine, provider, *, last_step: int | None = None, on_step=
     k, v = torch.empty_like(q), torch.empty_like(q)
     out = torch.empty(L, S, H, D, dtype=torch.float32, device=dev)
     last = cfg.n_image - 1 if last_step is None else last_step
-    for t in range(last + 1):
+    for t in range(first_step, last + 1):
         provider.image(q, k, v, 0, L, t, 1, st)
+        due = engine.update_due(t)
         for layer in range(L):
-            engine.append(layer, q[layer], k[layer], v[layer])
-            engine.attend(layer, q[layer], out[layer])
+            if fused:
+                if due:
+                    engine.evict(layer)
+                engine.step(layer, q[layer], k[layer], v[layer], out[layer])
+            else:
+                engine.append(layer, q[layer], k[layer], v[layer])
+                engine.attend(layer, q[layer], out[layer])
             if t == E - 1:
                 engine.identify(layer, q[layer])
         if on_step is not None:

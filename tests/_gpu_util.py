@@ -22,9 +22,9 @@ def flat(w, s, l, h):
     return (l * w.n_seqs + s) * w.n_heads + h
 
 
-def run_gpu(w, *, out_steps=(), pos_steps=(), pos_heads=(), last_step=None):
+def run_gpu(w, *, out_steps=(), pos_steps=(), pos_heads=(), last_step=None, fused=True):
     """One generation on the GPU. Returns outputs {t: [L,S,H,D] fp32},
-    positions {t: {flat head: positions}}, labels, n_h and the engine."""
+    positions {t: {flat head: sorted positions}}, labels, n_h and the engine."""
     import torch
     from paper_2605_20600_gb300 import hkv as H
     from paper_2605_20600_gb300.engine import Engine
@@ -42,10 +42,10 @@ def run_gpu(w, *, out_steps=(), pos_steps=(), pos_heads=(), last_step=None):
             c = eng.cache
             off, ln = c.off.cpu().numpy(), c.len.cpu().numpy()
             allpos = c.pos
-            poss[t] = {i: allpos[int(off[i]): int(off[i]) + int(ln[i])].cpu().numpy()
+            poss[t] = {i: np.sort(allpos[int(off[i]): int(off[i]) + int(ln[i])].cpu().numpy())
                        for i in pos_heads}
 
-    generate(eng, DeviceSynth(w, "cuda"), on_step=on_step, last_step=last_step)
+    generate(eng, DeviceSynth(w, "cuda"), on_step=on_step, last_step=last_step, fused=fused)
     torch.cuda.synchronize()
     eng.check()
     return outs, poss, eng.labels.cpu().numpy(), eng.n_h.cpu().numpy(), eng

@@ -47,7 +47,7 @@ def fake_cache(H, **kw):
 
 def test_every_declared_symbol_is_exported(H):
     names = declared_functions()
-    assert len(names) == 12
+    assert len(names) == 14
     for n in names:
         assert hasattr(H.lib(), n), n
     assert set(names) >= {"hkv_identify_heads", "hkv_allocate_budgets", "hkv_append_evict",
@@ -120,10 +120,16 @@ def test_null_and_misaligned_arguments(H):
     assert lib.hkv_repack(ctypes.byref(cfg), ctypes.byref(c), ctypes.byref(other), 0, None) == 1
     assert lib.hkv_allocate_budgets(ctypes.byref(cfg), None, 16, 16, 16, None, None) == 1
     assert lib.hkv_check(None, None) == 1
+    assert lib.hkv_decode_step(ctypes.byref(cfg), ctypes.byref(c), 0, 16, None, 16, 16, 16, 1 << 30, 0, None) == 1
+    assert lib.hkv_decode_step(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, 16, 16, 16, 8, 0, None) == 3
+    assert lib.hkv_decode_step(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 24, 16, 16, 16, 1 << 30, 0, None) == 8
+    assert lib.hkv_decode_step(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, 16, 16, 16, 1 << 30, 6, None) == 1
+    assert lib.hkv_evict(ctypes.byref(cfg), ctypes.byref(c), 5, None) == 1
 
 
 @pytest.mark.parametrize("name", ["decode_attention", "append_evict", "identify_heads",
-                                  "allocate_budgets", "repack", "prefill", "init_dense", "check"])
+                                  "allocate_budgets", "repack", "prefill", "init_dense", "check",
+                                  "decode_step", "evict"])
 def test_fault_injection_returns_the_code(H, name, monkeypatch):
     cfg = tiny_cfg(H)
     c = fake_cache(H)
@@ -138,6 +144,8 @@ def test_fault_injection_returns_the_code(H, name, monkeypatch):
         "prefill": lambda: lib.hkv_prefill(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, None),
         "init_dense": lambda: lib.hkv_init_dense(ctypes.byref(cfg), ctypes.byref(c), None),
         "check": lambda: lib.hkv_check(ctypes.byref(c), None),
+        "decode_step": lambda: lib.hkv_decode_step(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, 16, 16, 16, 1 << 30, 0, None),
+        "evict": lambda: lib.hkv_evict(ctypes.byref(cfg), ctypes.byref(c), 0, None),
     }
     assert calls[name]() == 6
 

@@ -60,3 +60,45 @@ def test_prefill_twice_is_a_state_error():
     with pytest.raises(H.HkvError) as e:
         eng.check()
     assert e.value.status == H.HKV_ERR_STATE
+
+
+def test_decode_step_refuses_a_due_update():
+    """hkv_decode_step on a head whose buffer is full (hkv_evict skipped)
+    reports a state error and takes no step; hkv_evict then unblocks it."""
+    import torch
+    from paper_2605_20600_gb300.runner import generate
+    from synth.gpu import DeviceSynth
+    H, eng, w = small_engine()
+    E, P = w.group_at, w.period
+    generate(eng, DeviceSynth(w, "cuda"), last_step=E + P - 1)       # buffer now full
+    eng.check()
+    ln = eng.cache.len.clone()
+    q = torch.zeros(w.n_seqs, w.n_heads, w.head_dim, device="cuda")
+    out = torch.zeros(w.n_seqs, w.n_heads, w.head_dim, device="cuda")
+    eng.step(0, q, q, q, out)
+    with pytest.raises(H.HkvError) as e:
+        eng.check()
+    assert e.value.status == H.HKV_ERR_STATE
+    assert torch.equal(eng.cache.len, ln)
+    eng.cache.err.zero_()
+    eng.ws.zero_()
+    eng.evict(0)
+    eng.step(0, q, q, q, out)
+    eng.check()
+    assert (eng.cache.len.cpu() <= eng.cache.cap.cpu()).all()
+
+
+def test_evict_is_a_no_op_when_not_due():
+    from paper_2605_20600_gb300.runner import generate
+    from synth.gpu import DeviceSynth
+    H, eng, w = small_engine()
+    generate(eng, DeviceSynth(w, "cuda"), last_step=w.group_at + 2)
+    before = (eng.cache.len.clone(), eng.cache.pos.clone(), eng.cache.k.clone())
+    eng.evict(0)
+    eng.check()
+    assert torch_equal_all(before, (eng.cache.len, eng.cache.pos, eng.cache.k))
+
+
+def torch_equal_all(a, b):
+    import torch
+    return all(torch.equal(x, y) for x, y in zip(a, b))

@@ -40,7 +40,8 @@ class HandProvider:
             v[0, 0].copy_(self.v[:, self.C + t])
 
 
-def test_hand_worked_grid_on_gpu():
+@pytest.mark.parametrize("fused", [True, False])
+def test_hand_worked_grid_on_gpu(fused):
     import torch
     from paper_2605_20600_gb300 import hkv as H
     from paper_2605_20600_gb300.engine import Engine
@@ -58,10 +59,11 @@ def test_hand_worked_grid_on_gpu():
     def on_step(t, out):
         cc = eng.cache
         off, ln = cc.off.cpu().numpy(), cc.len.cpu().numpy()
-        pos_at[t] = [cc.pos[int(off[h]): int(off[h]) + int(ln[h])].cpu().numpy() for h in range(2)]
+        pos_at[t] = [np.sort(cc.pos[int(off[h]): int(off[h]) + int(ln[h])].cpu().numpy())
+                     for h in range(2)]
         outs[t] = out.cpu().numpy()[0, 0]
 
-    generate(eng, HandProvider(heads, c["n_cond"], "cuda"), on_step=on_step)
+    generate(eng, HandProvider(heads, c["n_cond"], "cuda"), on_step=on_step, fused=fused)
     eng.check()
     labels, nh = eng.labels.cpu().numpy(), eng.n_h.cpu().numpy()
     hp = O.HeadParams(n_cond=c["n_cond"], n_image=c["n_image"], recent_w=c["recent_w"],
@@ -84,12 +86,13 @@ def test_hand_worked_grid_on_gpu():
             assert np.abs(outs[t][h] - tr.outputs[t]).max() < 1e-5, (hd["name"], t)
 
 
-def test_tiny_every_step_every_head():
+@pytest.mark.parametrize("fused", [True, False])
+def test_tiny_every_step_every_head(fused):
     w = configs.TINY
     N = w.n_image
     heads = [(0, 0, h) for h in range(w.n_heads)]
     outs, poss, labels, nh, eng = run_gpu(w, out_steps=range(N), pos_steps=range(N),
-                                          pos_heads=[flat(w, *x) for x in heads])
+                                          pos_heads=[flat(w, *x) for x in heads], fused=fused)
     lab = oracle_labels(w, [0], [0])
     ties = check_labels(w, labels, nh, lab, "tiny")
     assert not ties
@@ -113,19 +116,20 @@ def sampled_steps(w, rng, extra=12):
     return sorted(x for x in s if 0 <= x < N)
 
 
-REDUCED = [("lumina768", "1/4"), ("lumina1024", "1/4"), ("lumina1024", "1/6"),
-           ("lumina1024", "1/8"), ("llamagen_xl", "1/6"), ("janus_pro_7b", "1/8")]
+REDUCED = [("lumina768", "1/4", True), ("lumina1024", "1/4", True), ("lumina1024", "1/6", True),
+           ("lumina1024", "1/8", True), ("llamagen_xl", "1/6", True), ("janus_pro_7b", "1/8", True),
+           ("lumina1024", "1/8", False), ("llamagen_xl", "1/6", False)]
 
 
-@pytest.mark.parametrize("name,rho", REDUCED)
-def test_model_shapes_two_layers_two_seqs(name, rho):
+@pytest.mark.parametrize("name,rho,fused", REDUCED)
+def test_model_shapes_two_layers_two_seqs(name, rho, fused):
     from fractions import Fraction
     w = configs.ALL[name].with_(n_layers=2, n_seqs=2, rho=Fraction(rho))
     rng = np.random.default_rng(42)
     steps = sampled_steps(w, rng)
     heads = [(s, l, h) for l in range(w.n_layers) for s in range(w.n_seqs) for h in range(w.n_heads)]
     outs, poss, labels, nh, eng = run_gpu(w, out_steps=steps, pos_steps=steps,
-                                          pos_heads=[flat(w, *x) for x in heads])
+                                          pos_heads=[flat(w, *x) for x in heads], fused=fused)
     lab = oracle_labels(w, range(w.n_layers), range(w.n_seqs))
     ties = check_labels(w, labels, nh, lab, name)
     assert len(ties) <= 2, ties
