@@ -12,11 +12,13 @@
 //    heads (one round of loads), a block scan finds the CTA's first head,
 //    and a table of the next heads' (offset, length, start) goes to shared
 //    memory;
-//  * warp-specialised pipeline: one producer warp streams K/V tiles of 8 KB
+//  * warp-specialised pipeline: one producer warp streams K/V tiles of 7 KB
 //    into shared memory with the TMA engine (1D cp.async.bulk) through
 //    NS stages guarded by full/empty mbarriers; the query row of a head rides
 //    along with the head's first tile; consumer warps never wait on the
-//    producer's issue work;
+//    producer's issue work; an epilogue warp finishes each head segment
+//    (merge of the consumer warps' states, output or partial result,
+//    combine) while the consumers stream on;
 //  * consumers take whole token rows with 16-byte lanes (a 256-byte bf16 row
 //    is 16 lanes), a shuffle-xor tree per row for q.k, online softmax in the
 //    log2 domain with fp32 accumulation;
@@ -46,7 +48,7 @@ namespace {
 // Tuning knobs (compile time): bytes of K per pipeline stage, stages, and
 // a cap on resident CTAs per SM used to size the grid.
 #ifndef HKV_ATTN_TILE_BYTES
-#define HKV_ATTN_TILE_BYTES 8192
+#define HKV_ATTN_TILE_BYTES 7168
 #endif
 #ifndef HKV_ATTN_STAGES
 #define HKV_ATTN_STAGES 4
@@ -56,6 +58,21 @@ namespace {
 #endif
 
 constexpr int kCW = kAttnConsumerWarps;
+
+// Phase timestamps per CTA for latency studies; compiled out by default.
+#ifdef HKV_ATTN_TRACE
+__device__ unsigned long long *g_trace = nullptr;  // [layer][kAttnMaxGrid][8], set by the tracer
+#define HKV_TRACE(slot)                                                  \
+  do {                                                                   \
+    if (g_trace)                                                         \
+      g_trace[((size_t)(p.layer_base / p.nheads) * kAttnMaxGrid + blockIdx.x) * 8 + (slot)] = \
+          globaltimer();                                                 \
+  } while (0)
+#else
+#define HKV_TRACE(slot) \
+  do {                  \
+  } while (0)
+#endif
 
 template <int D, typename T>
 struct AttnShape {
@@ -80,9 +97,11 @@ constexpr int kTable = 32;  // heads whose (offset, length, start) sit in smem
 struct HeadTable {
   int h0;                   // first head of the CTA's range
   int n;                    // valid entries
+  int covers;               // the entries cover the CTA's whole range
   long long start[kTable];  // global token index where head h0 + j starts
   long long off[kTable];    // arena offset of head h0 + j
   int vlen[kTable];         // virtual length (len + fused)
+  int ntok[kTable];         // image tokens appended so far (fused)
 };
 
 __device__ __forceinline__ void pdl_wait() {
@@ -90,11 +109,6 @@ __device__ __forceinline__ void pdl_wait() {
 }
 __device__ __forceinline__ void pdl_launch_dependents() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-}
-
-// barrier among the consumer warps only (named barrier 1)
-__device__ __forceinline__ void consumer_sync() {
-  asm volatile("bar.sync 1, %0;" ::"n"(kCW * 32) : "memory");
 }
 
 template <bool FUSED>
@@ -155,8 +169,11 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
 
   extern __shared__ __align__(128) unsigned char stages[];
   __shared__ uint64_t full[NS], empty[NS];
+  __shared__ uint64_t epi_full, epi_free;   // hand-over of one segment's states
   __shared__ float red_acc[kCW][D];
   __shared__ float red_m[kCW], red_l[kCW];
+  __shared__ int seg_h, seg_final;
+  __shared__ long long seg_hs, seg_he;
   __shared__ HeadTable tab;
   __shared__ long long scan_scratch[33];
   __shared__ long long s_s0;
@@ -167,10 +184,13 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
   const int nheads = p.nheads;
 
   if (tid == 0) {
+    HKV_TRACE(0);
     for (int s = 0; s < NS; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], kCW);
     }
+    mbar_init(&epi_full, kCW);
+    mbar_init(&epi_free, 1);
     fence_barrier_init();
     s_abort = 0;
   }
@@ -238,13 +258,43 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
     tab.start[lane] = s_s0 + incl - L;
     tab.off[lane] = h < nheads ? p.off[h] : 0;
     tab.vlen[lane] = (int)L;
+    tab.ntok[lane] = (FUSED && h < nheads) ? p.ntok[p.layer_base + h] : 0;
+    const int n = nheads - h0 < kTable ? nheads - h0 : kTable;
+    const long long end = __shfl_sync(0xFFFFFFFFu, s_s0 + incl, n - 1);
     if (lane == 0) {
       tab.h0 = h0;
-      tab.n = nheads - h0 < kTable ? nheads - h0 : kTable;
+      tab.n = n;
+      tab.covers = end >= b;
     }
   }
   __syncthreads();
+  // Fused: a CTA whose heads all sit in the table reads no length, position
+  // counter or buffer count after this point, so it can count itself on the
+  // grid counter as soon as the previous kernel is done (the counter lives in
+  // the shared workspace); the last CTA to count advances the counters. The
+  // other CTAs count at the end.
+  const bool early = FUSED && (!active || tab.covers);
 
+  if (tid == 0) HKV_TRACE(1);
+  auto grid_arrive = [&]() {  // block-wide; called after the wait
+    __syncthreads();
+    if (tid == 0) {
+      __threadfence();
+      s_last = atomicAdd(p.gcnt, 1) == (int)gridDim.x - 1;
+    }
+    __syncthreads();
+    if (s_last) {
+      __threadfence();
+      for (int h = tid; h < nheads; h += kAttnThreads) {
+        const int i = p.layer_base + h;
+        p.len[h] += 1;
+        p.ntok[i] += 1;
+        if (p.label[i] != HKV_DENSE) p.nbuf[i] += 1;
+      }
+      if (tid == 0) *p.gcnt = 0;
+    }
+    __syncthreads();
+  };
   const HeadLookup<FUSED> look{tab, p};
   TileIter cit;
   cit.h = tab.h0;
@@ -253,57 +303,86 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
   cit.g = a;
   cit.b = b;
 
+  // ---- producer state (warp 0, lane 0) ----------------------------------
+  // A tile's old rows come from the arena; the query row (first tile of a
+  // head here) and the new token's K/V (fused, last tile of a head) come from
+  // this step's inputs, which may be written by the previous kernel.
+  const bool producer = active && tid == 0;
+  TileIter pit = cit;
+  int issued = 0;
+  auto issue_old = [&](Pending &pd) {  // expect + copy the arena rows, no arrival
+    const int stage = issued % NS;
+    const long long ge = pit.tile_end(TT);
+    const int r0 = (int)(pit.g - pit.hs), r1 = (int)(ge - pit.hs);   // head-local rows
+    const int real = FUSED ? pit.hl - 1 : pit.hl;                    // rows in the arena
+    const int n_old = (r1 < real ? r1 : real) - r0;
+    unsigned char *dk = stages + stage * S::kStageBytes;
+    pd.h = pit.h;
+    pd.slot_new = real - r0;
+    pd.first = pit.g == pit.hs || pit.g == a;
+    pd.has_new = FUSED && r1 == pit.hl;
+    if (n_old > 0) {
+      const uint32_t bytes = (uint32_t)n_old * RB;
+      const long long row = look.off(pit.h) + r0;
+      mbar_expect_tx(&full[stage], 2 * bytes);
+      bulk_g2s(dk, static_cast<const unsigned char *>(p.K) + row * RB, bytes, &full[stage]);
+      bulk_g2s(dk + TT * RB, static_cast<const unsigned char *>(p.V) + row * RB, bytes,
+               &full[stage]);
+    }
+    pit.advance(TT, look);
+    ++issued;
+  };
+  auto issue_extra = [&](const Pending &pd, int stage) {  // inputs, then arrive
+    unsigned char *dk = stages + stage * S::kStageBytes;
+    unsigned char *dv = dk + TT * RB;
+    mbar_arrive_expect_tx(&full[stage], (pd.has_new ? 2 * RB : 0) + (pd.first ? RB : 0));
+    if (pd.has_new) {
+      bulk_g2s(dk + pd.slot_new * RB,
+               static_cast<const unsigned char *>(p.k_new) + (size_t)pd.h * RB, RB, &full[stage]);
+      bulk_g2s(dv + pd.slot_new * RB,
+               static_cast<const unsigned char *>(p.v_new) + (size_t)pd.h * RB, RB, &full[stage]);
+    }
+    if (pd.first)
+      bulk_g2s(dv + TT * RB, static_cast<const unsigned char *>(p.q) + (size_t)pd.h * RB, RB,
+               &full[stage]);
+  };
+  Pending pre[NS];
+  int n_pre = 0;
+  if (producer)
+    for (; n_pre < NS && !pit.done(); ++n_pre) issue_old(pre[n_pre]);
+
+  if (p.prefetch) pdl_wait();  // the step's inputs are visible from here on
+  if (tid == 0) HKV_TRACE(2);
+  pdl_launch_dependents();
+  if (early) grid_arrive();
+
+  // Fused append of a head's new token (row, position, query) by the warp
+  // that finishes the head; nothing in this launch reads them.
+  auto append_row = [&](int h) {
+    const int i = p.layer_base + h;
+    const int jt = h - tab.h0;
+    const bool in_tab = jt >= 0 && jt < tab.n;
+    const int len = (in_tab ? tab.vlen[jt] : p.len[h] + 1) - 1;
+    const int nt = in_tab ? tab.ntok[jt] : p.ntok[i];
+    const long long row = look.off(h) + len;
+    const uint4 *ks = reinterpret_cast<const uint4 *>(static_cast<const unsigned char *>(p.k_new) + (size_t)h * RB);
+    const uint4 *vs = reinterpret_cast<const uint4 *>(static_cast<const unsigned char *>(p.v_new) + (size_t)h * RB);
+    const uint4 *qs = reinterpret_cast<const uint4 *>(static_cast<const unsigned char *>(p.q) + (size_t)h * RB);
+    uint4 *kd = reinterpret_cast<uint4 *>(static_cast<unsigned char *>(p.K) + row * RB);
+    uint4 *vd = reinterpret_cast<uint4 *>(static_cast<unsigned char *>(p.V) + row * RB);
+    uint4 *qd = reinterpret_cast<uint4 *>(static_cast<unsigned char *>(p.qbuf) +
+                                          ((size_t)i * p.period + nt % p.period) * RB);
+    for (int c = lane; c < RB / 16; c += 32) {
+      kd[c] = ks[c];
+      vd[c] = vs[c];
+      qd[c] = qs[c];
+    }
+    if (lane == 0) p.pos[row] = p.n_cond + nt;
+  };
+
   if (warp == 0) {
     // ---- producer ----------------------------------------------------------
-    // A tile's old rows come from the arena; the query row (first tile of a
-    // head here) and the new token's K/V (fused, last tile of a head) come
-    // from this step's inputs, which may be written by the previous kernel.
-    if (active && lane == 0) {
-      TileIter pit = cit;
-      int issued = 0;
-      auto issue_old = [&](Pending &pd) {  // expect + copy the arena rows, no arrival
-        const int stage = issued % NS;
-        const long long ge = pit.tile_end(TT);
-        const int r0 = (int)(pit.g - pit.hs), r1 = (int)(ge - pit.hs);   // head-local rows
-        const int real = FUSED ? pit.hl - 1 : pit.hl;                    // rows in the arena
-        const int n_old = (r1 < real ? r1 : real) - r0;
-        unsigned char *dk = stages + stage * S::kStageBytes;
-        pd.h = pit.h;
-        pd.slot_new = real - r0;
-        pd.first = pit.g == pit.hs || pit.g == a;
-        pd.has_new = FUSED && r1 == pit.hl;
-        if (n_old > 0) {
-          const uint32_t bytes = (uint32_t)n_old * RB;
-          const long long row = look.off(pit.h) + r0;
-          mbar_expect_tx(&full[stage], 2 * bytes);
-          bulk_g2s(dk, static_cast<const unsigned char *>(p.K) + row * RB, bytes, &full[stage]);
-          bulk_g2s(dk + TT * RB, static_cast<const unsigned char *>(p.V) + row * RB, bytes,
-                   &full[stage]);
-        }
-        pit.advance(TT, look);
-        ++issued;
-      };
-      auto issue_extra = [&](const Pending &pd, int stage) {  // inputs, then arrive
-        unsigned char *dk = stages + stage * S::kStageBytes;
-        unsigned char *dv = dk + TT * RB;
-        mbar_arrive_expect_tx(&full[stage], (pd.has_new ? 2 * RB : 0) + (pd.first ? RB : 0));
-        if (pd.has_new) {
-          bulk_g2s(dk + pd.slot_new * RB,
-                   static_cast<const unsigned char *>(p.k_new) + (size_t)pd.h * RB, RB,
-                   &full[stage]);
-          bulk_g2s(dv + pd.slot_new * RB,
-                   static_cast<const unsigned char *>(p.v_new) + (size_t)pd.h * RB, RB,
-                   &full[stage]);
-        }
-        if (pd.first)
-          bulk_g2s(dv + TT * RB, static_cast<const unsigned char *>(p.q) + (size_t)pd.h * RB, RB,
-                   &full[stage]);
-      };
-      Pending pre[NS];
-      int n_pre = 0;
-      for (; n_pre < NS && !pit.done(); ++n_pre) issue_old(pre[n_pre]);
-      if (p.prefetch) pdl_wait();  // the step's inputs are visible from here on
-      pdl_launch_dependents();
+    if (producer) {
 #pragma unroll
       for (int j = 0; j < NS; ++j)
         if (j < n_pre) issue_extra(pre[j], j);
@@ -319,15 +398,10 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
         issue_old(pd);
         issue_extra(pd, stage);
       }
-    } else {
-      if (p.prefetch) pdl_wait();
-      pdl_launch_dependents();
     }
-  } else {
+  } else if (warp <= kCW) {
     // ---- consumers ---------------------------------------------------------
     const int ctid = tid - 32, cw = warp - 1;
-    if (p.prefetch) pdl_wait();
-    pdl_launch_dependents();
     if (!FUSED && blockIdx.x == 0)  // empty heads (plain attention) are zeros
       for (int h = ctid; h < nheads; h += kCW * 32)
         if (p.len[h] == 0)
@@ -337,6 +411,7 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
       const int grp = lane / LPR, col = lane % LPR;
       float q[EPL], acc[EPL];
       float m = -INFINITY, l = 0.f;
+      int nseg = 0;
 #pragma unroll
       for (int e = 0; e < EPL; ++e) acc[e] = 0.f;
 
@@ -346,6 +421,7 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
           s_abort = 1;
           set_err(p.err, HKV_ERR_TIMEOUT);
         }
+        if (tile == 0 && ctid == 0) HKV_TRACE(3);
         const long long ge = cit.tile_end(TT);
         const int n = (int)(ge - cit.g);
         const long long he = cit.hs + cit.hl;
@@ -402,8 +478,9 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&empty[stage]);  // this warp is done with the stage
+        if (ctid == 0 && ge == b) HKV_TRACE(4);
 
-        if (ge == (b < he ? b : he)) {  // last tile of this head here: finish it
+        if (ge == (b < he ? b : he)) {  // last tile of this head here: hand it over
 #pragma unroll
           for (int o = LPR; o < 32; o <<= 1) {  // merge the row groups of the warp
             const float m2 = __shfl_xor_sync(0xFFFFFFFFu, m, o);
@@ -419,6 +496,11 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
             }
             m = mx;
           }
+          // the epilogue is done with the previous segment's states
+          if (nseg > 0 && !s_abort && !mbar_wait(&epi_free, (uint32_t)(nseg - 1) & 1u)) {
+            s_abort = 1;
+            set_err(p.err, HKV_ERR_TIMEOUT);
+          }
           if (lane < LPR) {
 #pragma unroll
             for (int e = 0; e < EPL; ++e) red_acc[cw][lane * EPL + e] = acc[e];
@@ -427,113 +509,101 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
               red_l[cw] = l;
             }
           }
-          consumer_sync();
-          const int h = cit.h;
-          const long long hs = cit.hs;
-          const bool whole = hs >= a && he <= b;
-          if (ctid < D) {
-            float mx = red_m[0];
-#pragma unroll
-            for (int w = 1; w < kCW; ++w) mx = fmaxf(mx, red_m[w]);
-            float L = 0.f, A = 0.f;
-#pragma unroll
-            for (int w = 0; w < kCW; ++w) {
-              const float s = red_m[w] == -INFINITY ? 0.f : exp2f(red_m[w] - mx);
-              L += red_l[w] * s;
-              A += red_acc[w][ctid] * s;
-            }
-            if (whole) {
-              p.out[(size_t)h * D + ctid] = A / L;
-            } else {
-              float *pp = p.part + ((size_t)blockIdx.x * 2 + (hs <= a ? 0 : 1)) * (D + 2);
-              pp[ctid] = A;
-              if (ctid == 0) {
-                pp[D] = mx;
-                pp[D + 1] = L;
-              }
-            }
+          if (cw == 0 && lane == 0) {
+            seg_h = cit.h;
+            seg_hs = cit.hs;
+            seg_he = he;
+            seg_final = ge == b;
           }
-          bool finisher = whole;
-          if (!whole) {
-            consumer_sync();
-            const long long c0 = hs / chunk, c1 = (he - 1) / chunk;
-            if (ctid == 0) {
-              __threadfence();
-              s_last = atomicAdd(&p.cnt[h], 1) == (int)(c1 - c0);
-            }
-            consumer_sync();
-            finisher = s_last;
-            if (finisher) {
-              __threadfence();
-              if (ctid < D) {
-                float mx = -INFINITY, L = 0.f, A = 0.f;
-                for (long long c = c0; c <= c1; ++c) {  // online merge in CTA order
-                  const int slot = (c == c0 && c * chunk < hs) ? 1 : 0;
-                  const float *pp = p.part + ((size_t)c * 2 + slot) * (D + 2);
-                  const float mc = __ldcg(pp + D), lc = __ldcg(pp + D + 1), ac = __ldcg(pp + ctid);
-                  const float mn2 = fmaxf(mx, mc);
-                  const float s0 = mx == -INFINITY ? 0.f : exp2f(mx - mn2);
-                  const float s1 = exp2f(mc - mn2);
-                  L = L * s0 + lc * s1;
-                  A = A * s0 + ac * s1;
-                  mx = mn2;
-                }
-                p.out[(size_t)h * D + ctid] = A / L;
-              }
-              if (ctid == 0) p.cnt[h] = 0;
-            }
-          }
-          if (FUSED && finisher) {
-            // append: the new token's row, position and query (read by no CTA
-            // of this launch, so any time is safe); counters advance at the end
-            const int i = p.layer_base + h;
-            const int len = cit.hl - 1;
-            const long long row = look.off(h) + len;
-            const int nt = p.ntok[i];
-            for (int pc = ctid; pc < 3 * (RB / 16); pc += kCW * 32) {
-              const int which = pc / (RB / 16), c16 = (pc % (RB / 16)) * 16;
-              const unsigned char *src = static_cast<const unsigned char *>(
-                  which == 0 ? p.k_new : which == 1 ? p.v_new : p.q) + (size_t)h * RB + c16;
-              unsigned char *dst =
-                  which == 0 ? static_cast<unsigned char *>(p.K) + row * RB + c16
-                  : which == 1 ? static_cast<unsigned char *>(p.V) + row * RB + c16
-                  : static_cast<unsigned char *>(p.qbuf) + ((size_t)i * p.period + nt % p.period) * RB + c16;
-              *reinterpret_cast<uint4 *>(dst) = *reinterpret_cast<const uint4 *>(src);
-            }
-            if (ctid == 0) p.pos[row] = p.n_cond + nt;
-          }
-          consumer_sync();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&epi_full);
+          ++nseg;
         }
         cit.advance(TT, look);
       }
+      if (ctid == 0) HKV_TRACE(5);
       if (s_abort && ctid == 0)  // drain what may still be in flight (bounded)
         for (int s = 0; s < NS; ++s) {
           mbar_wait(&full[s], 0);
           mbar_wait(&full[s], 1);
         }
     }
+  } else if (active) {
+    // ---- epilogue: finish each head segment the consumers hand over --------
+    constexpr int CPL = D / 32;  // output channels per lane
+    for (int k = 0;; ++k) {
+      if (!s_abort && !mbar_wait(&epi_full, (uint32_t)k & 1u)) {
+        s_abort = 1;
+        set_err(p.err, HKV_ERR_TIMEOUT);
+      }
+      if (s_abort) break;
+      const int h = seg_h;
+      const long long hs = seg_hs, he = seg_he;
+      const int fin = seg_final;
+      float mx = red_m[0];
+#pragma unroll
+      for (int w = 1; w < kCW; ++w) mx = fmaxf(mx, red_m[w]);
+      float L = 0.f, A[CPL];
+#pragma unroll
+      for (int c = 0; c < CPL; ++c) A[c] = 0.f;
+#pragma unroll
+      for (int w = 0; w < kCW; ++w) {
+        const float sw = red_m[w] == -INFINITY ? 0.f : exp2f(red_m[w] - mx);
+        L += red_l[w] * sw;
+#pragma unroll
+        for (int c = 0; c < CPL; ++c) A[c] += red_acc[w][lane + 32 * c] * sw;
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&epi_free);  // the consumers may reuse the slot
+      if (hs >= a && he <= b) {  // the whole head is here
+#pragma unroll
+        for (int c = 0; c < CPL; ++c) p.out[(size_t)h * D + lane + 32 * c] = A[c] / L;
+        if (FUSED) append_row(h);
+      } else {
+        float *pp = p.part + ((size_t)blockIdx.x * 2 + (hs <= a ? 0 : 1)) * (D + 2);
+#pragma unroll
+        for (int c = 0; c < CPL; ++c) pp[lane + 32 * c] = A[c];
+        if (lane == 0) {
+          pp[D] = mx;
+          pp[D + 1] = L;
+        }
+        __syncwarp();
+        const long long c0 = hs / chunk, c1 = (he - 1) / chunk;
+        int last = 0;
+        if (lane == 0) {
+          __threadfence();
+          last = atomicAdd(&p.cnt[h], 1) == (int)(c1 - c0);
+        }
+        last = __shfl_sync(0xFFFFFFFFu, last, 0);
+        if (last) {  // the last CTA to arrive merges the pieces in CTA order
+          __threadfence();
+          float gm = -INFINITY, GL = 0.f, GA[CPL];
+#pragma unroll
+          for (int c = 0; c < CPL; ++c) GA[c] = 0.f;
+          for (long long cc = c0; cc <= c1; ++cc) {
+            const int slot = (cc == c0 && cc * chunk < hs) ? 1 : 0;
+            const float *qq = p.part + ((size_t)cc * 2 + slot) * (D + 2);
+            const float mc = __ldcg(qq + D), lc = __ldcg(qq + D + 1);
+            const float mn2 = fmaxf(gm, mc);
+            const float s0 = gm == -INFINITY ? 0.f : exp2f(gm - mn2);
+            const float s1 = exp2f(mc - mn2);
+            GL = GL * s0 + lc * s1;
+#pragma unroll
+            for (int c = 0; c < CPL; ++c) GA[c] = GA[c] * s0 + __ldcg(qq + lane + 32 * c) * s1;
+            gm = mn2;
+          }
+#pragma unroll
+          for (int c = 0; c < CPL; ++c) p.out[(size_t)h * D + lane + 32 * c] = GA[c] / GL;
+          if (lane == 0) p.cnt[h] = 0;
+          if (FUSED) append_row(h);
+        }
+      }
+      if (fin) break;
+    }
   }
 
-  if (FUSED) {
-    // the last CTA of the grid advances the counters: every CTA has read the
-    // lengths by now
-    __syncthreads();
-    if (tid == 0) {
-      __threadfence();
-      s_last = atomicAdd(p.gcnt, 1) == (int)gridDim.x - 1;
-    }
-    __syncthreads();
-    if (s_last) {
-      __threadfence();
-      for (int h = tid; h < nheads; h += kAttnThreads) {
-        const int i = p.layer_base + h;
-        p.len[h] += 1;
-        p.ntok[i] += 1;
-        if (p.label[i] != HKV_DENSE) p.nbuf[i] += 1;
-      }
-      if (tid == 0) *p.gcnt = 0;
-    }
-  }
+  if (FUSED && !early) grid_arrive();  // the CTAs that read lengths late
+  if (tid == 0) HKV_TRACE(6);
 }
 
 template <int D, typename T>
@@ -580,6 +650,13 @@ cudaError_t launch_t(const AttnArgs &a, int grid, bool fused, cudaStream_t s) {
 }
 
 }  // namespace
+
+#ifdef HKV_ATTN_TRACE
+// tracer builds only: where the phase timestamps go
+extern "C" int hkv_debug_set_trace(unsigned long long *buf) {
+  return cudaMemcpyToSymbol(g_trace, &buf, sizeof(buf)) == cudaSuccess ? 0 : 7;
+}
+#endif
 
 size_t attention_smem_bytes(int D, int dtype) {
   if (dtype == HKV_BF16) return D == 64 ? smem_bytes<64, __nv_bfloat16>() : smem_bytes<128, __nv_bfloat16>();

@@ -36,12 +36,13 @@ struct AttnArgs {
                               // previous kernel (its writes do not touch it)
 };
 
-// decode attention CTA: one producer warp (TMA) + consumer warps
+// decode attention CTA: one producer warp (TMA), consumer warps, one
+// epilogue warp (merges, partial results, combine)
 #ifndef HKV_ATTN_CONSUMER_WARPS
-#define HKV_ATTN_CONSUMER_WARPS 8
+#define HKV_ATTN_CONSUMER_WARPS 7
 #endif
 constexpr int kAttnConsumerWarps = HKV_ATTN_CONSUMER_WARPS;
-constexpr int kAttnThreads = 32 * (kAttnConsumerWarps + 1);
+constexpr int kAttnThreads = 32 * (kAttnConsumerWarps + 2);  // + producer + epilogue
 constexpr int kAttnMaxGrid = 4096;
 
 size_t attention_smem_bytes(int D, int dtype);
