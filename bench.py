@@ -273,7 +273,9 @@ def run_ours(args):
     with torch.cuda.graph(graph):
         period_calls()
     stream = torch.cuda.current_stream()
-    launches_per_step = P * L + L
+    # per period: every decode step is an attention and a finishing kernel;
+    # every layer's update is one kernel
+    launches_per_step = 2 * P * L + L
 
     def barrier():
         if world > 1:
@@ -373,7 +375,7 @@ def run_ours(args):
                        "parallelism": "replicas" if world > 1 else "single GPU"},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": None,
-                         "kernel": "attn_kernel<fused> (hkv_decode_step: append + attention)",
+                         "kernel": "hkv_decode_step: attn_kernel<fused> + finish_kernel<fused>",
                          "bytes_per_launch": bytes_per_launch, "launch_us": attn_us,
                          "launch_us_isolated": statistics.mean(step_us),
                          "evict_us_per_period": sum(evict_us), "copy_us_per_period": copy_us,

@@ -147,11 +147,11 @@ const char *hkv_status_str(hkv_status s);
 hkv_status hkv_validate_config(const hkv_config *cfg);
 
 /* Bytes of device workspace hkv_decode_attention and hkv_decode_step need
- * for this config (split-K partial results, per-head and grid arrival
- * counters). The workspace must be zero-filled before its first use; every
- * call leaves its counters at zero again (after a call that reported an
- * error, zero it again). Concurrent calls must not share a workspace.
- * Host only. */
+ * for this config (split-K partial results, where each head starts in the
+ * work split, and a small control block the two kernels of a call share).
+ * The workspace must be zero-filled before its first use; every call leaves
+ * it ready for the next one (after a call that reported an error, zero it
+ * again). Concurrent calls must not share a workspace. Host only. */
 size_t hkv_workspace_size(const hkv_config *cfg);
 
 /* Sets up the uncompressed cache of Step 1 (cache prefilling): every head
@@ -191,9 +191,10 @@ hkv_status hkv_append_evict(const hkv_config *cfg, const hkv_cache *cache, int l
  * the step that follows the P-th buffered token. */
 hkv_status hkv_evict(const hkv_config *cfg, const hkv_cache *cache, int layer, hkv_stream_t stream);
 
-/* One decode step of one layer in a single launch: the append of the new
- * token (Sec. 3, KV Cache) fused with the attention of Eq. 1 over the cache
- * including that token. out[s][h][:] = softmax(q k^T / sqrt(d)) V over the
+/* One decode step of one layer: the append of the new token (Sec. 3, KV
+ * Cache) fused with the attention of Eq. 1 over the cache including that
+ * token, in two kernels chained on `stream` (attention over the cache, then
+ * a finishing kernel that combines heads split across CTAs and appends). out[s][h][:] = softmax(q k^T / sqrt(d)) V over the
  * head's len live tokens and the new one (whose K/V are read straight from
  * k and v), fp32; then k, v join the arena at row len, q joins the Q_past
  * ring, and len, ntok (and nbuf for compressed heads) advance by one.
@@ -209,7 +210,8 @@ hkv_status hkv_decode_step(const hkv_config *cfg, const hkv_cache *cache, int la
 /* Eq. 1 for one new query per head over that head's live tokens (any mix
  * of lengths): out[s][h][:] = softmax(q k^T / sqrt(d)) V, fp32 accumulation,
  * written in fp32 ([S][H][head_dim]). Split-K over the layer's total token
- * count with a per-head combine; workspace of hkv_workspace_size bytes.
+ * count, then a second kernel combines the heads split across CTAs;
+ * workspace of hkv_workspace_size bytes.
  * A head with len = 0 yields zeros. */
 hkv_status hkv_decode_attention(const hkv_config *cfg, const hkv_cache *cache, int layer,
                                 const void *q, float *out, void *workspace, size_t ws_bytes,
@@ -219,18 +221,20 @@ hkv_status hkv_decode_attention(const hkv_config *cfg, const hkv_cache *cache, i
  * the paper has no counterpart to this entry point. A plain C host program
  * without a device allocator, or a plugin inside a host framework that owns
  * and budgets all device memory, may have no way to provide the workspace
- * that hkv_decode_attention takes. Here the split-K partials and per-head
- * counters live in a fixed device array inside the library (1.25 MiB: 1 MiB
- * of partials and 65536 counters), which every GPU that loads the library
- * holds until the process exits. Same inputs, outputs and results as
+ * that hkv_decode_attention takes. Here the split-K partials, the heads'
+ * starts in the work split and the kernels' control block live in a fixed
+ * device array inside the library (1.5 MiB: 1 MiB of partials, 512 KiB for
+ * up to 65536 heads, 256 bytes), which every GPU that loads the library
+ * holds until the process exits. Nothing in it has to start at zero: each
+ * call writes what it reads. Same inputs, outputs and results as
  * hkv_decode_attention; it allocates nothing.
  *  - More than 65536 heads per layer (n_seqs * n_heads) -> HKV_ERR_CAPACITY.
  *  - The first call on a device, with that device current, looks up the
  *    array's device address and prepares the kernel; make that first call
  *    before any stream capture.
- *  - Every call uses the same array and clears its counters on `stream`
- *    first; calls that may overlap on the GPU (other streams, other host
- *    threads) race on it and must be serialised by the caller. */
+ *  - Every call uses the same array; calls that may overlap on the GPU
+ *    (other streams, other host threads) race on it and must be serialised
+ *    by the caller. */
 hkv_status hkv_decode_attention_noalloc(const hkv_config *cfg, const hkv_cache *cache, int layer,
                                         const void *q, float *out, hkv_stream_t stream);
 

@@ -136,17 +136,23 @@ int max_segment(const hkv_config *c) {
   return a > b ? a : b;
 }
 
+// split-K partials: two slots per CTA
 size_t part_bytes(const hkv_config *c) {
-  const size_t b = (size_t)kAttnMaxGrid * 2 * (size_t)(c->head_dim + 2) * sizeof(float);
+  const size_t b =
+      (size_t)kAttnMaxGrid * 2 * (size_t)attn_part_floats(c->head_dim) * sizeof(float);
   return (b + 255) & ~(size_t)255;
 }
 
-size_t cnt_bytes(const hkv_config *c) {
-  return ((size_t)c->n_seqs * c->n_heads * sizeof(int32_t) + 15) & ~(size_t)15;
+// where each head of a layer starts in the attention kernel's index space
+size_t hs_bytes(const hkv_config *c) {
+  return ((size_t)c->n_seqs * c->n_heads * sizeof(long long) + 255) & ~(size_t)255;
 }
 
+constexpr size_t kCtlBytes = 256;  // AttnCtl, padded
+
 // Fills the attention launch arguments for one layer; the workspace holds
-// the split-K partials, the per-head counters and the grid counter.
+// the split-K partials, the heads' starts in the index space and the
+// control block the attention kernel leaves for the finishing kernel.
 AttnArgs attn_args(const hkv_config *cfg, const hkv_cache *cache, int layer, const void *q,
                    float *out, void *workspace) {
   const int hpl = cfg->n_seqs * cfg->n_heads;
@@ -160,8 +166,8 @@ AttnArgs attn_args(const hkv_config *cfg, const hkv_cache *cache, int layer, con
   a.out = out;
   unsigned char *ws = static_cast<unsigned char *>(workspace);
   a.part = reinterpret_cast<float *>(ws);
-  a.cnt = reinterpret_cast<int32_t *>(ws + part_bytes(cfg));
-  a.gcnt = reinterpret_cast<int32_t *>(ws + part_bytes(cfg) + cnt_bytes(cfg));
+  a.hs = reinterpret_cast<long long *>(ws + part_bytes(cfg));
+  a.ctl = reinterpret_cast<AttnCtl *>(ws + part_bytes(cfg) + hs_bytes(cfg));
   a.err = cache->err;
   a.pos = cache->pos;
   a.nbuf = cache->nbuf;
@@ -177,7 +183,9 @@ AttnArgs attn_args(const hkv_config *cfg, const hkv_cache *cache, int layer, con
   return a;
 }
 
-hkv_status attn_grid(const hkv_config *cfg, int *grid) {
+// attention CTAs: every SM filled; finishing CTAs: one warp per head, at
+// most two one-warp CTAs per SM (what fits beside three attention CTAs)
+hkv_status attn_grid(const hkv_config *cfg, int *grid, int *finish_grid) {
   DeviceState *st;
   hkv_status s = device_state(&st);
   if (s != HKV_OK) return s;
@@ -186,6 +194,9 @@ hkv_status attn_grid(const hkv_config *cfg, int *grid) {
   if (s != HKV_OK) return s;
   int g = st->sms * ctas;
   *grid = g > kAttnMaxGrid ? kAttnMaxGrid : g;
+  const int per = kFinishThreads / 32;
+  const int f = (heads_per_layer(cfg) + per - 1) / per;
+  *finish_grid = f < 2 * st->sms ? f : 2 * st->sms;
   return HKV_OK;
 }
 
@@ -234,7 +245,7 @@ hkv_status hkv_validate_config(const hkv_config *c) {
 
 size_t hkv_workspace_size(const hkv_config *c) {
   if (!c || hkv_validate_config(c) != HKV_OK) return 0;
-  return part_bytes(c) + cnt_bytes(c) + 16;
+  return part_bytes(c) + hs_bytes(c) + kCtlBytes;
 }
 
 hkv_status hkv_init_dense(const hkv_config *cfg, const hkv_cache *cache, hkv_stream_t stream) {
@@ -288,11 +299,11 @@ hkv_status hkv_decode_attention(const hkv_config *cfg, const hkv_cache *cache, i
   if (!q || !out || !workspace) return HKV_ERR_INVALID_ARG;
   if (!aligned16(q) || !aligned16(out) || !aligned16(workspace)) return HKV_ERR_ALIGN;
   if (ws_bytes < hkv_workspace_size(cfg)) return HKV_ERR_CAPACITY;
-  int grid = 0;
-  HKV_TRY(attn_grid(cfg, &grid));
+  int grid = 0, fgrid = 0;
+  HKV_TRY(attn_grid(cfg, &grid, &fgrid));
   const AttnArgs a = attn_args(cfg, cache, layer, q, out, workspace);
   return cuda_status(
-      launch_attention(a, cfg->head_dim, cfg->dtype, grid, false, (cudaStream_t)stream));
+      launch_attention(a, cfg->head_dim, cfg->dtype, grid, fgrid, false, (cudaStream_t)stream));
 }
 
 hkv_status hkv_decode_step(const hkv_config *cfg, const hkv_cache *cache, int layer,
@@ -307,14 +318,14 @@ hkv_status hkv_decode_step(const hkv_config *cfg, const hkv_cache *cache, int la
     return HKV_ERR_ALIGN;
   if (ws_bytes < hkv_workspace_size(cfg)) return HKV_ERR_CAPACITY;
   if (flags & ~HKV_STEP_PREFETCH) return HKV_ERR_INVALID_ARG;
-  int grid = 0;
-  HKV_TRY(attn_grid(cfg, &grid));
+  int grid = 0, fgrid = 0;
+  HKV_TRY(attn_grid(cfg, &grid, &fgrid));
   AttnArgs a = attn_args(cfg, cache, layer, q, out, workspace);
   a.k_new = k;
   a.v_new = v;
   a.prefetch = (flags & HKV_STEP_PREFETCH) ? 1 : 0;
   return cuda_status(
-      launch_attention(a, cfg->head_dim, cfg->dtype, grid, true, (cudaStream_t)stream));
+      launch_attention(a, cfg->head_dim, cfg->dtype, grid, fgrid, true, (cudaStream_t)stream));
 }
 
 hkv_status hkv_evict(const hkv_config *cfg, const hkv_cache *cache, int layer,

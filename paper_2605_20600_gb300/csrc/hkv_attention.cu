@@ -2,38 +2,46 @@
 // Eq. 1 applied to each head's retained tokens), optionally fused with the
 // append of the step's new token.
 //
-// Design (GB300, memory bound: every retained K/V byte is read once):
-//  * split-K over the layer's TOTAL token count: the concatenation of all
-//    heads' live tokens is cut into gridDim.x equal contiguous ranges, so
-//    local heads (short) and global heads (long) load-balance exactly; a
-//    range may cover the end of one head, whole heads, and the start of
-//    another;
-//  * the prologue gives every thread a contiguous slice of the layer's
-//    heads (one round of loads), a block scan finds the CTA's first head,
-//    and a table of the next heads' (offset, length, start) goes to shared
+// Two kernels per layer, chained with programmatic dependent launch:
+//
+// attention kernel (memory bound: every retained K/V byte is read once)
+//  * split-K over the layer's total work, counted in tile slots: each head
+//    is rounded up to whole tiles of TT rows, since under a saturated memory
+//    system a tile costs one pipeline stage for one memory latency whatever
+//    its fill. The concatenation of all heads' slots is split into
+//    gridDim.x equal contiguous ranges, one per CTA, so local heads (short)
+//    and global heads (long) load-balance; a range may cover the end of one
+//    head, whole heads and the start of another;
+//  * the prologue gives every thread a contiguous slice of the layer's heads
+//    (one round of loads), a block scan locates each CTA's first head, and a
+//    table of (offset, length, start) of the CTA's heads goes to shared
 //    memory;
 //  * warp-specialised pipeline: one producer warp streams K/V tiles of 7 KB
-//    into shared memory with the TMA engine (1D cp.async.bulk) through
-//    NS stages guarded by full/empty mbarriers; the query row of a head rides
-//    along with the head's first tile; consumer warps never wait on the
-//    producer's issue work; an epilogue warp finishes each head segment
-//    (merge of the consumer warps' states, output or partial result,
-//    combine) while the consumers stream on;
+//    into shared memory with the TMA engine (1D cp.async.bulk) through NS
+//    stages guarded by full/empty mbarriers, each with a description of its
+//    tile; the query row of a head rides along with the head's first tile
+//    and, fused, the new token's K/V with its last; an epilogue warp merges
+//    the consumer warps' states of each head segment and writes the output
+//    (a head wholly inside the piece) or a partial result (a split head)
+//    while the consumers stream on;
 //  * consumers take whole token rows with 16-byte lanes (a 256-byte bf16 row
 //    is 16 lanes), a shuffle-xor tree per row for q.k, online softmax in the
 //    log2 domain with fp32 accumulation;
-//  * a head split across CTAs is combined by the last CTA to arrive (per-head
-//    atomic counter, no spinning); partials are merged in CTA order, so the
-//    result does not depend on arrival order;
-//  * fused append: the head's virtual length is len + 1, the new token's K/V
-//    come straight from the step's input rows, the CTA that finishes a head
-//    writes that head's new row, and the last CTA of the grid (grid-wide
-//    arrival counter) advances every head's counters once no CTA can still
-//    be reading them;
-//  * programmatic dependent launch: every thread waits for the previous
-//    kernel of the stream (griddepcontrol.wait) before it reads the step's
-//    inputs or writes anything; with the prefetch flag the prologue and the
-//    first NS tiles of old K/V rows go ahead of that wait;
+//  * no fences, atomics or cache writes: the kernel only reads the cache
+//    and writes outputs and partial results;
+//
+// finishing kernel (one warp per head, after the attention kernel completes)
+//  * merges the partial results of each split head in index order, so the
+//    result does not depend on timing;
+//  * fused: appends the new token (K/V row, position, query for the periodic
+//    update) and advances the head's length and counters;
+//
+//  * programmatic dependent launch: every thread of either kernel waits for
+//    the previous kernel of the stream (griddepcontrol.wait) before it reads
+//    what that kernel writes or writes anything; with the prefetch flag the
+//    attention prologue and the first NS tiles of old K/V rows go ahead of
+//    that wait (HKV_ATTN_PRE_TILES of them: tiles in flight then delay the
+//    previous finishing kernel, whose few loads are on the critical path);
 //  * every wait on an mbarrier is bounded; one that runs out flags the
 //    error and lets the CTA finish its control flow without the data.
 #include <math.h>
@@ -45,8 +53,9 @@
 namespace hkv {
 namespace {
 
-// Tuning knobs (compile time): bytes of K per pipeline stage, stages, and
-// a cap on resident CTAs per SM used to size the grid.
+// Tuning knobs (compile time): bytes of K per pipeline stage, stages, a cap
+// on resident CTAs per SM used to size the grid, tiles loaded before the
+// wait for the previous kernel (prefetch), tiles sent to L2 beyond those.
 #ifndef HKV_ATTN_TILE_BYTES
 #define HKV_ATTN_TILE_BYTES 7168
 #endif
@@ -56,22 +65,40 @@ namespace {
 #ifndef HKV_ATTN_MAX_CTAS_PER_SM
 #define HKV_ATTN_MAX_CTAS_PER_SM 32
 #endif
+#ifndef HKV_ATTN_PRE_TILES
+#define HKV_ATTN_PRE_TILES 3
+#endif
+#ifndef HKV_ATTN_L2_TILES
+#define HKV_ATTN_L2_TILES 0
+#endif
+static_assert(HKV_ATTN_PRE_TILES >= 0 && HKV_ATTN_PRE_TILES <= HKV_ATTN_STAGES, "prefetch depth");
 
 constexpr int kCW = kAttnConsumerWarps;
 
-// Phase timestamps per CTA for latency studies; compiled out by default.
+// Phase timestamps and counters per CTA for latency studies; compiled out by
+// default.
 #ifdef HKV_ATTN_TRACE
-__device__ unsigned long long *g_trace = nullptr;  // [layer][kAttnMaxGrid][8], set by the tracer
-#define HKV_TRACE(slot)                                                  \
-  do {                                                                   \
-    if (g_trace)                                                         \
-      g_trace[((size_t)(p.layer_base / p.nheads) * kAttnMaxGrid + blockIdx.x) * 8 + (slot)] = \
-          globaltimer();                                                 \
+__device__ unsigned long long *g_trace = nullptr;  // [layer][kAttnMaxGrid][32], set by the tracer
+#define HKV_TRACE_AT(slot) \
+  g_trace[((size_t)(p.layer_base / p.nheads) * kAttnMaxGrid + blockIdx.x) * 32 + (slot)]
+#define HKV_TRACE(slot)                              \
+  do {                                               \
+    if (g_trace) HKV_TRACE_AT(slot) = globaltimer(); \
   } while (0)
+#define HKV_TRACE_ADD(slot, v)              \
+  do {                                      \
+    if (g_trace) HKV_TRACE_AT(slot) += (v); \
+  } while (0)
+#define HKV_CLOCK() globaltimer()
 #else
 #define HKV_TRACE(slot) \
   do {                  \
   } while (0)
+#define HKV_TRACE_ADD(slot, v) \
+  do {                         \
+    (void)(v);                 \
+  } while (0)
+#define HKV_CLOCK() 0ull
 #endif
 
 template <int D, typename T>
@@ -85,23 +112,65 @@ struct AttnShape {
   static constexpr int kSteps = kTT / (kCW * kRPW);
   static constexpr int kNS = HKV_ATTN_STAGES;     // pipeline stages
   static constexpr int kStageBytes = 2 * kTT * kRB + kRB;   // K, V, q row
-  static constexpr int kMinChunk = 2 * kTT;       // fewest tokens per CTA
+  static constexpr int kMinChunk = 2 * kTT;       // fewest indices per CTA range
   static_assert(kLPR >= 1 && kLPR <= 32 && 32 % kLPR == 0, "row mapping");
   static_assert(kSteps >= 1 && kTT % (kCW * kRPW) == 0, "tile mapping");
-  static_assert(D <= kCW * 32, "one consumer thread per output channel");
+  static_assert(D <= kCW * 32 && D % 32 == 0, "output channels");
   static_assert(kStageBytes % 16 == 0, "TMA alignment");
 };
 
-constexpr int kTable = 32;  // heads whose (offset, length, start) sit in smem
+constexpr int kTable = 32;  // heads of a CTA's range kept in smem
 
 struct HeadTable {
-  int h0;                   // first head of the CTA's range
+  int h0;                   // first head of the table
   int n;                    // valid entries
-  int covers;               // the entries cover the CTA's whole range
-  long long start[kTable];  // global token index where head h0 + j starts
+  long long start[kTable];  // index (slot space) where head h0 + j starts
   long long off[kTable];    // arena offset of head h0 + j
   int vlen[kTable];         // virtual length (len + fused)
-  int ntok[kTable];         // image tokens appended so far (fused)
+};
+
+constexpr int kFirst = 1, kLast = 2, kDone = 4;
+
+struct TileMeta {           // producer -> consumers, one per stage
+  int h, n, flags;          // head, rows, kFirst | kLast | kDone
+  long long hs, he;         // the head's rows in the index space
+};
+
+struct SegMeta {            // consumers -> epilogue; h < 0: no more segments
+  int h;
+  long long hs, he;
+};
+
+// N consecutive floats as one vector access (N = 2 or 4)
+template <int N>
+struct Vec;
+template <>
+struct Vec<4> {
+  __device__ static __forceinline__ void st(float *p, const float *v) {
+    *reinterpret_cast<float4 *>(p) = make_float4(v[0], v[1], v[2], v[3]);
+  }
+  __device__ static __forceinline__ void lds(const float *p, float *v) {
+    const float4 x = *reinterpret_cast<const float4 *>(p);
+    v[0] = x.x, v[1] = x.y, v[2] = x.z, v[3] = x.w;
+  }
+  __device__ static __forceinline__ void ldcg(const float *p, float *v) {
+    const float4 x = __ldcg(reinterpret_cast<const float4 *>(p));
+    v[0] = x.x, v[1] = x.y, v[2] = x.z, v[3] = x.w;
+  }
+};
+template <>
+struct Vec<2> {
+  __device__ static __forceinline__ void st(float *p, const float *v) {
+    *reinterpret_cast<float2 *>(p) = make_float2(v[0], v[1]);
+  }
+  __device__ static __forceinline__ void lds(const float *p, float *v) {
+    const float2 x = *reinterpret_cast<const float2 *>(p);
+    v[0] = x.x, v[1] = x.y;
+  }
+  __device__ static __forceinline__ void ldcg(const float *p, float *v) {
+    const float2 x = __ldcg(reinterpret_cast<const float2 *>(p));
+    v[0] = x.x, v[1] = x.y;
+  }
 };
 
 __device__ __forceinline__ void pdl_wait() {
@@ -111,8 +180,15 @@ __device__ __forceinline__ void pdl_launch_dependents() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
+// Head h of n rows takes slot_len(n) indices: whole tiles of TT rows, the
+// last one partly filled.
+template <int TT>
+__device__ __forceinline__ long long slot_len(long long n) {
+  return (n + TT - 1) / TT * TT;
+}
+
 template <bool FUSED>
-struct HeadLookup {
+struct HeadLookup {  // the table, else global memory
   const HeadTable &t;
   const AttnArgs &p;
   __device__ __forceinline__ int vlen(int h) const {
@@ -127,28 +203,30 @@ struct HeadLookup {
   }
 };
 
-// Walks the tiles of one CTA's token range [g, b) head by head.
+// Walks the tiles of a slot-aligned range [g, b) of the index space head by
+// head.
+template <int TT>
 struct TileIter {
   int h;         // current head (layer-local index)
   int hl;        // its (virtual) length
-  long long hs;  // global token index where head h starts
-  long long g;   // start of the current tile
-  long long b;   // end of the CTA's range
+  long long hs;  // index where head h starts
+  long long g;   // start of the current tile (a slot boundary)
+  long long b;   // end of the range (a slot boundary)
 
   __device__ __forceinline__ bool done() const { return g >= b; }
-  __device__ __forceinline__ long long tile_end(int tt) const {
-    long long e = g + tt;
+  __device__ __forceinline__ long long tile_end() const {  // end of the tile's rows
+    long long e = g + TT;
     const long long he = hs + hl;
     if (e > he) e = he;
     if (e > b) e = b;
     return e;
   }
   template <class L>
-  __device__ __forceinline__ void advance(int tt, const L &look) {
-    g = tile_end(tt);
+  __device__ __forceinline__ void advance(const L &look) {
+    g += TT;
     if (g >= b) return;
-    while (g >= hs + hl) {  // next head holding token g (skips empty heads)
-      hs += hl;
+    while (g >= hs + slot_len<TT>(hl)) {  // next head holding slot g (skips empty heads)
+      hs += slot_len<TT>(hl);
       ++h;
       hl = look.vlen(h);
     }
@@ -170,21 +248,29 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
   extern __shared__ __align__(128) unsigned char stages[];
   __shared__ uint64_t full[NS], empty[NS];
   __shared__ uint64_t epi_full, epi_free;   // hand-over of one segment's states
-  __shared__ float red_acc[kCW][D];
+  __shared__ __align__(16) float red_acc[kCW][D];
   __shared__ float red_m[kCW], red_l[kCW];
-  __shared__ int seg_h, seg_final;
-  __shared__ long long seg_hs, seg_he;
+  __shared__ TileMeta meta[NS];
+  __shared__ SegMeta seg;
   __shared__ HeadTable tab;
   __shared__ long long scan_scratch[33];
   __shared__ long long s_s0;
-  __shared__ int s_h0, s_bad, s_last;
+  __shared__ int s_h0, s_bad;
   __shared__ volatile int s_abort;
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int nheads = p.nheads;
+  const int G = gridDim.x;
 
   if (tid == 0) {
     HKV_TRACE(0);
+#ifdef HKV_ATTN_TRACE
+    if (g_trace) {
+      unsigned smid;
+      asm volatile("mov.u32 %0, %%smid;" : "=r"(smid));
+      HKV_TRACE_AT(16) = smid;
+    }
+#endif
     for (int s = 0; s < NS; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], kCW);
@@ -193,6 +279,9 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
     mbar_init(&epi_free, 1);
     fence_barrier_init();
     s_abort = 0;
+    s_bad = 0;
+    s_h0 = 0;
+    s_s0 = 0;
   }
   // Without prefetch, wait for the previous kernel's writes first. With it,
   // the prologue and the first tiles of old K/V rows (which the caller
@@ -200,8 +289,8 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
   if (!p.prefetch) pdl_wait();
 
   // ---- prologue: every thread takes a contiguous slice of the layer's heads
-  // (all of its loads in flight at once), a block scan gives each slice its
-  // first token, and the slice holding token a names the CTA's first head.
+  // (all of its loads in flight at once); a block scan gives each slice its
+  // first slot.
   const int per = (nheads + kAttnThreads - 1) / kAttnThreads;
   const int h_lo = tid * per < nheads ? tid * per : nheads;
   const int h_hi = h_lo + per < nheads ? h_lo + per : nheads;
@@ -219,28 +308,31 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
       else if (p.label[p.layer_base + h] != HKV_DENSE && p.nbuf[p.layer_base + h] >= p.period)
         bad = bad ? bad : HKV_ERR_STATE;  // the periodic update is due first
     }
-    mine += l + (FUSED ? 1 : 0);
+    mine += slot_len<TT>(l + (FUSED ? 1 : 0));
   }
   long long total;
   const long long slice_start = block_excl_scan<long long>(mine, scan_scratch, &total);
-  if (tid == 0) s_bad = 0;
-  __syncthreads();
   if (bad) atomicMax(&s_bad, bad);
   __syncthreads();
   if (s_bad) {
     pdl_wait();
-    if (blockIdx.x == 0 && tid == 0) set_err(p.err, (uint32_t)s_bad);
+    if (blockIdx.x == 0 && tid == 0) {
+      set_err(p.err, (uint32_t)s_bad);
+      p.ctl->valid = 0;  // nothing for the finishing kernel to do
+    }
     return;
   }
-  long long chunk = (total + gridDim.x - 1) / gridDim.x;
+  // whole slots per CTA; rounding up leaves the last CTAs, which start
+  // last, with less
+  long long chunk = slot_len<TT>((total + G - 1) / G);
   if (chunk < S::kMinChunk) chunk = S::kMinChunk;
   const long long a = (long long)blockIdx.x * chunk;
   const long long b = a + chunk < total ? a + chunk : total;
-  const bool active = a < total;
-  if (active && mine > 0 && slice_start <= a && a < slice_start + mine) {
+  const bool st_active = a < total;
+  if (st_active && mine > 0 && slice_start <= a && a < slice_start + mine) {
     long long st = slice_start;
     for (int h = h_lo; h < h_hi; ++h) {
-      const long long L = p.len[h] + (FUSED ? 1 : 0);
+      const long long L = slot_len<TT>(p.len[h] + (FUSED ? 1 : 0));
       if (a < st + L) {
         s_h0 = h;
         s_s0 = st;
@@ -250,69 +342,42 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
     }
   }
   __syncthreads();
-  if (active && warp == 0) {  // table of the heads from h0 on
-    const int h0 = s_h0;
+  if (warp == 0) {  // table of the heads from the CTA's first head on
+    const int h0 = st_active ? s_h0 : 0;
     const int h = h0 + lane;
-    const long long L = h < nheads ? p.len[h] + (FUSED ? 1 : 0) : 0;
+    const bool in = st_active && h < nheads;
+    const int vl = in ? p.len[h] + (FUSED ? 1 : 0) : 0;
+    const long long L = slot_len<TT>(vl);
     const long long incl = warp_incl_scan(L);
     tab.start[lane] = s_s0 + incl - L;
-    tab.off[lane] = h < nheads ? p.off[h] : 0;
-    tab.vlen[lane] = (int)L;
-    tab.ntok[lane] = (FUSED && h < nheads) ? p.ntok[p.layer_base + h] : 0;
-    const int n = nheads - h0 < kTable ? nheads - h0 : kTable;
-    const long long end = __shfl_sync(0xFFFFFFFFu, s_s0 + incl, n - 1);
+    tab.off[lane] = in ? p.off[h] : 0;
+    tab.vlen[lane] = vl;
     if (lane == 0) {
       tab.h0 = h0;
-      tab.n = n;
-      tab.covers = end >= b;
+      tab.n = st_active ? (nheads - h0 < kTable ? nheads - h0 : kTable) : 0;
     }
   }
   __syncthreads();
-  // Fused: a CTA whose heads all sit in the table reads no length, position
-  // counter or buffer count after this point, so it can count itself on the
-  // grid counter as soon as the previous kernel is done (the counter lives in
-  // the shared workspace); the last CTA to count advances the counters. The
-  // other CTAs count at the end.
-  const bool early = FUSED && (!active || tab.covers);
-
   if (tid == 0) HKV_TRACE(1);
-  auto grid_arrive = [&]() {  // block-wide; called after the wait
-    __syncthreads();
-    if (tid == 0) {
-      __threadfence();
-      s_last = atomicAdd(p.gcnt, 1) == (int)gridDim.x - 1;
-    }
-    __syncthreads();
-    if (s_last) {
-      __threadfence();
-      for (int h = tid; h < nheads; h += kAttnThreads) {
-        const int i = p.layer_base + h;
-        p.len[h] += 1;
-        p.ntok[i] += 1;
-        if (p.label[i] != HKV_DENSE) p.nbuf[i] += 1;
-      }
-      if (tid == 0) *p.gcnt = 0;
-    }
-    __syncthreads();
-  };
   const HeadLookup<FUSED> look{tab, p};
-  TileIter cit;
-  cit.h = tab.h0;
-  cit.hs = tab.start[0];
-  cit.hl = tab.vlen[0];
-  cit.g = a;
-  cit.b = b;
 
   // ---- producer state (warp 0, lane 0) ----------------------------------
   // A tile's old rows come from the arena; the query row (first tile of a
-  // head here) and the new token's K/V (fused, last tile of a head) come from
-  // this step's inputs, which may be written by the previous kernel.
-  const bool producer = active && tid == 0;
-  TileIter pit = cit;
+  // head in a piece) and the new token's K/V (fused, last tile of a head)
+  // come from this step's inputs, which may be written by the previous
+  // kernel.
+  const bool producer = tid == 0;
+  TileIter<TT> pit;
+  pit.h = tab.h0;
+  pit.hs = tab.start[0];
+  pit.hl = tab.vlen[0];
+  pit.g = st_active ? a : 0;
+  pit.b = st_active ? b : 0;
   int issued = 0;
-  auto issue_old = [&](Pending &pd) {  // expect + copy the arena rows, no arrival
+  auto issue_old = [&](Pending &pd) {  // describe + expect + copy the arena rows
     const int stage = issued % NS;
-    const long long ge = pit.tile_end(TT);
+    const long long ge = pit.tile_end();
+    const long long he = pit.hs + pit.hl;
     const int r0 = (int)(pit.g - pit.hs), r1 = (int)(ge - pit.hs);   // head-local rows
     const int real = FUSED ? pit.hl - 1 : pit.hl;                    // rows in the arena
     const int n_old = (r1 < real ? r1 : real) - r0;
@@ -321,6 +386,12 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
     pd.slot_new = real - r0;
     pd.first = pit.g == pit.hs || pit.g == a;
     pd.has_new = FUSED && r1 == pit.hl;
+    TileMeta &mt = meta[stage];
+    mt.h = pit.h;
+    mt.n = (int)(ge - pit.g);
+    mt.flags = (pd.first ? kFirst : 0) | (ge == (b < he ? b : he) ? kLast : 0);
+    mt.hs = pit.hs;
+    mt.he = he;
     if (n_old > 0) {
       const uint32_t bytes = (uint32_t)n_old * RB;
       const long long row = look.off(pit.h) + r0;
@@ -329,7 +400,7 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
       bulk_g2s(dk + TT * RB, static_cast<const unsigned char *>(p.V) + row * RB, bytes,
                &full[stage]);
     }
-    pit.advance(TT, look);
+    pit.advance(look);
     ++issued;
   };
   auto issue_extra = [&](const Pending &pd, int stage) {  // inputs, then arrive
@@ -348,37 +419,47 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
   };
   Pending pre[NS];
   int n_pre = 0;
-  if (producer)
-    for (; n_pre < NS && !pit.done(); ++n_pre) issue_old(pre[n_pre]);
+  if (producer) {
+    for (; n_pre < (p.prefetch ? HKV_ATTN_PRE_TILES : NS) && !pit.done(); ++n_pre)
+      issue_old(pre[n_pre]);
+    // While the previous kernels finish, the memory system would idle once
+    // those tiles are in: with prefetch, the next HKV_ATTN_L2_TILES tiles of
+    // old rows go to L2 as well.
+    if (p.prefetch && HKV_ATTN_L2_TILES > 0) {
+      TileIter<TT> it = pit;
+      for (int j = 0; j < HKV_ATTN_L2_TILES && !it.done(); ++j) {
+        const long long ge = it.tile_end();
+        const int r0 = (int)(it.g - it.hs), r1 = (int)(ge - it.hs);
+        const int real = FUSED ? it.hl - 1 : it.hl;
+        const int n_old = (r1 < real ? r1 : real) - r0;
+        if (n_old > 0) {
+          const long long row = look.off(it.h) + r0;
+          bulk_prefetch_l2(static_cast<const unsigned char *>(p.K) + row * RB, (uint32_t)n_old * RB);
+          bulk_prefetch_l2(static_cast<const unsigned char *>(p.V) + row * RB, (uint32_t)n_old * RB);
+        }
+        it.advance(look);
+      }
+    }
+  }
 
   if (p.prefetch) pdl_wait();  // the step's inputs are visible from here on
   if (tid == 0) HKV_TRACE(2);
   pdl_launch_dependents();
-  if (early) grid_arrive();
-
-  // Fused append of a head's new token (row, position, query) by the warp
-  // that finishes the head; nothing in this launch reads them.
-  auto append_row = [&](int h) {
-    const int i = p.layer_base + h;
-    const int jt = h - tab.h0;
-    const bool in_tab = jt >= 0 && jt < tab.n;
-    const int len = (in_tab ? tab.vlen[jt] : p.len[h] + 1) - 1;
-    const int nt = in_tab ? tab.ntok[jt] : p.ntok[i];
-    const long long row = look.off(h) + len;
-    const uint4 *ks = reinterpret_cast<const uint4 *>(static_cast<const unsigned char *>(p.k_new) + (size_t)h * RB);
-    const uint4 *vs = reinterpret_cast<const uint4 *>(static_cast<const unsigned char *>(p.v_new) + (size_t)h * RB);
-    const uint4 *qs = reinterpret_cast<const uint4 *>(static_cast<const unsigned char *>(p.q) + (size_t)h * RB);
-    uint4 *kd = reinterpret_cast<uint4 *>(static_cast<unsigned char *>(p.K) + row * RB);
-    uint4 *vd = reinterpret_cast<uint4 *>(static_cast<unsigned char *>(p.V) + row * RB);
-    uint4 *qd = reinterpret_cast<uint4 *>(static_cast<unsigned char *>(p.qbuf) +
-                                          ((size_t)i * p.period + nt % p.period) * RB);
-    for (int c = lane; c < RB / 16; c += 32) {
-      kd[c] = ks[c];
-      vd[c] = vs[c];
-      qd[c] = qs[c];
+  // Block 0 tells the finishing kernel where every head starts and how the
+  // work was split (the workspace is free: the previous finishing kernel is
+  // done).
+  if (blockIdx.x == 0) {
+    long long st = slice_start;
+    for (int h = h_lo; h < h_hi; ++h) {
+      p.hs[h] = st;
+      st += slot_len<TT>(p.len[h] + (FUSED ? 1 : 0));
     }
-    if (lane == 0) p.pos[row] = p.n_cond + nt;
-  };
+    if (tid == 0) {
+      p.ctl->chunk = chunk;
+      p.ctl->grid = G;
+      p.ctl->valid = 1;
+    }
+  }
 
   if (warp == 0) {
     // ---- producer ----------------------------------------------------------
@@ -389,7 +470,8 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
       while (!pit.done()) {
         const int stage = issued % NS;
         // the consumers are done with the tile that used this stage before
-        if (s_abort || !mbar_wait(&empty[stage], (uint32_t)(issued / NS - 1) & 1u)) {
+        if (s_abort ||
+            (issued >= NS && !mbar_wait(&empty[stage], (uint32_t)(issued / NS - 1) & 1u))) {
           s_abort = 1;
           set_err(p.err, HKV_ERR_TIMEOUT);
           break;
@@ -398,148 +480,169 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
         issue_old(pd);
         issue_extra(pd, stage);
       }
+      if (!s_abort) {  // no more tiles: a closing record for the consumers
+        const int stage = issued % NS;
+        if (issued >= NS && !mbar_wait(&empty[stage], (uint32_t)(issued / NS - 1) & 1u)) {
+          s_abort = 1;
+          set_err(p.err, HKV_ERR_TIMEOUT);
+        } else {
+          meta[stage].flags = kDone;
+          mbar_arrive(&full[stage]);
+        }
+      }
     }
   } else if (warp <= kCW) {
     // ---- consumers ---------------------------------------------------------
     const int ctid = tid - 32, cw = warp - 1;
-    if (!FUSED && blockIdx.x == 0)  // empty heads (plain attention) are zeros
-      for (int h = ctid; h < nheads; h += kCW * 32)
-        if (p.len[h] == 0)
-          for (int d = 0; d < D; ++d) p.out[(size_t)h * D + d] = 0.f;
-
-    if (active) {
-      const int grp = lane / LPR, col = lane % LPR;
-      float q[EPL], acc[EPL];
-      float m = -INFINITY, l = 0.f;
-      int nseg = 0;
+    const int grp = lane / LPR, col = lane % LPR;
+    float q[EPL], acc[EPL];
+    float m = -INFINITY, l = 0.f;
+    int nseg = 0;
 #pragma unroll
-      for (int e = 0; e < EPL; ++e) acc[e] = 0.f;
+    for (int e = 0; e < EPL; ++e) acc[e] = 0.f;
 
-      for (int tile = 0; !cit.done(); ++tile) {
-        const int stage = tile % NS;
-        if (!s_abort && !mbar_wait(&full[stage], (uint32_t)(tile / NS) & 1u)) {
-          s_abort = 1;
-          set_err(p.err, HKV_ERR_TIMEOUT);
-        }
-        if (tile == 0 && ctid == 0) HKV_TRACE(3);
-        const long long ge = cit.tile_end(TT);
-        const int n = (int)(ge - cit.g);
-        const long long he = cit.hs + cit.hl;
-        const unsigned char *Ks = stages + stage * S::kStageBytes;
-        const unsigned char *Vs = Ks + TT * RB;
-        if (cit.g == cit.hs || cit.g == a) {  // first tile of this head here
-          Elem<T>::unpack(*reinterpret_cast<const uint4 *>(Vs + TT * RB + col * 16), q);
+    for (int tile = 0;; ++tile) {
+      const int stage = tile % NS;
+      if (!s_abort && !mbar_wait(&full[stage], (uint32_t)(tile / NS) & 1u)) {
+        s_abort = 1;
+        set_err(p.err, HKV_ERR_TIMEOUT);
+      }
+      if (s_abort) break;
+      const int flags = meta[stage].flags;
+      if (flags & kDone) break;
+      if (tile == 0 && ctid == 0) HKV_TRACE(3);
+      if (ctid == 0) HKV_TRACE_ADD(17, 1);
+      const int n = meta[stage].n;
+      const unsigned char *Ks = stages + stage * S::kStageBytes;
+      const unsigned char *Vs = Ks + TT * RB;
+      if (flags & kFirst) {  // first tile of this head in this piece
+        Elem<T>::unpack(*reinterpret_cast<const uint4 *>(Vs + TT * RB + col * 16), q);
 #pragma unroll
-          for (int e = 0; e < EPL; ++e) {
-            q[e] *= p.qscale;
-            acc[e] = 0.f;
-          }
-          m = -INFINITY;
-          l = 0.f;
+        for (int e = 0; e < EPL; ++e) {
+          q[e] *= p.qscale;
+          acc[e] = 0.f;
         }
+        m = -INFINITY;
+        l = 0.f;
+      }
 
-        float sc[S::kSteps];
+      float sc[S::kSteps];
+#pragma unroll
+      for (int st = 0; st < S::kSteps; ++st) {
+        const int r = st * (kCW * RPW) + cw * RPW + grp;
+        float dot = 0.f;
+        if (r < n) {
+          float kf[EPL];
+          Elem<T>::unpack(*reinterpret_cast<const uint4 *>(Ks + r * RB + col * 16), kf);
+#pragma unroll
+          for (int e = 0; e < EPL; ++e) dot = fmaf(q[e], kf[e], dot);
+        }
+#pragma unroll
+        for (int o = LPR / 2; o >= 1; o >>= 1) dot += __shfl_xor_sync(0xFFFFFFFFu, dot, o);
+        sc[st] = r < n ? dot : -INFINITY;
+      }
+      float mt = sc[0];
+#pragma unroll
+      for (int st = 1; st < S::kSteps; ++st) mt = fmaxf(mt, sc[st]);
+      const float mn = fmaxf(m, mt);
+      if (mn != -INFINITY) {
+        const float corr = exp2f(m - mn);
+        l *= corr;
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) acc[e] *= corr;
 #pragma unroll
         for (int st = 0; st < S::kSteps; ++st) {
           const int r = st * (kCW * RPW) + cw * RPW + grp;
-          float dot = 0.f;
           if (r < n) {
-            float kf[EPL];
-            Elem<T>::unpack(*reinterpret_cast<const uint4 *>(Ks + r * RB + col * 16), kf);
+            const float pr = exp2f(sc[st] - mn);
+            l += pr;
+            float vf[EPL];
+            Elem<T>::unpack(*reinterpret_cast<const uint4 *>(Vs + r * RB + col * 16), vf);
 #pragma unroll
-            for (int e = 0; e < EPL; ++e) dot = fmaf(q[e], kf[e], dot);
+            for (int e = 0; e < EPL; ++e) acc[e] = fmaf(pr, vf[e], acc[e]);
           }
-#pragma unroll
-          for (int o = LPR / 2; o >= 1; o >>= 1) dot += __shfl_xor_sync(0xFFFFFFFFu, dot, o);
-          sc[st] = r < n ? dot : -INFINITY;
         }
-        float mt = sc[0];
-#pragma unroll
-        for (int st = 1; st < S::kSteps; ++st) mt = fmaxf(mt, sc[st]);
-        const float mn = fmaxf(m, mt);
-        if (mn != -INFINITY) {
-          const float corr = exp2f(m - mn);
-          l *= corr;
-#pragma unroll
-          for (int e = 0; e < EPL; ++e) acc[e] *= corr;
-#pragma unroll
-          for (int st = 0; st < S::kSteps; ++st) {
-            const int r = st * (kCW * RPW) + cw * RPW + grp;
-            if (r < n) {
-              const float pr = exp2f(sc[st] - mn);
-              l += pr;
-              float vf[EPL];
-              Elem<T>::unpack(*reinterpret_cast<const uint4 *>(Vs + r * RB + col * 16), vf);
-#pragma unroll
-              for (int e = 0; e < EPL; ++e) acc[e] = fmaf(pr, vf[e], acc[e]);
-            }
-          }
-          m = mn;
+        m = mn;
+      }
+      if (flags & kLast) {  // last tile of this head in this piece: hand it over
+        SegMeta sm;
+        if (cw == 0 && lane == 0) {
+          sm.h = meta[stage].h;
+          sm.hs = meta[stage].hs;
+          sm.he = meta[stage].he;
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&empty[stage]);  // this warp is done with the stage
-        if (ctid == 0 && ge == b) HKV_TRACE(4);
-
-        if (ge == (b < he ? b : he)) {  // last tile of this head here: hand it over
 #pragma unroll
-          for (int o = LPR; o < 32; o <<= 1) {  // merge the row groups of the warp
-            const float m2 = __shfl_xor_sync(0xFFFFFFFFu, m, o);
-            const float l2 = __shfl_xor_sync(0xFFFFFFFFu, l, o);
-            const float mx = fmaxf(m, m2);
-            const float s1 = m == -INFINITY ? 0.f : exp2f(m - mx);
-            const float s2 = m2 == -INFINITY ? 0.f : exp2f(m2 - mx);
-            l = l * s1 + l2 * s2;
+        for (int o = LPR; o < 32; o <<= 1) {  // merge the row groups of the warp
+          const float m2 = __shfl_xor_sync(0xFFFFFFFFu, m, o);
+          const float l2 = __shfl_xor_sync(0xFFFFFFFFu, l, o);
+          const float mx = fmaxf(m, m2);
+          const float s1 = m == -INFINITY ? 0.f : exp2f(m - mx);
+          const float s2 = m2 == -INFINITY ? 0.f : exp2f(m2 - mx);
+          l = l * s1 + l2 * s2;
 #pragma unroll
-            for (int e = 0; e < EPL; ++e) {
-              const float a2 = __shfl_xor_sync(0xFFFFFFFFu, acc[e], o);
-              acc[e] = acc[e] * s1 + a2 * s2;
-            }
-            m = mx;
+          for (int e = 0; e < EPL; ++e) {
+            const float a2 = __shfl_xor_sync(0xFFFFFFFFu, acc[e], o);
+            acc[e] = acc[e] * s1 + a2 * s2;
           }
-          // the epilogue is done with the previous segment's states
-          if (nseg > 0 && !s_abort && !mbar_wait(&epi_free, (uint32_t)(nseg - 1) & 1u)) {
-            s_abort = 1;
-            set_err(p.err, HKV_ERR_TIMEOUT);
-          }
-          if (lane < LPR) {
-#pragma unroll
-            for (int e = 0; e < EPL; ++e) red_acc[cw][lane * EPL + e] = acc[e];
-            if (lane == 0) {
-              red_m[cw] = m;
-              red_l[cw] = l;
-            }
-          }
-          if (cw == 0 && lane == 0) {
-            seg_h = cit.h;
-            seg_hs = cit.hs;
-            seg_he = he;
-            seg_final = ge == b;
-          }
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&epi_full);
-          ++nseg;
+          m = mx;
         }
-        cit.advance(TT, look);
+        // the epilogue is done with the previous segment's states
+        const unsigned long long tw = HKV_CLOCK();
+        if (nseg > 0 && !s_abort && !mbar_wait(&epi_free, (uint32_t)(nseg - 1) & 1u)) {
+          s_abort = 1;
+          set_err(p.err, HKV_ERR_TIMEOUT);
+        }
+        if (cw == 0 && lane == 0) HKV_TRACE_ADD(11, HKV_CLOCK() - tw);
+        if (lane < LPR) {
+#pragma unroll
+          for (int e = 0; e < EPL; ++e) red_acc[cw][lane * EPL + e] = acc[e];
+          if (lane == 0) {
+            red_m[cw] = m;
+            red_l[cw] = l;
+          }
+        }
+        if (cw == 0 && lane == 0) seg = sm;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&epi_full);
+        ++nseg;
+      } else {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[stage]);  // this warp is done with the stage
       }
-      if (ctid == 0) HKV_TRACE(5);
-      if (s_abort && ctid == 0)  // drain what may still be in flight (bounded)
-        for (int s = 0; s < NS; ++s) {
-          mbar_wait(&full[s], 0);
-          mbar_wait(&full[s], 1);
-        }
     }
-  } else if (active) {
+    if (ctid == 0) HKV_TRACE(4);
+    // tell the epilogue there is nothing more
+    if (nseg > 0 && !s_abort && !mbar_wait(&epi_free, (uint32_t)(nseg - 1) & 1u)) {
+      s_abort = 1;
+      set_err(p.err, HKV_ERR_TIMEOUT);
+    }
+    if (cw == 0 && lane == 0) seg.h = -1;
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&epi_full);
+    if (s_abort && ctid == 0)  // drain what may still be in flight (bounded)
+      for (int s = 0; s < NS; ++s) {
+        mbar_wait(&full[s], 0);
+        mbar_wait(&full[s], 1);
+      }
+  } else {
     // ---- epilogue: finish each head segment the consumers hand over --------
-    constexpr int CPL = D / 32;  // output channels per lane
+    // A lane owns CPL consecutive output channels, so each of its stores of
+    // an output row or a partial result is one vector access.
+    constexpr int CPL = D / 32;
+    using V = Vec<CPL>;
+    constexpr int PS = attn_part_floats(D);  // floats per partial slot
     for (int k = 0;; ++k) {
       if (!s_abort && !mbar_wait(&epi_full, (uint32_t)k & 1u)) {
         s_abort = 1;
         set_err(p.err, HKV_ERR_TIMEOUT);
       }
       if (s_abort) break;
-      const int h = seg_h;
-      const long long hs = seg_hs, he = seg_he;
-      const int fin = seg_final;
+      const int h = seg.h;
+      if (h < 0) break;
+      if (lane == 0) HKV_TRACE_ADD(9, 1);
+      const long long hs = seg.hs, he = seg.he;
       float mx = red_m[0];
 #pragma unroll
       for (int w = 1; w < kCW; ++w) mx = fmaxf(mx, red_m[w]);
@@ -550,60 +653,173 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
       for (int w = 0; w < kCW; ++w) {
         const float sw = red_m[w] == -INFINITY ? 0.f : exp2f(red_m[w] - mx);
         L += red_l[w] * sw;
+        float r[CPL];
+        V::lds(&red_acc[w][CPL * lane], r);
 #pragma unroll
-        for (int c = 0; c < CPL; ++c) A[c] += red_acc[w][lane + 32 * c] * sw;
+        for (int c = 0; c < CPL; ++c) A[c] = fmaf(r[c], sw, A[c]);
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&epi_free);  // the consumers may reuse the slot
-      if (hs >= a && he <= b) {  // the whole head is here
+      if (hs >= a && he <= b) {  // the whole head is in this CTA's range
 #pragma unroll
-        for (int c = 0; c < CPL; ++c) p.out[(size_t)h * D + lane + 32 * c] = A[c] / L;
-        if (FUSED) append_row(h);
+        for (int c = 0; c < CPL; ++c) A[c] /= L;
+        V::st(p.out + (size_t)h * D + CPL * lane, A);
       } else {
-        float *pp = p.part + ((size_t)blockIdx.x * 2 + (hs <= a ? 0 : 1)) * (D + 2);
-#pragma unroll
-        for (int c = 0; c < CPL; ++c) pp[lane + 32 * c] = A[c];
+        // Partial result of this CTA's range: it holds the end of one split
+        // head (slot 0) and the start of another (slot 1).
+        float *pp = p.part + ((size_t)blockIdx.x * 2 + (a < hs ? 1 : 0)) * PS;
+        V::st(pp + CPL * lane, A);
         if (lane == 0) {
           pp[D] = mx;
           pp[D + 1] = L;
         }
-        __syncwarp();
-        const long long c0 = hs / chunk, c1 = (he - 1) / chunk;
-        int last = 0;
-        if (lane == 0) {
-          __threadfence();
-          last = atomicAdd(&p.cnt[h], 1) == (int)(c1 - c0);
-        }
-        last = __shfl_sync(0xFFFFFFFFu, last, 0);
-        if (last) {  // the last CTA to arrive merges the pieces in CTA order
-          __threadfence();
-          float gm = -INFINITY, GL = 0.f, GA[CPL];
+      }
+    }
+    if (lane == 0) HKV_TRACE(5);
+  }
+  if (tid == 0) HKV_TRACE(6);
+}
+
+// One warp per head: merge the partial results of a split head in index
+// order; fused, append the new token and advance the head's counters. Every
+// load that does not depend on another goes out first, so a head costs about
+// two round trips to memory.
+template <int D, typename T, bool FUSED>
+__global__ void __maxnreg__(kFinishRegs)
+    finish_kernel(const AttnArgs p) {
+  using S = AttnShape<D, T>;
+  constexpr int RB = S::kRB;
+  constexpr int CPL = D / 32;
+  using V = Vec<CPL>;
+  constexpr int PS = attn_part_floats(D);
+  constexpr int MB = 16 / CPL;  // partial results loaded per batch
+  static_assert(RB / 16 <= 32, "one 16-byte piece of a row per lane");
+  // Let the next kernel (the next layer's attention) start its prologue now;
+  // it waits for this kernel before it reads anything written here.
+  HKV_TRACE(20);
+  pdl_launch_dependents();
+  pdl_wait();  // the attention kernel is complete
+  HKV_TRACE(21);
+  const int lane = threadIdx.x & 31;
+  const int nw = gridDim.x * (kFinishThreads / 32);
+  const int w0 = blockIdx.x * (kFinishThreads / 32) + (threadIdx.x >> 5);
+  const int valid = p.ctl->valid;
+  const long long chunk = p.ctl->chunk;
+  if (!valid) return;
+
+  for (int h = w0; h < p.nheads; h += nw) {
+    const int i = p.layer_base + h;
+    const int len = p.len[h];
+    const long long hs = p.hs[h];
+    // fused: the new token's rows and the head's counters
+    uint4 kx = {}, vx = {}, qx = {};
+    int nt = 0, nb = 0;
+    long long off = 0;
+    bool dense = true;
+    if (FUSED) {
+      nt = p.ntok[i];
+      nb = p.nbuf[i];
+      dense = p.label[i] == HKV_DENSE;
+      off = p.off[h];
+      if (lane < RB / 16) {
+        kx = reinterpret_cast<const uint4 *>(static_cast<const unsigned char *>(p.k_new) + (size_t)h * RB)[lane];
+        vx = reinterpret_cast<const uint4 *>(static_cast<const unsigned char *>(p.v_new) + (size_t)h * RB)[lane];
+        qx = reinterpret_cast<const uint4 *>(static_cast<const unsigned char *>(p.q) + (size_t)h * RB)[lane];
+      }
+    }
+    const int vl = len + (FUSED ? 1 : 0);
+    float *orow = p.out + (size_t)h * D + CPL * lane;
+    if (vl == 0) {  // an empty head (plain attention) yields zeros
+      float z[CPL];
 #pragma unroll
-          for (int c = 0; c < CPL; ++c) GA[c] = 0.f;
-          for (long long cc = c0; cc <= c1; ++cc) {
-            const int slot = (cc == c0 && cc * chunk < hs) ? 1 : 0;
-            const float *qq = p.part + ((size_t)cc * 2 + slot) * (D + 2);
-            const float mc = __ldcg(qq + D), lc = __ldcg(qq + D + 1);
-            const float mn2 = fmaxf(gm, mc);
-            const float s0 = gm == -INFINITY ? 0.f : exp2f(gm - mn2);
-            const float s1 = exp2f(mc - mn2);
-            GL = GL * s0 + lc * s1;
+      for (int c = 0; c < CPL; ++c) z[c] = 0.f;
+      V::st(orow, z);
+      continue;
+    }
+    const long long he = hs + vl;
+    const long long k0 = hs / chunk, k1 = (he - 1) / chunk;
+    if (k0 < k1) {
+      // The head is split over the ranges of CTAs k0..k1. The maximum over
+      // the pieces first (lanes take pieces), then the weighted sums in index
+      // order; loads go out MB pieces at a time.
+      auto part_of = [&](long long kk) {
+        const int slot = (kk == k0 && kk * chunk < hs) ? 1 : 0;
+        return p.part + ((size_t)kk * 2 + slot) * PS;
+      };
+      const int np = (int)(k1 - k0 + 1);
+      float v[MB][CPL];
+      auto load_batch = [&](int t0) {  // pieces t0 .. t0 + MB - 1
 #pragma unroll
-            for (int c = 0; c < CPL; ++c) GA[c] = GA[c] * s0 + __ldcg(qq + lane + 32 * c) * s1;
-            gm = mn2;
+        for (int u = 0; u < MB; ++u) {
+          if (t0 + u < np) {
+            V::ldcg(part_of(k0 + t0 + u) + CPL * lane, v[u]);
+          } else {
+#pragma unroll
+            for (int c = 0; c < CPL; ++c) v[u][c] = 0.f;
           }
+        }
+      };
+      float m0 = -INFINITY, l0 = 0.f;  // the first 32 pieces' maxima and sums
+      if (lane < np) {
+        const float *qq = part_of(k0 + lane);
+        m0 = __ldcg(qq + D);
+        l0 = __ldcg(qq + D + 1);
+      }
+      load_batch(0);
+      float gm = m0;
+      for (int j = lane + 32; j < np; j += 32) gm = fmaxf(gm, __ldcg(part_of(k0 + j) + D));
 #pragma unroll
-          for (int c = 0; c < CPL; ++c) p.out[(size_t)h * D + lane + 32 * c] = GA[c] / GL;
-          if (lane == 0) p.cnt[h] = 0;
-          if (FUSED) append_row(h);
+      for (int o = 16; o >= 1; o >>= 1) gm = fmaxf(gm, __shfl_xor_sync(0xFFFFFFFFu, gm, o));
+      float GL = 0.f, GA[CPL];
+#pragma unroll
+      for (int c = 0; c < CPL; ++c) GA[c] = 0.f;
+      for (int j0 = 0; j0 < np; j0 += 32) {
+        float mj = m0, lj = l0;
+        if (j0 > 0) {
+          mj = -INFINITY;
+          lj = 0.f;
+          if (j0 + lane < np) {
+            const float *qq = part_of(k0 + j0 + lane);
+            mj = __ldcg(qq + D);
+            lj = __ldcg(qq + D + 1);
+          }
+        }
+        // weight of piece j0 + lane (zero past the last piece)
+        const float wj = mj == -INFINITY ? 0.f : exp2f(mj - gm);
+        const float lw = lj * wj;
+        const int cnt = np - j0 < 32 ? np - j0 : 32;
+        for (int t0 = 0; t0 < cnt; t0 += MB) {
+          if (j0 + t0 > 0) load_batch(j0 + t0);
+#pragma unroll
+          for (int u = 0; u < MB; ++u) {
+            const float w = __shfl_sync(0xFFFFFFFFu, wj, t0 + u);
+            GL += __shfl_sync(0xFFFFFFFFu, lw, t0 + u);
+#pragma unroll
+            for (int c = 0; c < CPL; ++c) GA[c] = fmaf(v[u][c], w, GA[c]);
+          }
         }
       }
-      if (fin) break;
+#pragma unroll
+      for (int c = 0; c < CPL; ++c) GA[c] /= GL;
+      V::st(orow, GA);
+    }
+    if (FUSED) {  // the new token: K/V row, position, query; then counters
+      const long long row = off + len;
+      if (lane < RB / 16) {
+        reinterpret_cast<uint4 *>(static_cast<unsigned char *>(p.K) + row * RB)[lane] = kx;
+        reinterpret_cast<uint4 *>(static_cast<unsigned char *>(p.V) + row * RB)[lane] = vx;
+        reinterpret_cast<uint4 *>(static_cast<unsigned char *>(p.qbuf) +
+                                  ((size_t)i * p.period + nt % p.period) * RB)[lane] = qx;
+      }
+      if (lane == 0) {
+        p.pos[row] = p.n_cond + nt;
+        p.len[h] = len + 1;
+        p.ntok[i] = nt + 1;
+        if (!dense) p.nbuf[i] = nb + 1;
+      }
     }
   }
-
-  if (FUSED && !early) grid_arrive();  // the CTAs that read lengths late
-  if (tid == 0) HKV_TRACE(6);
+  HKV_TRACE(22);
 }
 
 template <int D, typename T>
@@ -632,21 +848,31 @@ cudaError_t prepare_both(int *ctas) {
   return e;
 }
 
-template <int D, typename T>
-cudaError_t launch_t(const AttnArgs &a, int grid, bool fused, cudaStream_t s) {
+template <typename K>
+cudaError_t launch_pdl(K kernel, int grid, int threads, size_t smem, const AttnArgs &a,
+                       cudaStream_t s) {
   static const bool pdl = getenv("HKV_NO_PDL") == nullptr;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(kAttnThreads);
-  cfg.dynamicSmemBytes = smem_bytes<D, T>();
+  cfg.blockDim = dim3(threads);
+  cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  return fused ? cudaLaunchKernelEx(&cfg, attn_kernel<D, T, true>, a)
-               : cudaLaunchKernelEx(&cfg, attn_kernel<D, T, false>, a);
+  return cudaLaunchKernelEx(&cfg, kernel, a);
+}
+
+template <int D, typename T>
+cudaError_t launch_t(const AttnArgs &a, int grid, int finish_grid, bool fused, cudaStream_t s) {
+  cudaError_t e =
+      fused ? launch_pdl(attn_kernel<D, T, true>, grid, kAttnThreads, smem_bytes<D, T>(), a, s)
+            : launch_pdl(attn_kernel<D, T, false>, grid, kAttnThreads, smem_bytes<D, T>(), a, s);
+  if (e != cudaSuccess) return e;
+  return fused ? launch_pdl(finish_kernel<D, T, true>, finish_grid, kFinishThreads, 0, a, s)
+               : launch_pdl(finish_kernel<D, T, false>, finish_grid, kFinishThreads, 0, a, s);
 }
 
 }  // namespace
@@ -668,12 +894,13 @@ cudaError_t attention_prepare(int D, int dtype, int *ctas) {
   return D == 64 ? prepare_both<64, float>(ctas) : prepare_both<128, float>(ctas);
 }
 
-cudaError_t launch_attention(const AttnArgs &a, int D, int dtype, int grid, bool fused,
-                             cudaStream_t s) {
+cudaError_t launch_attention(const AttnArgs &a, int D, int dtype, int grid, int finish_grid,
+                             bool fused, cudaStream_t s) {
   if (dtype == HKV_BF16)
-    return D == 64 ? launch_t<64, __nv_bfloat16>(a, grid, fused, s)
-                   : launch_t<128, __nv_bfloat16>(a, grid, fused, s);
-  return D == 64 ? launch_t<64, float>(a, grid, fused, s) : launch_t<128, float>(a, grid, fused, s);
+    return D == 64 ? launch_t<64, __nv_bfloat16>(a, grid, finish_grid, fused, s)
+                   : launch_t<128, __nv_bfloat16>(a, grid, finish_grid, fused, s);
+  return D == 64 ? launch_t<64, float>(a, grid, finish_grid, fused, s)
+                 : launch_t<128, float>(a, grid, finish_grid, fused, s);
 }
 
 }  // namespace hkv

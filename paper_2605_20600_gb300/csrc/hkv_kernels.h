@@ -9,8 +9,17 @@
 
 namespace hkv {
 
-// split-K decode attention over one layer of a ragged cache, optionally
-// fused with the append of the step's new token
+// Written by block 0 of the attention kernel for the finishing kernel.
+struct AttnCtl {
+  long long chunk;   // indices of the work split per CTA
+  int grid;          // CTAs of the attention launch
+  int valid;         // 1: the attention launch passed its checks
+};
+
+// Split-K decode attention over one layer of a ragged cache, optionally
+// fused with the append of the step's new token: an attention kernel that
+// streams the cache and a finishing kernel that combines split heads,
+// appends the new token and advances the counters.
 struct AttnArgs {
   void *K, *V;                // arena
   const int64_t *off;         // layer slice of segment offsets
@@ -19,9 +28,9 @@ struct AttnArgs {
   const void *q;              // [nheads][D]
   const void *k_new, *v_new;  // [nheads][D] new token (fused)
   float *out;                 // [nheads][D]
-  float *part;                // [grid][2][D + 2] partial results
-  int32_t *cnt;               // [nheads] arrival counters (zero between calls)
-  int32_t *gcnt;              // grid arrival counter (fused; zero between calls)
+  float *part;                // [grid][2][attn_part_floats(D)] partial results
+  long long *hs;              // [nheads] where each head starts in the index space
+  AttnCtl *ctl;
   uint32_t *err;
   // fused append: full [L*S*H] arrays and the layer's first flat head
   int32_t *pos, *nbuf, *ntok;
@@ -37,18 +46,27 @@ struct AttnArgs {
 };
 
 // decode attention CTA: one producer warp (TMA), consumer warps, one
-// epilogue warp (merges, partial results, combine)
+// epilogue warp (merges, outputs, partial results)
 #ifndef HKV_ATTN_CONSUMER_WARPS
 #define HKV_ATTN_CONSUMER_WARPS 7
 #endif
 constexpr int kAttnConsumerWarps = HKV_ATTN_CONSUMER_WARPS;
 constexpr int kAttnThreads = 32 * (kAttnConsumerWarps + 2);  // + producer + epilogue
 constexpr int kAttnMaxGrid = 4096;
+constexpr int kFinishThreads = 32;  // finishing kernel: one warp per head and CTA
+// registers of a finishing thread: two of its CTAs fit in what three
+// attention CTAs leave of an SM's 64K registers
+constexpr int kFinishRegs = 48;
+// floats of one split-K partial result: D accumulators, the running maximum
+// and the sum, padded to 16 bytes for vector access
+__host__ __device__ constexpr int attn_part_floats(int D) { return D + 4; }
 
 size_t attention_smem_bytes(int D, int dtype);
 cudaError_t attention_prepare(int D, int dtype, int *ctas_per_sm);
-cudaError_t launch_attention(const AttnArgs &a, int D, int dtype, int grid, bool fused,
-                             cudaStream_t s);
+// launches the attention kernel on `grid` CTAs and the finishing kernel on
+// `finish_grid` CTAs
+cudaError_t launch_attention(const AttnArgs &a, int D, int dtype, int grid, int finish_grid,
+                             bool fused, cudaStream_t s);
 
 // per-head cache maintenance (append / update / repack / prefill / identify)
 struct CacheArgs {

@@ -22,11 +22,15 @@ namespace {
 
 using namespace hkv;
 
-// Split-K partials (up to 1 MiB) followed by one arrival counter per head of
-// a layer (up to 65536 heads): 1.25 MiB in total.
+// Split-K partials (up to 1 MiB), then where each head of a layer starts in
+// the attention kernel's index space (up to 65536 heads), then the control
+// block the attention kernel leaves for the finishing kernel: 1.5 MiB in
+// total. The kernels write all of it before reading it, so nothing in it has
+// to start at zero.
 constexpr size_t kPartBytes = 1u << 20;
 constexpr int kMaxHeadsPerLayer = 65536;
-constexpr size_t kScratchBytes = kPartBytes + (size_t)kMaxHeadsPerLayer * sizeof(int32_t);
+constexpr size_t kHsBytes = (size_t)kMaxHeadsPerLayer * sizeof(long long);
+constexpr size_t kScratchBytes = kPartBytes + kHsBytes + 256;
 
 static __device__ __align__(256) unsigned char g_scratch[kScratchBytes];
 
@@ -84,7 +88,7 @@ extern "C" hkv_status hkv_decode_attention_noalloc(const hkv_config *cfg, const 
     return HKV_ERR_ALIGN;
   if (layer < 0 || layer >= cfg->n_layers) return HKV_ERR_INVALID_ARG;
   const int hpl = cfg->n_seqs * cfg->n_heads;
-  if (hpl > kMaxHeadsPerLayer) return HKV_ERR_CAPACITY;  // counters would not fit
+  if (hpl > kMaxHeadsPerLayer) return HKV_ERR_CAPACITY;  // head starts would not fit
 
   NoAllocDevice *st = nullptr;
   const hkv_status ss = setup(cfg->head_dim, cfg->dtype, &st);
@@ -92,16 +96,15 @@ extern "C" hkv_status hkv_decode_attention_noalloc(const hkv_config *cfg, const 
   const int ctas = st->ctas[cfg->dtype == HKV_BF16 ? 1 : 0][cfg->head_dim == 128 ? 1 : 0];
 
   // as many CTAs as the partial area holds, at most the usual grid
-  const size_t per_cta = 2 * (size_t)(cfg->head_dim + 2) * sizeof(float);
+  const size_t per_cta = 2 * (size_t)attn_part_floats(cfg->head_dim) * sizeof(float);
   int grid = st->sms * ctas;
   if (grid > kAttnMaxGrid) grid = kAttnMaxGrid;
   if ((size_t)grid * per_cta > kPartBytes) grid = (int)(kPartBytes / per_cta);
+  const int per = kFinishThreads / 32;
+  int fgrid = (hpl + per - 1) / per;
+  if (fgrid > 2 * st->sms) fgrid = 2 * st->sms;
 
   cudaStream_t s = (cudaStream_t)stream;
-  int32_t *cnt = reinterpret_cast<int32_t *>(st->scratch + kPartBytes);
-  // the array keeps whatever the previous call left: start the counters at 0
-  if (cudaMemsetAsync(cnt, 0, (size_t)hpl * sizeof(int32_t), s) != cudaSuccess)
-    return HKV_ERR_CUDA;
 
   AttnArgs a = {};
   a.K = cache->k;
@@ -111,12 +114,13 @@ extern "C" hkv_status hkv_decode_attention_noalloc(const hkv_config *cfg, const 
   a.q = q;
   a.out = out;
   a.part = reinterpret_cast<float *>(st->scratch);
-  a.cnt = cnt;
+  a.hs = reinterpret_cast<long long *>(st->scratch + kPartBytes);
+  a.ctl = reinterpret_cast<AttnCtl *>(st->scratch + kPartBytes + kHsBytes);
   a.err = cache->err;
   a.arena_tokens = cache->capacity_tokens;
   a.nheads = hpl;
   a.qscale = (float)(1.4426950408889634 / sqrt((double)cfg->head_dim));
-  return launch_attention(a, cfg->head_dim, cfg->dtype, grid, false, s) == cudaSuccess
+  return launch_attention(a, cfg->head_dim, cfg->dtype, grid, fgrid, false, s) == cudaSuccess
              ? HKV_OK
              : HKV_ERR_CUDA;
 }
