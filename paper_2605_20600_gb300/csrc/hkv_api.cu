@@ -136,23 +136,30 @@ int max_segment(const hkv_config *c) {
   return a > b ? a : b;
 }
 
+size_t align256(size_t b) { return (b + 255) & ~(size_t)255; }
+
 // split-K partials: two slots per CTA
 size_t part_bytes(const hkv_config *c) {
-  const size_t b =
-      (size_t)kAttnMaxGrid * 2 * (size_t)attn_part_floats(c->head_dim) * sizeof(float);
-  return (b + 255) & ~(size_t)255;
+  return align256((size_t)kAttnMaxGrid * 2 * attn_part_floats(c->head_dim) * sizeof(float));
 }
 
-// where each head of a layer starts in the attention kernel's index space
-size_t hs_bytes(const hkv_config *c) {
-  return ((size_t)c->n_seqs * c->n_heads * sizeof(long long) + 255) & ~(size_t)255;
+// split-K partials: the first pieces of every head of a layer
+size_t inline_bytes(const hkv_config *c) {
+  return align256((size_t)c->n_seqs * c->n_heads * attn_inline_slots(c->head_dim) *
+                  attn_part_floats(c->head_dim) * sizeof(float));
+}
+
+// where the pieces of each head of a layer are
+size_t pieces_bytes(const hkv_config *c) {
+  return align256((size_t)c->n_seqs * c->n_heads * sizeof(int2));
 }
 
 constexpr size_t kCtlBytes = 256;  // AttnCtl, padded
 
 // Fills the attention launch arguments for one layer; the workspace holds
-// the split-K partials, the heads' starts in the index space and the
-// control block the attention kernel leaves for the finishing kernel.
+// the split-K partials (per CTA, and inline per head), where each head's
+// pieces are and the control block the attention kernel leaves for the
+// finishing kernel.
 AttnArgs attn_args(const hkv_config *cfg, const hkv_cache *cache, int layer, const void *q,
                    float *out, void *workspace) {
   const int hpl = cfg->n_seqs * cfg->n_heads;
@@ -166,8 +173,11 @@ AttnArgs attn_args(const hkv_config *cfg, const hkv_cache *cache, int layer, con
   a.out = out;
   unsigned char *ws = static_cast<unsigned char *>(workspace);
   a.part = reinterpret_cast<float *>(ws);
-  a.hs = reinterpret_cast<long long *>(ws + part_bytes(cfg));
-  a.ctl = reinterpret_cast<AttnCtl *>(ws + part_bytes(cfg) + hs_bytes(cfg));
+  a.part_inline = reinterpret_cast<float *>(ws + part_bytes(cfg));
+  a.nis = attn_inline_slots(cfg->head_dim);
+  a.pieces = reinterpret_cast<int2 *>(ws + part_bytes(cfg) + inline_bytes(cfg));
+  a.ctl = reinterpret_cast<AttnCtl *>(ws + part_bytes(cfg) + inline_bytes(cfg) +
+                                      pieces_bytes(cfg));
   a.err = cache->err;
   a.pos = cache->pos;
   a.nbuf = cache->nbuf;
@@ -245,7 +255,7 @@ hkv_status hkv_validate_config(const hkv_config *c) {
 
 size_t hkv_workspace_size(const hkv_config *c) {
   if (!c || hkv_validate_config(c) != HKV_OK) return 0;
-  return part_bytes(c) + hs_bytes(c) + kCtlBytes;
+  return part_bytes(c) + inline_bytes(c) + pieces_bytes(c) + kCtlBytes;
 }
 
 hkv_status hkv_init_dense(const hkv_config *cfg, const hkv_cache *cache, hkv_stream_t stream) {

@@ -27,14 +27,16 @@
 //  * consumers take whole token rows with 16-byte lanes (a 256-byte bf16 row
 //    is 16 lanes), a shuffle-xor tree per row for q.k, online softmax in the
 //    log2 domain with fp32 accumulation;
-//  * no fences, atomics or cache writes: the kernel only reads the cache
-//    and writes outputs and partial results;
+//  * no fences or atomics;
+//
+//  * fused: the CTA whose range holds a head's last row appends the new
+//    token (K/V row, position, query for the periodic update): nothing in
+//    the launch reads them;
 //
 // finishing kernel (one warp per head, after the attention kernel completes)
 //  * merges the partial results of each split head in index order, so the
 //    result does not depend on timing;
-//  * fused: appends the new token (K/V row, position, query for the periodic
-//    update) and advances the head's length and counters;
+//  * fused: advances each head's length and counters;
 //
 //  * programmatic dependent launch: every thread of either kernel waits for
 //    the previous kernel of the stream (griddepcontrol.wait) before it reads
@@ -445,21 +447,9 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
   if (p.prefetch) pdl_wait();  // the step's inputs are visible from here on
   if (tid == 0) HKV_TRACE(2);
   pdl_launch_dependents();
-  // Block 0 tells the finishing kernel where every head starts and how the
-  // work was split (the workspace is free: the previous finishing kernel is
-  // done).
-  if (blockIdx.x == 0) {
-    long long st = slice_start;
-    for (int h = h_lo; h < h_hi; ++h) {
-      p.hs[h] = st;
-      st += slot_len<TT>(p.len[h] + (FUSED ? 1 : 0));
-    }
-    if (tid == 0) {
-      p.ctl->chunk = chunk;
-      p.ctl->grid = G;
-      p.ctl->valid = 1;
-    }
-  }
+  // the launch passed its checks (the workspace is free: the previous
+  // finishing kernel is done)
+  if (blockIdx.x == 0 && tid == 0) p.ctl->valid = 1;
 
   if (warp == 0) {
     // ---- producer ----------------------------------------------------------
@@ -664,15 +654,42 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
 #pragma unroll
         for (int c = 0; c < CPL; ++c) A[c] /= L;
         V::st(p.out + (size_t)h * D + CPL * lane, A);
+        if (lane == 0) p.pieces[h] = make_int2(1, 0);
       } else {
-        // Partial result of this CTA's range: it holds the end of one split
-        // head (slot 0) and the start of another (slot 1).
-        float *pp = p.part + ((size_t)blockIdx.x * 2 + (a < hs ? 1 : 0)) * PS;
+        // Piece j of the np CTA ranges the head touches; the CTA with its
+        // first piece records np and where piece 0 sits.
+        const long long k0 = hs / chunk;
+        const int j = (int)(blockIdx.x - k0);
+        const int s1 = a < hs ? 1 : 0;  // piece 0 starts inside this range
+        float *pp = j < p.nis ? p.part_inline + ((size_t)h * p.nis + j) * PS
+                              : p.part + ((size_t)blockIdx.x * 2 + s1) * PS;
         V::st(pp + CPL * lane, A);
         if (lane == 0) {
           pp[D] = mx;
           pp[D + 1] = L;
+          if (j == 0)
+            p.pieces[h] = make_int2((int)((he - 1) / chunk - k0 + 1), (int)(2 * k0 + s1));
         }
+      }
+      // Fused: the CTA whose range holds the head's last row appends the new
+      // token (K/V row at index len, its position, q into the ring of the
+      // periodic update). Nothing in this launch reads them; the finishing
+      // kernel advances the counters once every CTA is done.
+      if (FUSED && he <= b) {
+        const int i = p.layer_base + h;
+        const int len = (int)(he - hs) - 1;
+        const long long row = look.off(h) + len;
+        const int nt = p.ntok[i];
+        for (int c = lane; c < RB / 16; c += 32) {
+          const uint4 kx = reinterpret_cast<const uint4 *>(static_cast<const unsigned char *>(p.k_new) + (size_t)h * RB)[c];
+          const uint4 vx = reinterpret_cast<const uint4 *>(static_cast<const unsigned char *>(p.v_new) + (size_t)h * RB)[c];
+          const uint4 qx = reinterpret_cast<const uint4 *>(static_cast<const unsigned char *>(p.q) + (size_t)h * RB)[c];
+          reinterpret_cast<uint4 *>(static_cast<unsigned char *>(p.K) + row * RB)[c] = kx;
+          reinterpret_cast<uint4 *>(static_cast<unsigned char *>(p.V) + row * RB)[c] = vx;
+          reinterpret_cast<uint4 *>(static_cast<unsigned char *>(p.qbuf) +
+                                    ((size_t)i * p.period + nt % p.period) * RB)[c] = qx;
+        }
+        if (lane == 0) p.pos[row] = p.n_cond + nt;
       }
     }
     if (lane == 0) HKV_TRACE(5);
@@ -681,19 +698,17 @@ __global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p)
 }
 
 // One warp per head: merge the partial results of a split head in index
-// order; fused, append the new token and advance the head's counters. Every
-// load that does not depend on another goes out first, so a head costs about
-// two round trips to memory.
+// order; fused, advance the head's counters. A head's first pieces sit in
+// inline slots of its own and the attention kernel records how many pieces
+// there are, so every load goes out at once: a head whose pieces are all
+// inline costs one round trip to memory.
 template <int D, typename T, bool FUSED>
 __global__ void __maxnreg__(kFinishRegs)
     finish_kernel(const AttnArgs p) {
-  using S = AttnShape<D, T>;
-  constexpr int RB = S::kRB;
   constexpr int CPL = D / 32;
   using V = Vec<CPL>;
   constexpr int PS = attn_part_floats(D);
-  constexpr int MB = 16 / CPL;  // partial results loaded per batch
-  static_assert(RB / 16 <= 32, "one 16-byte piece of a row per lane");
+  constexpr int MB = attn_inline_slots(D);  // partial results loaded per batch
   // Let the next kernel (the next layer's attention) start its prologue now;
   // it waits for this kernel before it reads anything written here.
   HKV_TRACE(20);
@@ -703,85 +718,75 @@ __global__ void __maxnreg__(kFinishRegs)
   const int lane = threadIdx.x & 31;
   const int nw = gridDim.x * (kFinishThreads / 32);
   const int w0 = blockIdx.x * (kFinishThreads / 32) + (threadIdx.x >> 5);
+  const int nis = p.nis;
   const int valid = p.ctl->valid;
-  const long long chunk = p.ctl->chunk;
-  if (!valid) return;
 
   for (int h = w0; h < p.nheads; h += nw) {
+    // One round of loads, none depending on another: where the head's pieces
+    // are, the maxima, sums and accumulators of its inline pieces and the
+    // head's counters. Inline slots past the piece count hold older data and
+    // are not used.
     const int i = p.layer_base + h;
+    const float *rec = p.part_inline + (size_t)h * nis * PS;
+    const int2 pc = p.pieces[h];
+    float m0 = -INFINITY, l0 = 0.f;
+    if (lane < nis) {
+      m0 = __ldcg(rec + (size_t)lane * PS + D);
+      l0 = __ldcg(rec + (size_t)lane * PS + D + 1);
+    }
+    float v[MB][CPL];
+#pragma unroll
+    for (int u = 0; u < MB; ++u) {
+      if (u < nis) {
+        V::ldcg(rec + (size_t)u * PS + CPL * lane, v[u]);
+      } else {
+#pragma unroll
+        for (int c = 0; c < CPL; ++c) v[u][c] = 0.f;
+      }
+    }
     const int len = p.len[h];
-    const long long hs = p.hs[h];
-    // fused: the new token's rows and the head's counters
-    uint4 kx = {}, vx = {}, qx = {};
     int nt = 0, nb = 0;
-    long long off = 0;
     bool dense = true;
     if (FUSED) {
       nt = p.ntok[i];
       nb = p.nbuf[i];
       dense = p.label[i] == HKV_DENSE;
-      off = p.off[h];
-      if (lane < RB / 16) {
-        kx = reinterpret_cast<const uint4 *>(static_cast<const unsigned char *>(p.k_new) + (size_t)h * RB)[lane];
-        vx = reinterpret_cast<const uint4 *>(static_cast<const unsigned char *>(p.v_new) + (size_t)h * RB)[lane];
-        qx = reinterpret_cast<const uint4 *>(static_cast<const unsigned char *>(p.q) + (size_t)h * RB)[lane];
-      }
     }
-    const int vl = len + (FUSED ? 1 : 0);
-    float *orow = p.out + (size_t)h * D + CPL * lane;
-    if (vl == 0) {  // an empty head (plain attention) yields zeros
-      float z[CPL];
+    if (!valid) return;  // the attention launch failed its checks
+    if (!FUSED && len == 0) {  // an empty head (plain attention) yields zeros; it
+      float z[CPL];            // has no tiles, so its pieces are not recorded
 #pragma unroll
       for (int c = 0; c < CPL; ++c) z[c] = 0.f;
-      V::st(orow, z);
+      V::st(p.out + (size_t)h * D + CPL * lane, z);
       continue;
     }
-    const long long he = hs + vl;
-    const long long k0 = hs / chunk, k1 = (he - 1) / chunk;
-    if (k0 < k1) {
-      // The head is split over the ranges of CTAs k0..k1. The maximum over
-      // the pieces first (lanes take pieces), then the weighted sums in index
-      // order; loads go out MB pieces at a time.
-      auto part_of = [&](long long kk) {
-        const int slot = (kk == k0 && kk * chunk < hs) ? 1 : 0;
-        return p.part + ((size_t)kk * 2 + slot) * PS;
+    const int np = pc.x;
+    if (np > 1) {
+      // Merge in piece (index) order: the maximum first, then the weighted
+      // sums. Pieces past the inline ones load MB at a time.
+      auto piece = [&](int j) {
+        return j < nis ? rec + (size_t)j * PS
+                       : p.part + (size_t)(j == 0 ? pc.y : pc.y - (pc.y & 1) + 2 * j) * PS;
       };
-      const int np = (int)(k1 - k0 + 1);
-      float v[MB][CPL];
-      auto load_batch = [&](int t0) {  // pieces t0 .. t0 + MB - 1
-#pragma unroll
-        for (int u = 0; u < MB; ++u) {
-          if (t0 + u < np) {
-            V::ldcg(part_of(k0 + t0 + u) + CPL * lane, v[u]);
-          } else {
-#pragma unroll
-            for (int c = 0; c < CPL; ++c) v[u][c] = 0.f;
-          }
-        }
-      };
-      float m0 = -INFINITY, l0 = 0.f;  // the first 32 pieces' maxima and sums
-      if (lane < np) {
-        const float *qq = part_of(k0 + lane);
-        m0 = __ldcg(qq + D);
-        l0 = __ldcg(qq + D + 1);
-      }
-      load_batch(0);
-      float gm = m0;
-      for (int j = lane + 32; j < np; j += 32) gm = fmaxf(gm, __ldcg(part_of(k0 + j) + D));
+      const bool all_inline = np <= nis;
+      float gm = lane < np && lane < nis ? m0 : -INFINITY;
+      for (int j = (all_inline ? 32 : (lane < nis ? lane + 32 : lane)); j < np; j += 32)
+        gm = fmaxf(gm, __ldcg(piece(j) + D));
 #pragma unroll
       for (int o = 16; o >= 1; o >>= 1) gm = fmaxf(gm, __shfl_xor_sync(0xFFFFFFFFu, gm, o));
       float GL = 0.f, GA[CPL];
 #pragma unroll
       for (int c = 0; c < CPL; ++c) GA[c] = 0.f;
       for (int j0 = 0; j0 < np; j0 += 32) {
-        float mj = m0, lj = l0;
-        if (j0 > 0) {
-          mj = -INFINITY;
-          lj = 0.f;
-          if (j0 + lane < np) {
-            const float *qq = part_of(k0 + j0 + lane);
-            mj = __ldcg(qq + D);
-            lj = __ldcg(qq + D + 1);
+        float mj = -INFINITY, lj = 0.f;
+        const int j = j0 + lane;
+        if (j < np) {
+          if (j < nis) {
+            mj = m0;
+            lj = l0;
+          } else {
+            mj = __ldcg(piece(j) + D);
+            lj = __ldcg(piece(j) + D + 1);
           }
         }
         // weight of piece j0 + lane (zero past the last piece)
@@ -789,34 +794,35 @@ __global__ void __maxnreg__(kFinishRegs)
         const float lw = lj * wj;
         const int cnt = np - j0 < 32 ? np - j0 : 32;
         for (int t0 = 0; t0 < cnt; t0 += MB) {
-          if (j0 + t0 > 0) load_batch(j0 + t0);
+          if (j0 + t0 >= nis) {
+#pragma unroll
+            for (int u = 0; u < MB; ++u) {
+              if (j0 + t0 + u < np) {
+                V::ldcg(piece(j0 + t0 + u) + CPL * lane, v[u]);
+              } else {
+#pragma unroll
+                for (int c = 0; c < CPL; ++c) v[u][c] = 0.f;
+              }
+            }
+          }
 #pragma unroll
           for (int u = 0; u < MB; ++u) {
             const float w = __shfl_sync(0xFFFFFFFFu, wj, t0 + u);
             GL += __shfl_sync(0xFFFFFFFFu, lw, t0 + u);
+            if (j0 + t0 + u < np)  // an unused inline slot may hold anything
 #pragma unroll
-            for (int c = 0; c < CPL; ++c) GA[c] = fmaf(v[u][c], w, GA[c]);
+              for (int c = 0; c < CPL; ++c) GA[c] = fmaf(v[u][c], w, GA[c]);
           }
         }
       }
 #pragma unroll
       for (int c = 0; c < CPL; ++c) GA[c] /= GL;
-      V::st(orow, GA);
+      V::st(p.out + (size_t)h * D + CPL * lane, GA);
     }
-    if (FUSED) {  // the new token: K/V row, position, query; then counters
-      const long long row = off + len;
-      if (lane < RB / 16) {
-        reinterpret_cast<uint4 *>(static_cast<unsigned char *>(p.K) + row * RB)[lane] = kx;
-        reinterpret_cast<uint4 *>(static_cast<unsigned char *>(p.V) + row * RB)[lane] = vx;
-        reinterpret_cast<uint4 *>(static_cast<unsigned char *>(p.qbuf) +
-                                  ((size_t)i * p.period + nt % p.period) * RB)[lane] = qx;
-      }
-      if (lane == 0) {
-        p.pos[row] = p.n_cond + nt;
-        p.len[h] = len + 1;
-        p.ntok[i] = nt + 1;
-        if (!dense) p.nbuf[i] = nb + 1;
-      }
+    if (FUSED && lane == 0) {  // the new token joined the head in the attention kernel
+      p.len[h] = len + 1;
+      p.ntok[i] = nt + 1;
+      if (!dense) p.nbuf[i] = nb + 1;
     }
   }
   HKV_TRACE(22);

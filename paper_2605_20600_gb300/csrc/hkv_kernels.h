@@ -11,9 +11,8 @@ namespace hkv {
 
 // Written by block 0 of the attention kernel for the finishing kernel.
 struct AttnCtl {
-  long long chunk;   // indices of the work split per CTA
-  int grid;          // CTAs of the attention launch
   int valid;         // 1: the attention launch passed its checks
+  int pad[3];
 };
 
 // Split-K decode attention over one layer of a ragged cache, optionally
@@ -28,8 +27,14 @@ struct AttnArgs {
   const void *q;              // [nheads][D]
   const void *k_new, *v_new;  // [nheads][D] new token (fused)
   float *out;                 // [nheads][D]
-  float *part;                // [grid][2][attn_part_floats(D)] partial results
-  long long *hs;              // [nheads] where each head starts in the index space
+  // Partial results (attn_part_floats(D) floats each) of a head split over
+  // the ranges of CTAs k0 .. k0 + np - 1: piece j < nis in the head's inline
+  // slot part_inline[h][j], else in the CTA slots part[2 * (k0 + j) + s]
+  // (s = 1 only for a piece 0 that starts inside its CTA's range).
+  float *part;                // [grid][2][...]
+  float *part_inline;         // [nheads][nis][...]
+  int nis;                    // inline slots per head (0: none)
+  int2 *pieces;               // [nheads] {np (1: not split), 2 * k0 + s of piece 0}
   AttnCtl *ctl;
   uint32_t *err;
   // fused append: full [L*S*H] arrays and the layer's first flat head
@@ -62,6 +67,8 @@ constexpr int kFinishRegs = 48;
 __host__ __device__ constexpr int attn_part_floats(int D) { return D + 4; }
 
 size_t attention_smem_bytes(int D, int dtype);
+// inline partial slots per head that the finishing kernel reads in one batch
+__host__ __device__ constexpr int attn_inline_slots(int D) { return 16 / (D / 32); }
 cudaError_t attention_prepare(int D, int dtype, int *ctas_per_sm);
 // launches the attention kernel on `grid` CTAs and the finishing kernel on
 // `finish_grid` CTAs

@@ -22,15 +22,15 @@ namespace {
 
 using namespace hkv;
 
-// Split-K partials (up to 1 MiB), then where each head of a layer starts in
-// the attention kernel's index space (up to 65536 heads), then the control
-// block the attention kernel leaves for the finishing kernel: 1.5 MiB in
-// total. The kernels write all of it before reading it, so nothing in it has
-// to start at zero.
+// Split-K partials (two per CTA, up to 1 MiB), then where the pieces of each
+// head of a layer are (up to 65536 heads), then the control block the
+// attention kernel leaves for the finishing kernel: 1.5 MiB in total. The
+// kernels write all of it before reading it, so nothing in it has to start
+// at zero.
 constexpr size_t kPartBytes = 1u << 20;
 constexpr int kMaxHeadsPerLayer = 65536;
-constexpr size_t kHsBytes = (size_t)kMaxHeadsPerLayer * sizeof(long long);
-constexpr size_t kScratchBytes = kPartBytes + kHsBytes + 256;
+constexpr size_t kPiecesBytes = (size_t)kMaxHeadsPerLayer * sizeof(int2);
+constexpr size_t kScratchBytes = kPartBytes + kPiecesBytes + 256;
 
 static __device__ __align__(256) unsigned char g_scratch[kScratchBytes];
 
@@ -88,7 +88,7 @@ extern "C" hkv_status hkv_decode_attention_noalloc(const hkv_config *cfg, const 
     return HKV_ERR_ALIGN;
   if (layer < 0 || layer >= cfg->n_layers) return HKV_ERR_INVALID_ARG;
   const int hpl = cfg->n_seqs * cfg->n_heads;
-  if (hpl > kMaxHeadsPerLayer) return HKV_ERR_CAPACITY;  // head starts would not fit
+  if (hpl > kMaxHeadsPerLayer) return HKV_ERR_CAPACITY;  // piece records would not fit
 
   NoAllocDevice *st = nullptr;
   const hkv_status ss = setup(cfg->head_dim, cfg->dtype, &st);
@@ -114,8 +114,9 @@ extern "C" hkv_status hkv_decode_attention_noalloc(const hkv_config *cfg, const 
   a.q = q;
   a.out = out;
   a.part = reinterpret_cast<float *>(st->scratch);
-  a.hs = reinterpret_cast<long long *>(st->scratch + kPartBytes);
-  a.ctl = reinterpret_cast<AttnCtl *>(st->scratch + kPartBytes + kHsBytes);
+  a.nis = 0;  // no inline slots: every piece in the CTA slots
+  a.pieces = reinterpret_cast<int2 *>(st->scratch + kPartBytes);
+  a.ctl = reinterpret_cast<AttnCtl *>(st->scratch + kPartBytes + kPiecesBytes);
   a.err = cache->err;
   a.arena_tokens = cache->capacity_tokens;
   a.nheads = hpl;

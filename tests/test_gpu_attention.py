@@ -51,9 +51,9 @@ def run_case(lens, D, dtype, seed, n_layers=1, layer=0, repeat=2):
         outs.append(out.cpu().numpy())
     H.hkv_check(cb.c)
     # the workspace ends with the kernels' 256-byte control block: the launch
-    # passed its checks (int32 at byte 12)
+    # passed its checks (int32 at byte 0)
     ctl = ws[-256:].view(torch.int32)
-    assert int(ctl[3]) == 1
+    assert int(ctl[0]) == 1
     Kx = cb.k.float().cpu().numpy().astype(np.float64)
     Vx = cb.v.float().cpu().numpy().astype(np.float64)
     qx = q.float().cpu().numpy().astype(np.float64)
