@@ -72,6 +72,15 @@ def describe(w, n_steps_window):
             f"period of P decode steps x L layers")
 
 
+def bench_config(w, world):
+    """The workload both arms report (same keys, same values)."""
+    return {"workload": describe(w, w.period), "rho": str(w.rho),
+            "decode_steps_per_step": w.period, "layers": w.n_layers,
+            "window_start_step": steady_start(w),
+            "l2": "no flush: inputs and the per-step KV working set exceed L2",
+            "parallelism": "replicas" if world > 1 else "single GPU"}
+
+
 # ---------------------------------------------------------------------------
 # CPU oracle timing (the baseline leg; runs in spawned processes)
 # ---------------------------------------------------------------------------
@@ -128,7 +137,7 @@ def run_reference(args):
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1000.0 * (w.n_seqs / w.cfg_rows) * w.period / value,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": {"workload": describe(w, w.period)},
+        "data": "synthetic", "config": bench_config(w, args.gpus),
         "cpu_baseline": {"value": value, "unit": "image tokens/s", "cores": workers,
                          "kind": "oracle",
                          "sample": f"per step {4 * workers} random heads, one period each after "
@@ -367,12 +376,8 @@ def run_ours(args):
             "metric": METRIC, "value": value, "unit": "image tokens/s", "n_gpus": world,
             "steps": K, "warmup": W, "ms_per_step": ms / K, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-            "config": {"workload": describe(w, P), "rho": str(w.rho),
-                       "decode_steps_per_step": P, "layers": L,
-                       "global_head_fraction": float((labels == 1).mean()),
-                       "window_start_step": t0,
-                       "l2": "no flush: inputs and the per-step KV working set exceed L2",
-                       "parallelism": "replicas" if world > 1 else "single GPU"},
+            "config": bench_config(w, world),
+            "global_head_fraction": float((labels == 1).mean()),
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": None,
                          "kernel": "hkv_decode_step: attn_kernel<fused> + finish_kernel<fused>",

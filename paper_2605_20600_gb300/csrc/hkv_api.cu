@@ -194,7 +194,7 @@ AttnArgs attn_args(const hkv_config *cfg, const hkv_cache *cache, int layer, con
 }
 
 // attention CTAs: every SM filled; finishing CTAs: one warp per head, at
-// most two one-warp CTAs per SM (what fits beside three attention CTAs)
+// most two one-warp CTAs per SM (they fit beside the attention CTAs)
 hkv_status attn_grid(const hkv_config *cfg, int *grid, int *finish_grid) {
   DeviceState *st;
   hkv_status s = device_state(&st);

@@ -16,7 +16,7 @@
 //    (one round of loads), a block scan locates each CTA's first head, and a
 //    table of (offset, length, start) of the CTA's heads goes to shared
 //    memory;
-//  * warp-specialised pipeline: one producer warp streams K/V tiles of 7 KB
+//  * warp-specialised pipeline: one producer warp streams K/V tiles of 10.5 KB
 //    into shared memory with the TMA engine (1D cp.async.bulk) through NS
 //    stages guarded by full/empty mbarriers, each with a description of its
 //    tile; the query row of a head rides along with the head's first tile
@@ -59,13 +59,13 @@ namespace {
 // on resident CTAs per SM used to size the grid, tiles loaded before the
 // wait for the previous kernel (prefetch), tiles sent to L2 beyond those.
 #ifndef HKV_ATTN_TILE_BYTES
-#define HKV_ATTN_TILE_BYTES 7168
+#define HKV_ATTN_TILE_BYTES 10752
 #endif
 #ifndef HKV_ATTN_STAGES
 #define HKV_ATTN_STAGES 4
 #endif
 #ifndef HKV_ATTN_MAX_CTAS_PER_SM
-#define HKV_ATTN_MAX_CTAS_PER_SM 32
+#define HKV_ATTN_MAX_CTAS_PER_SM 2
 #endif
 #ifndef HKV_ATTN_PRE_TILES
 #define HKV_ATTN_PRE_TILES 3
@@ -242,7 +242,7 @@ struct Pending {
 };
 
 template <int D, typename T, bool FUSED>
-__global__ void __launch_bounds__(kAttnThreads, 3) attn_kernel(const AttnArgs p) {
+__global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p) {
   using S = AttnShape<D, T>;
   constexpr int LPR = S::kLPR, EPL = S::kEPL, RPW = S::kRPW, TT = S::kTT;
   constexpr int RB = S::kRB, NS = S::kNS;
