@@ -56,8 +56,8 @@ namespace hkv {
 namespace {
 
 // Tuning knobs (compile time): bytes of K per pipeline stage, stages, a cap
-// on resident CTAs per SM used to size the grid, tiles loaded before the
-// wait for the previous kernel (prefetch), tiles sent to L2 beyond those.
+// on resident CTAs per SM used to size the grid, and tiles loaded before the
+// wait for the previous kernel (prefetch).
 #ifndef HKV_ATTN_TILE_BYTES
 #define HKV_ATTN_TILE_BYTES 10752
 #endif
@@ -70,9 +70,7 @@ namespace {
 #ifndef HKV_ATTN_PRE_TILES
 #define HKV_ATTN_PRE_TILES 3
 #endif
-#ifndef HKV_ATTN_L2_TILES
-#define HKV_ATTN_L2_TILES 0
-#endif
+
 static_assert(HKV_ATTN_PRE_TILES >= 0 && HKV_ATTN_PRE_TILES <= HKV_ATTN_STAGES, "prefetch depth");
 
 constexpr int kCW = kAttnConsumerWarps;
@@ -421,28 +419,9 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
   };
   Pending pre[NS];
   int n_pre = 0;
-  if (producer) {
+  if (producer)
     for (; n_pre < (p.prefetch ? HKV_ATTN_PRE_TILES : NS) && !pit.done(); ++n_pre)
       issue_old(pre[n_pre]);
-    // While the previous kernels finish, the memory system would idle once
-    // those tiles are in: with prefetch, the next HKV_ATTN_L2_TILES tiles of
-    // old rows go to L2 as well.
-    if (p.prefetch && HKV_ATTN_L2_TILES > 0) {
-      TileIter<TT> it = pit;
-      for (int j = 0; j < HKV_ATTN_L2_TILES && !it.done(); ++j) {
-        const long long ge = it.tile_end();
-        const int r0 = (int)(it.g - it.hs), r1 = (int)(ge - it.hs);
-        const int real = FUSED ? it.hl - 1 : it.hl;
-        const int n_old = (r1 < real ? r1 : real) - r0;
-        if (n_old > 0) {
-          const long long row = look.off(it.h) + r0;
-          bulk_prefetch_l2(static_cast<const unsigned char *>(p.K) + row * RB, (uint32_t)n_old * RB);
-          bulk_prefetch_l2(static_cast<const unsigned char *>(p.V) + row * RB, (uint32_t)n_old * RB);
-        }
-        it.advance(look);
-      }
-    }
-  }
 
   if (p.prefetch) pdl_wait();  // the step's inputs are visible from here on
   if (tid == 0) HKV_TRACE(2);
@@ -753,6 +732,10 @@ __global__ void __maxnreg__(kFinishRegs)
       dense = p.label[i] == HKV_DENSE;
     }
     if (!valid) return;  // the attention launch failed its checks
+#ifdef HKV_ATTN_TRACE
+    if (g_trace && h == w0 && lane == 0 && (len + nt + nb + pc.x + (int)(m0 + l0 + v[0][0])) != 0x7fffffff)
+      HKV_TRACE_AT(23) = globaltimer();  // the first head's loads are back
+#endif
     if (!FUSED && len == 0) {  // an empty head (plain attention) yields zeros; it
       float z[CPL];            // has no tiles, so its pieces are not recorded
 #pragma unroll

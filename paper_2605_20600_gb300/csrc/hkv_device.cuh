@@ -133,12 +133,6 @@ __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t by
       : "memory");
 }
 
-// brings `bytes` (multiple of 16, 16-byte aligned) of global memory into L2
-// through the TMA engine, without a destination or completion
-__device__ __forceinline__ void bulk_prefetch_l2(const void *src, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
-}
-
 // ---------------------------------------------------------------------------
 // block-wide scans (all threads must call; `scratch` holds >= 33 entries)
 // ---------------------------------------------------------------------------
