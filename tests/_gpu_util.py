@@ -22,9 +22,11 @@ def flat(w, s, l, h):
     return (l * w.n_seqs + s) * w.n_heads + h
 
 
-def run_gpu(w, *, out_steps=(), pos_steps=(), pos_heads=(), last_step=None, fused=True):
-    """One generation on the GPU. Returns outputs {t: [L,S,H,D] fp32},
-    positions {t: {flat head: sorted positions}}, labels, n_h and the engine."""
+def run_gpu(w, *, out_steps=(), pos_steps=(), pos_heads=(), last_step=None, fused=True,
+            out_heads=None):
+    """One generation on the GPU. Returns outputs {t: [L,S,H,D] fp32, or
+    {(s, l, h): [D]} for out_heads}, positions {t: {flat head: sorted
+    positions}}, labels, n_h and the engine."""
     import torch
     from paper_2605_20600_gb300 import hkv as H
     from paper_2605_20600_gb300.engine import Engine
@@ -35,9 +37,16 @@ def run_gpu(w, *, out_steps=(), pos_steps=(), pos_heads=(), last_step=None, fuse
     out_steps, pos_steps = set(out_steps), set(pos_steps)
     outs, poss = {}, {}
 
+    if out_heads is not None:
+        sel = [torch.tensor([x[i] for x in out_heads], device="cuda") for i in (1, 0, 2)]
+
     def on_step(t, out):
         if t in out_steps:
-            outs[t] = out.cpu().numpy()
+            if out_heads is None:
+                outs[t] = out.cpu().numpy()
+            else:
+                rows = out[sel[0], sel[1], sel[2]].cpu().numpy()
+                outs[t] = {x: rows[j] for j, x in enumerate(out_heads)}
         if t in pos_steps:
             c = eng.cache
             off, ln = c.off.cpu().numpy(), c.len.cpu().numpy()
