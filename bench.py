@@ -72,6 +72,24 @@ def describe(w, n_steps_window):
             f"period of P decode steps x L layers")
 
 
+def max_over_ranks(x: float, device) -> float:
+    """The job's time is the slowest rank's: every rank calls this after its
+    timed region (no-op on one process)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_value(world, images_per_rank, steps_per_period, periods, ms) -> float:
+    """Whole-job image tokens/s: the tokens every rank produced over the
+    slowest rank's time."""
+    return world * images_per_rank * steps_per_period * periods / (ms / 1e3)
+
+
 def bench_config(w, world):
     """The workload both arms report (same keys, same values)."""
     return {"workload": describe(w, w.period), "rho": str(w.rho),
@@ -313,12 +331,9 @@ def run_ours(args):
     ms = ev0.elapsed_time(ev1)
     clocks = clk.summary()
     eng.check()
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms, dev)
     images = S / w.cfg_rows
-    value = world * images * P * K / (ms / 1e3)
+    value = job_value(world, images, P, K, ms)
 
     # dominant kernel: the fused decode step (append + attention). One more
     # period is replayed from a copy of the graph with an event pair around
