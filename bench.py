@@ -72,6 +72,32 @@ def describe(w, n_steps_window):
             f"period of P decode steps x L layers")
 
 
+def profiled_traffic(workload, bytes_per_launch, n_heads):
+    """DRAM bytes per decode step from the committed ncu summary: the
+    attention kernel's measured traffic ratio to its algorithmic bytes, scaled
+    to this launch, plus the finishing kernel's bytes per head. None for
+    another kernel instantiation (the capture is of the Lumina-1024 shape:
+    D = 128, bf16) or when the kernel source has changed since the capture."""
+    if workload != "lumina1024":
+        return None
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "decode_step_lumina1024_rho4.md")
+    src = os.path.join(ROOT, "paper_2605_20600_gb300", "csrc", "hkv_attention.cu")
+    try:
+        vals = {}
+        for line in open(path):
+            k, _, v = line.strip().partition(": ")
+            if k in ("source_sha256", "attn_traffic_ratio", "finish_traffic_bytes_per_head"):
+                vals[k] = v
+        with open(src, "rb") as f:
+            if hashlib.sha256(f.read()).hexdigest() != vals["source_sha256"]:
+                return None
+        return (float(vals["attn_traffic_ratio"]) * bytes_per_launch
+                + float(vals["finish_traffic_bytes_per_head"]) * n_heads)
+    except (OSError, KeyError, ValueError):
+        return None
+
+
 def max_over_ranks(x: float, device) -> float:
     """The job's time is the slowest rank's: every rank calls this after its
     timed region (no-op on one process)."""
@@ -419,9 +445,13 @@ def run_ours(args):
             "config": bench_config(w, world),
             "global_head_fraction": float((labels == 1).mean()),
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                         "frac": achieved / peak, "traffic": None,
+                         "frac": achieved / peak,
+                         "traffic": profiled_traffic(w.name, bytes_per_launch, S * Hh),
                          "kernel": "hkv_decode_step: attn_kernel<fused> + finish_kernel<fused>",
                          "bytes_per_launch": bytes_per_launch, "launch_us": attn_us,
+                         # the first step of the period, per layer (what a
+                         # profiler capturing the first launches sees)
+                         "bytes_first_step": per_launch[:L],
                          "launch_us_isolated": statistics.mean(step_us),
                          "evict_us_per_period": sum(evict_us), "copy_us_per_period": copy_us,
                          "peak_kind": peak_kind},
