@@ -188,7 +188,11 @@ hkv_status hkv_append_evict(const hkv_config *cfg, const hkv_cache *cache, int l
  * same update hkv_append_evict runs before its append, without the append.
  * Heads whose buffer is not full are left as they are, so the call is
  * harmless when no update is due; with hkv_decode_step it must run before
- * the step that follows the P-th buffered token. */
+ * the step that follows the P-th buffered token. The update stages the P
+ * buffered queries, then rows of keys, in shared memory: the larger of
+ * P * head_dim * elem and 256 * (head_dim * elem + 16) bytes, plus 16 bytes
+ * per token of the longest segment, must fit in 227 KB, else
+ * HKV_ERR_CAPACITY (also for hkv_append_evict and hkv_repack). */
 hkv_status hkv_evict(const hkv_config *cfg, const hkv_cache *cache, int layer, hkv_stream_t stream);
 
 /* One decode step of one layer: the append of the new token (Sec. 3, KV

@@ -291,7 +291,7 @@ hkv_status hkv_append_evict(const hkv_config *cfg, const hkv_cache *cache, int l
   if (!aligned16(q) || !aligned16(k) || !aligned16(v)) return HKV_ERR_ALIGN;
   DeviceState *st;
   HKV_TRY(device_state(&st));
-  const size_t smem = update_smem_bytes(max_segment(cfg), cfg->head_dim);
+  const size_t smem = update_smem_bytes(max_segment(cfg), cfg->head_dim, cfg->period, cfg->dtype);
   HKV_TRY(update_ready(st, cfg->head_dim, cfg->dtype, smem));
   const int hpl = heads_per_layer(cfg);
   return cuda_status(launch_append_evict(cache_args(cache), method_args(cfg), layer * hpl, hpl, q,
@@ -346,7 +346,7 @@ hkv_status hkv_evict(const hkv_config *cfg, const hkv_cache *cache, int layer,
   if (layer < 0 || layer >= cfg->n_layers) return HKV_ERR_INVALID_ARG;
   DeviceState *st;
   HKV_TRY(device_state(&st));
-  const size_t smem = update_smem_bytes(max_segment(cfg), cfg->head_dim);
+  const size_t smem = update_smem_bytes(max_segment(cfg), cfg->head_dim, cfg->period, cfg->dtype);
   HKV_TRY(update_ready(st, cfg->head_dim, cfg->dtype, smem));
   const int hpl = heads_per_layer(cfg);
   return cuda_status(launch_evict(cache_args(cache), method_args(cfg), layer * hpl, hpl,
@@ -366,7 +366,7 @@ hkv_status hkv_identify_heads(const hkv_config *cfg, const hkv_cache *cache, int
   HKV_TRY(device_state(&st));
   const int max_len = cfg->n_cond + cfg->group_at;
   HKV_TRY(update_ready(st, cfg->head_dim, cfg->dtype,
-                       update_smem_bytes(max_segment(cfg), cfg->head_dim)));
+                       update_smem_bytes(max_segment(cfg), cfg->head_dim, cfg->period, cfg->dtype)));
   const int hpl = heads_per_layer(cfg);
   return cuda_status(launch_identify(cache_args(cache), method_args(cfg), layer * hpl, hpl, q,
                                      label_out, nh_out, cfg->head_dim, cfg->dtype, max_len,
@@ -407,7 +407,7 @@ hkv_status hkv_repack(const hkv_config *cfg, const hkv_cache *dense, const hkv_c
   if (dense->qbuf != ragged->qbuf) return HKV_ERR_INVALID_ARG;
   DeviceState *st;
   HKV_TRY(device_state(&st));
-  const size_t smem = update_smem_bytes(max_segment(cfg), cfg->head_dim);
+  const size_t smem = update_smem_bytes(max_segment(cfg), cfg->head_dim, cfg->period, cfg->dtype);
   HKV_TRY(update_ready(st, cfg->head_dim, cfg->dtype, smem));
   const int hpl = heads_per_layer(cfg);
   return cuda_status(launch_repack(cache_args(dense), cache_args(ragged), method_args(cfg),

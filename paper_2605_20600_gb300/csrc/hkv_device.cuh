@@ -133,6 +133,16 @@ __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t by
       : "memory");
 }
 
+// 16-byte asynchronous global -> shared copy (both ends 16-byte aligned) and
+// the wait for all of the thread's outstanding ones
+__device__ __forceinline__ void cp_async16(void *dst, const void *src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;" ::: "memory");
+}
+
 // ---------------------------------------------------------------------------
 // block-wide scans (all threads must call; `scratch` holds >= 33 entries)
 // ---------------------------------------------------------------------------

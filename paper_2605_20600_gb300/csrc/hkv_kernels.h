@@ -96,8 +96,9 @@ struct MethodArgs {
 
 constexpr int kCacheThreads = 256;
 
-// dynamic shared memory of the update paths for segments of up to max_len tokens
-size_t update_smem_bytes(int max_len, int D);
+// dynamic shared memory of the update paths for segments of up to max_len
+// tokens and a query ring of P rows
+size_t update_smem_bytes(int max_len, int D, int P, int dtype);
 cudaError_t update_prepare(int D, int dtype, size_t smem);
 
 cudaError_t launch_append_evict(const CacheArgs &c, const MethodArgs &m, int layer_base,

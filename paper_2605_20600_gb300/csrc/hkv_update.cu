@@ -32,6 +32,21 @@ namespace {
 
 constexpr int NT = kCacheThreads;
 
+// Phase timestamps per head of the update for latency studies; compiled out
+// by default.
+#ifdef HKV_UPD_TRACE
+__device__ unsigned long long *g_utrace = nullptr;  // [head of the layer][8], set by the tracer
+#define HKV_UTRACE(slot)                                                   \
+  do {                                                                     \
+    if (g_utrace && threadIdx.x == 0)                                      \
+      g_utrace[(size_t)blockIdx.x * 8 + (slot)] = globaltimer();           \
+  } while (0)
+#else
+#define HKV_UTRACE(slot) \
+  do {                   \
+  } while (0)
+#endif
+
 __device__ __forceinline__ void pdl_wait() {
   asm volatile("griddepcontrol.wait;" ::: "memory");
 }
@@ -47,16 +62,20 @@ struct SegRef {
   int len;                       // live source rows
   int dst_cap;                   // destination capacity (rows)
   bool in_place;
+  uint32_t *err;                 // the cache's error word
 };
 
 struct UpdShared {
   unsigned long long prefix[2];
   int rem[2];
   int iscan[33];
+  long long lscan[33];
+  uint64_t ring_bar;  // completion of the bulk copy of the query ring
 };
 
 // Shared-memory work area of one update (dynamic).
 struct UpdSmem {
+  unsigned char *ring;       // [P][D] the buffered queries (<= 4 B each)
   unsigned long long *keys;  // [max_len]
   int *ps;                   // [max_len] positions of the source rows
   int *aux;                  // [max_len] class, then keep flag, then rank
@@ -64,9 +83,18 @@ struct UpdSmem {
   int *hist;                 // [512]
 };
 
-__device__ __forceinline__ UpdSmem carve(unsigned char *dyn, int max_len, int D) {
+// the query ring (P rows of es-byte elements); after q-bar it is the score
+// stage: NT/32 warps x 32 rows of D * es + 16 bytes
+__host__ __device__ constexpr size_t ring_bytes(int P, int D, int es) {
+  return (size_t)P * D * es > (size_t)(NT / 32) * 32 * (D * es + 16)
+             ? (size_t)P * D * es
+             : (size_t)(NT / 32) * 32 * (D * es + 16);
+}
+
+__device__ __forceinline__ UpdSmem carve(unsigned char *dyn, int max_len, int D, int P, int es) {
   UpdSmem u;
-  u.keys = reinterpret_cast<unsigned long long *>(dyn);
+  u.ring = dyn;
+  u.keys = reinterpret_cast<unsigned long long *>(dyn + ring_bytes(P, D, es));
   u.ps = reinterpret_cast<int *>(u.keys + max_len);
   u.aux = u.ps + max_len;
   u.qbar = reinterpret_cast<float *>(u.aux + max_len);
@@ -114,21 +142,30 @@ __device__ void radix_select2(const unsigned long long *keys, const int *cls, in
         const int incl = warp_incl_scan(sum);
         const int excl = incl - sum;
         if (excl < target && target <= incl) {
-          int run = excl, digit = -1, rem = 0;
+          int run = excl, digit = -1, rem = 0, in_bin = 0;
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
             if (digit < 0 && run + c[e] >= target) {
               digit = lane * 8 + e;
               rem = target - run;
+              in_bin = c[e];
             }
             run += c[e];
           }
           sh.prefix[s] |= (unsigned long long)digit << shift;
-          sh.rem[s] = rem;
+          if (rem == in_bin) {
+            // every key of this bin is among the k: the bin's upper end
+            // bounds exactly k keys (keys are unique), no further digit
+            sh.prefix[s] |= shift > 0 ? (1ull << shift) - 1ull : 0ull;
+            sh.rem[s] = 0;
+          } else {
+            sh.rem[s] = rem;
+          }
         }
       }
     }
     __syncthreads();
+    if (sh.rem[0] == 0 && sh.rem[1] == 0) break;
   }
 }
 
@@ -161,6 +198,7 @@ __device__ int select_evictions(const SegRef &sg, int label, const MethodArgs &m
     nh += hist ? 1 : 0;
   }
   const int NH = block_sum(nh, sh);  // history candidates (Eq. 2)
+  HKV_UTRACE(1);
   int M = 0;
   if (label == HKV_LOCAL) M = NH;    // Eq. 3: no history
   else if (NH > m.hist_budget) M = NH - m.hist_budget;
@@ -170,7 +208,9 @@ __device__ int select_evictions(const SegRef &sg, int label, const MethodArgs &m
     const int n_long = (int)floor((double)NH * m.r_s);
     if (n_long > 0 && n_long < NH) {
       for (int r = tid; r < sg.len; r += NT) u.keys[r] = (unsigned long long)(uint32_t)u.ps[r];
-      radix_select2(u.keys, u.aux, sg.len, n_long, 0, 24, u.hist, sh);
+      const int maxp = C + ntok;  // positions are below it: start at its top byte
+      const int top = maxp < (1 << 8) ? 0 : maxp < (1 << 16) ? 8 : maxp < (1 << 24) ? 16 : 24;
+      radix_select2(u.keys, u.aux, sg.len, n_long, 0, top, u.hist, sh);
       const int p_long = (int)sh.prefix[0];
       for (int r = tid; r < sg.len; r += NT)
         if (u.aux[r] == 0) u.aux[r] = u.ps[r] <= p_long ? 0 : 1;
@@ -178,35 +218,67 @@ __device__ int select_evictions(const SegRef &sg, int label, const MethodArgs &m
       for (int r = tid; r < sg.len; r += NT)
         if (u.aux[r] == 0) u.aux[r] = n_long == NH ? 0 : 1;
     }
-    // Eq. 6 scores: q-bar = the P buffered queries, oldest first
+    HKV_UTRACE(2);
+    // Eq. 6 scores: q-bar = the P buffered queries, oldest first. The ring
+    // comes in with one bulk copy; the sums keep their order.
     const int P = m.P;
+    if (tid == 0) {
+      mbar_init(&sh.ring_bar, 1);
+      fence_barrier_init();
+    }
+    __syncthreads();
+    if (tid == 0) {
+      const uint32_t bytes = (uint32_t)P * RB;
+      mbar_arrive_expect_tx(&sh.ring_bar, bytes);
+      bulk_g2s(u.ring, qring, bytes, &sh.ring_bar);
+    }
+    if (!mbar_wait(&sh.ring_bar, 0) && tid == 0) set_err(sg.err, HKV_ERR_TIMEOUT);
     for (int d = tid; d < D; d += NT) {
       float acc = 0.f;
       for (int pp = 0; pp < P; ++pp) {
         int slot = (ntok - P + pp) % P;
         if (slot < 0) slot += P;
-        acc = __fadd_rn(acc, Elem<T>::load1(qring, (size_t)slot * D + d));
+        acc = __fadd_rn(acc, Elem<T>::load1(u.ring, (size_t)slot * D + d));
       }
       u.qbar[d] = acc;
     }
     __syncthreads();
-    for (int r = tid; r < sg.len; r += NT) {
-      if (u.aux[r] < 0) continue;
-      const unsigned char *krow = sg.sk + (size_t)r * RB;
-      float s = 0.f;
-#pragma unroll 4
-      for (int pc = 0; pc < LPR; ++pc) {
-        float kf[EPL];
-        Elem<T>::unpack(*reinterpret_cast<const uint4 *>(krow + pc * 16), kf);
-#pragma unroll
-        for (int e = 0; e < EPL; ++e) s = __fadd_rn(s, __fmul_rn(u.qbar[pc * EPL + e], kf[e]));
+    HKV_UTRACE(3);
+    // Each warp stages 32 rows at a time in the (now free) ring area with
+    // coalesced 16-byte async copies, at a row stride of LPR + 1 pieces so
+    // that lane l reading row l, piece j, hits distinct banks; then lane l
+    // sums its row in the fixed order.
+    constexpr int RS = LPR + 1;  // row stride in 16-byte pieces
+    const int warp = tid >> 5, lane = tid & 31;
+    unsigned char *stage = u.ring + (size_t)warp * 32 * RS * 16;
+    for (int base = warp * 32; base < sg.len; base += (NT / 32) * 32) {
+      const int nrows = sg.len - base < 32 ? sg.len - base : 32;
+      for (int w = lane; w < nrows * LPR; w += 32) {
+        const int rr = w / LPR, pc = w % LPR;
+        cp_async16(stage + (rr * RS + pc) * 16, sg.sk + (size_t)(base + rr) * RB + pc * 16);
       }
-      s = __fadd_rn(s, 0.f);  // -0 reads as +0
-      uint32_t bits = __float_as_uint(s);
-      bits = (bits & 0x80000000u) ? ~bits : (bits | 0x80000000u);  // order-preserving
-      u.keys[r] = ((unsigned long long)bits << 32) | (uint32_t)u.ps[r];
+      cp_async_wait_all();
+      __syncwarp();
+      const int r = base + lane;
+      if (lane < nrows && u.aux[r] >= 0) {
+        const unsigned char *krow = stage + lane * RS * 16;
+        float s = 0.f;
+#pragma unroll 4
+        for (int pc = 0; pc < LPR; ++pc) {
+          float kf[EPL];
+          Elem<T>::unpack(*reinterpret_cast<const uint4 *>(krow + pc * 16), kf);
+#pragma unroll
+          for (int e = 0; e < EPL; ++e) s = __fadd_rn(s, __fmul_rn(u.qbar[pc * EPL + e], kf[e]));
+        }
+        s = __fadd_rn(s, 0.f);  // -0 reads as +0
+        uint32_t bits = __float_as_uint(s);
+        bits = (bits & 0x80000000u) ? ~bits : (bits | 0x80000000u);  // order-preserving
+        u.keys[r] = ((unsigned long long)bits << 32) | (uint32_t)u.ps[r];
+      }
+      __syncwarp();  // the stage is rewritten next round
     }
     __syncthreads();
+    HKV_UTRACE(4);
     // M/2 from each subset; a short subset hands its excess to the other
     int m_long = M / 2, m_near = M - M / 2;
     if (m_long > n_long) {
@@ -225,6 +297,7 @@ __device__ int select_evictions(const SegRef &sg, int label, const MethodArgs &m
                              : c == 1 ? (m_near > 0 && u.keys[r] <= thr1) : false;
       u.aux[r] = ev ? 0 : 1;
     }
+    HKV_UTRACE(5);
   } else {
     for (int r = tid; r < sg.len; r += NT) u.aux[r] = (u.aux[r] == 0 && M > 0) ? 0 : 1;
   }
@@ -245,39 +318,60 @@ __device__ __forceinline__ void copy_piece(unsigned char *dk, unsigned char *dv,
 // In place: the new length is len - M; every evicted row below it takes a
 // surviving row from above it (the i-th hole the i-th survivor). Sources
 // are all >= new_len and destinations < new_len, so the moves are
-// independent. Returns the new length.
+// independent. Each thread ranks a contiguous run of rows (one block scan
+// for holes and fills together), and each copy batch issues all of its
+// loads before its stores. Returns the new length.
 template <int D, typename T>
 __device__ int fill_holes(const SegRef &sg, int M, const UpdSmem &u, UpdShared &sh) {
   constexpr int RB = D * (int)sizeof(T);
   constexpr int LPR = RB / 16;
+  constexpr int B = 4;  // pieces per thread in flight
   const int tid = threadIdx.x;
-  const int new_len = sg.len - M;
-  if (M == 0) return sg.len;
-  // rank holes (evicted, r < new_len) and fills (kept, r >= new_len); the
-  // keys area is free now and holds the two index lists
-  int *hole = reinterpret_cast<int *>(u.keys);  // [<= M]
-  int *fill = hole + M;                          // [<= M]
-  int hrun = 0, frun = 0;
-  for (int base = 0; base < sg.len; base += NT) {
-    const int r = base + tid;
-    const int keep = r < sg.len ? u.aux[r] : 1;
-    const int is_hole = (r < new_len && !keep) ? 1 : 0;
-    const int is_fill = (r >= new_len && r < sg.len && keep) ? 1 : 0;
-    int ht, ft;
-    const int hx = block_excl_scan<int>(is_hole, sh.iscan, &ht);
-    const int fx = block_excl_scan<int>(is_fill, sh.iscan, &ft);
-    if (is_hole) hole[hrun + hx] = r;
-    if (is_fill) fill[frun + fx] = r;
-    hrun += ht;
-    frun += ft;
+  const int len = sg.len, new_len = len - M;
+  if (M == 0) return len;
+  // the keys area is free now and holds the two index lists
+  int *hole = reinterpret_cast<int *>(u.keys);  // [M]
+  int *fill = hole + M;                          // [M]
+  const int per = (len + NT - 1) / NT;
+  const int r0 = tid * per < len ? tid * per : len;
+  const int r1 = r0 + per < len ? r0 + per : len;
+  long long nh = 0, nf = 0;
+  for (int r = r0; r < r1; ++r) {
+    const int keep = u.aux[r];
+    nh += (r < new_len && !keep) ? 1 : 0;
+    nf += (r >= new_len && keep) ? 1 : 0;
+  }
+  long long tot;
+  const long long ex = block_excl_scan<long long>((nh << 32) | nf, sh.lscan, &tot);
+  int hp = (int)(ex >> 32), fp = (int)(ex & 0xFFFFFFFFll);
+  for (int r = r0; r < r1; ++r) {
+    const int keep = u.aux[r];
+    if (r < new_len && !keep) hole[hp++] = r;
+    if (r >= new_len && keep) fill[fp++] = r;
   }
   __syncthreads();
-  const int k = hrun < frun ? hrun : frun;  // equal by construction
-  for (int w = tid; w < k * LPR; w += NT) {
-    const int j = w / LPR, pc = w % LPR;
-    const int dr = hole[j], sr = fill[j];
-    copy_piece<D, T>(sg.dk + (size_t)dr * RB, sg.dv + (size_t)dr * RB, sg.sk + (size_t)sr * RB,
-                     sg.sv + (size_t)sr * RB, pc);
+  const int k = (int)(tot >> 32);  // = M: holes and fills pair up
+  const int total = k * LPR;
+  for (int w0 = 0; w0 < total; w0 += NT * B) {
+    uint4 kb[B], vb[B];
+#pragma unroll
+    for (int j = 0; j < B; ++j) {
+      const int w = w0 + j * NT + tid;
+      if (w < total) {
+        const size_t src = (size_t)fill[w / LPR] * RB + (w % LPR) * 16;
+        kb[j] = __ldcg(reinterpret_cast<const uint4 *>(sg.sk + src));
+        vb[j] = __ldcg(reinterpret_cast<const uint4 *>(sg.sv + src));
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < B; ++j) {
+      const int w = w0 + j * NT + tid;
+      if (w < total) {
+        const size_t dst = (size_t)hole[w / LPR] * RB + (w % LPR) * 16;
+        *reinterpret_cast<uint4 *>(sg.dk + dst) = kb[j];
+        *reinterpret_cast<uint4 *>(sg.dv + dst) = vb[j];
+      }
+    }
   }
   for (int j = tid; j < k; j += NT) sg.dpos[hole[j]] = u.ps[fill[j]];
   __syncthreads();
@@ -350,8 +444,11 @@ __global__ void __launch_bounds__(NT)
   unsigned char *V = static_cast<unsigned char *>(c.V) + off * RB;
   int32_t *pos = c.pos + off;
   const unsigned char *qring = static_cast<const unsigned char *>(c.qbuf) + (size_t)i * m.P * RB;
-  SegRef sg{K, V, pos, K, V, pos, len, cp, true};
-  const int nl = update_in_place<D, T>(sg, lab, m, qring, c.ntok[i], carve(dyn, max_len, D), sh);
+  SegRef sg{K, V, pos, K, V, pos, len, cp, true, c.err};
+  HKV_UTRACE(0);
+  const int nl =
+      update_in_place<D, T>(sg, lab, m, qring, c.ntok[i], carve(dyn, max_len, D, m.P, (int)sizeof(T)), sh);
+  HKV_UTRACE(6);
   if (tid == 0) {
     c.len[i] = nl;
     c.nbuf[i] = 0;
@@ -388,8 +485,8 @@ __global__ void __launch_bounds__(NT)
       if (tid == 0) set_err(c.err, HKV_ERR_CAPACITY);
       return;
     }
-    SegRef sg{K, V, pos, K, V, pos, len, cp, true};
-    len = update_in_place<D, T>(sg, lab, m, qring, ntok, carve(dyn, max_len, D), sh);
+    SegRef sg{K, V, pos, K, V, pos, len, cp, true, c.err};
+    len = update_in_place<D, T>(sg, lab, m, qring, ntok, carve(dyn, max_len, D, m.P, (int)sizeof(T)), sh);
     nbuf = 0;
   }
   if (len >= cp) {
@@ -456,9 +553,10 @@ __global__ void __launch_bounds__(NT)
             rg.pos + doff,
             slen,
             dcap,
-            false};
+            false,
+            rg.err};
   const unsigned char *qring = static_cast<const unsigned char *>(dn.qbuf) + (size_t)i * m.P * RB;
-  const UpdSmem u = carve(dyn, max_len, D);
+  const UpdSmem u = carve(dyn, max_len, D, m.P, (int)sizeof(T));
   const int M = select_evictions<D, T>(sg, lab, m, qring, dn.ntok[i], u, sh);
   if (slen - M > dcap) {
     if (tid == 0) set_err(rg.err, HKV_ERR_CAPACITY);
@@ -653,6 +751,17 @@ __global__ void budgets_kernel(const uint8_t *label, int32_t *budget, int32_t *c
   if (__syncthreads_or(bad) && threadIdx.x == 0) off[n - 1] = -1;  // reported as a state error
 }
 
+}  // namespace
+
+#ifdef HKV_UPD_TRACE
+// tracer builds only: where the update's phase timestamps go
+extern "C" int hkv_debug_set_utrace(unsigned long long *buf) {
+  return cudaMemcpyToSymbol(g_utrace, &buf, sizeof(buf)) == cudaSuccess ? 0 : 7;
+}
+#endif
+
+namespace {
+
 template <int D, typename T>
 cudaError_t prepare_t(size_t smem) {
   cudaError_t e = cudaFuncSetAttribute(append_evict_kernel<D, T>,
@@ -666,6 +775,14 @@ cudaError_t prepare_t(size_t smem) {
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(identify_kernel<D, T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
+  // all of an SM's L1 as shared memory, so that every head of a layer (one
+  // CTA each) is resident at once
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(evict_kernel<D, T>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             100);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(append_evict_kernel<D, T>,
+                             cudaFuncAttributePreferredSharedMemoryCarveout, 100);
   return e;
 }
 
@@ -713,16 +830,17 @@ cudaError_t pdl_launch(void (*kernel)(KArgs...), int grid, int block, size_t sme
   return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
 
-int max_len_of(size_t smem, int D) {
-  return (int)((smem - (size_t)D * 4 - 512 * 4 - 64) / 16);
+int max_len_of(size_t smem, int D, int P, int es) {
+  return (int)((smem - ring_bytes(P, D, es) - (size_t)D * 4 - 512 * 4 - 64) / 16);
 }
 
 }  // namespace
 
-size_t update_smem_bytes(int max_len, int D) {
-  // keys (8 B), positions (4 B), class/flag/rank (4 B) per row; q-bar; two
-  // 256-bin histograms
-  return (size_t)max_len * 16 + (size_t)D * 4 + 512 * 4 + 64;
+size_t update_smem_bytes(int max_len, int D, int P, int dtype) {
+  // the query ring / score stage; keys (8 B), positions (4 B), class/flag/
+  // rank (4 B) per row; q-bar; two 256-bin histograms
+  return ring_bytes(P, D, dtype == HKV_BF16 ? 2 : 4) + (size_t)max_len * 16 + (size_t)D * 4 +
+         512 * 4 + 64;
 }
 
 cudaError_t update_prepare(int D, int dtype, size_t smem) {
@@ -733,7 +851,7 @@ cudaError_t update_prepare(int D, int dtype, size_t smem) {
 cudaError_t launch_append_evict(const CacheArgs &c, const MethodArgs &m, int layer_base,
                                 int nheads, const void *q, const void *k, const void *v, int D,
                                 int dtype, size_t smem, cudaStream_t s) {
-  const int max_len = max_len_of(smem, D);
+  const int max_len = max_len_of(smem, D, m.P, dtype == HKV_BF16 ? 2 : 4);
   HKV_DISPATCH(D, dtype,
                return pdl_launch(append_evict_kernel<kD, kT>, nheads, NT, smem, s, c, m,
                                  layer_base, q, k, v, max_len));
@@ -742,7 +860,7 @@ cudaError_t launch_append_evict(const CacheArgs &c, const MethodArgs &m, int lay
 
 cudaError_t launch_evict(const CacheArgs &c, const MethodArgs &m, int layer_base, int nheads,
                          int D, int dtype, size_t smem, cudaStream_t s) {
-  const int max_len = max_len_of(smem, D);
+  const int max_len = max_len_of(smem, D, m.P, dtype == HKV_BF16 ? 2 : 4);
   HKV_DISPATCH(D, dtype,
                return pdl_launch(evict_kernel<kD, kT>, nheads, NT, smem, s, c, m, layer_base,
                                  max_len));
@@ -752,7 +870,7 @@ cudaError_t launch_evict(const CacheArgs &c, const MethodArgs &m, int layer_base
 cudaError_t launch_repack(const CacheArgs &dense, const CacheArgs &ragged, const MethodArgs &m,
                           int layer_base, int nheads, int D, int dtype, size_t smem,
                           cudaStream_t s) {
-  const int max_len = max_len_of(smem, D);
+  const int max_len = max_len_of(smem, D, m.P, dtype == HKV_BF16 ? 2 : 4);
   HKV_DISPATCH(D, dtype,
                return pdl_launch(repack_kernel<kD, kT>, nheads, NT, smem, s, dense, ragged, m,
                                  layer_base, max_len));
