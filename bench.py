@@ -468,6 +468,138 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+def run_strategies(args):
+    """--strategies: decode attention over one steady-state cache (every
+    layer, right after the period's update) three ways, as the paper's
+    alternatives for heads of different lengths: the ragged split-K kernel of
+    this library (hkv_decode_attention), padding every head to the longest
+    capacity with a key mask, and one dense batch per head group (local,
+    global). The two baselines run PyTorch's scaled_dot_product_attention on
+    padded tensors built once (the cache as it would be stored in that
+    layout); the outputs of all three are cross-checked."""
+    import numpy as np
+    import torch
+    import torch.nn.functional as F
+
+    from paper_2605_20600_gb300 import hkv as H
+    from paper_2605_20600_gb300.engine import Engine, torch_dtype
+    from paper_2605_20600_gb300.runner import generate
+    from synth.gpu import DeviceSynth
+
+    dev = torch.device("cuda", 0)
+    w = workload(args)
+    L, S, Hh, D, P = w.n_layers, w.n_seqs, w.n_heads, w.head_dim, w.period
+    t0 = steady_start(w)
+    cfg = H.make_config(n_layers=L, n_seqs=S, n_heads=Hh, head_dim=D, dtype=w.dtype,
+                        n_cond=w.n_cond, n_image=w.n_image, row_len=w.row_len,
+                        recent_w=w.recent_w, local_w=w.w_loc, period=P, group_at=w.group_at,
+                        rho=w.rho, tau=w.tau, r_s=w.r_s)
+    eng = Engine(cfg, dev)
+    synth = DeviceSynth(w, dev)
+    generate(eng, synth, last_step=t0 - 1)
+    eng.release_dense()
+    for layer in range(L):
+        eng.evict(layer)
+    torch.cuda.synchronize()
+    eng.check()
+    dt = torch_dtype(cfg)
+    q = torch.empty(1, L, S, Hh, D, dtype=dt, device=dev)
+    kk, vv = torch.empty_like(q), torch.empty_like(q)
+    synth.image(q, kk, vv, 0, L, t0, 1)
+    q = q[0]
+    c = eng.cache
+    n = S * Hh
+    off = c.off.view(L, n).long()
+    ln = c.len.view(L, n).long()
+    cap = c.cap.view(L, n).long()
+    lab = eng.labels.view(L, n)
+    es = 2 if cfg.dtype == 1 else 4
+    lmax = int(cap.max())
+
+    def padded(o, l, width):
+        """K, V [..., width, D] and mask [..., width] for heads at offsets o with
+        live lengths l (rows past the length repeat row 0 and are masked)."""
+        ar = torch.arange(width, device=dev)
+        mask = ar < l[..., None]
+        idx = torch.where(mask, o[..., None] + ar, o[..., None])
+        return c.k[idx], c.v[idx], mask
+
+    reps = max(3, args.steps)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+
+    def timed(fn):
+        for _ in range(2):
+            fn()
+        torch.cuda.synchronize()
+        ev[0].record()
+        for _ in range(reps):
+            fn()
+        ev[1].record()
+        torch.cuda.synchronize()
+        return ev[0].elapsed_time(ev[1]) * 1e3 / (reps * L)   # us per layer
+
+    out_ours = torch.empty(L, n, D, dtype=torch.float32, device=dev)
+
+    def ours():
+        for layer in range(L):
+            eng.attend(layer, q[layer], out_ours[layer])
+
+    us_ours = timed(ours)
+    eng.check()
+    bytes_ours = float((ln.sum() * D * 2 * es).item()) / L
+
+    Kp, Vp, Mp = padded(off, ln, lmax)
+    out_pad = torch.empty(L, n, D, dtype=dt, device=dev)
+
+    def pad():
+        for layer in range(L):
+            o = F.scaled_dot_product_attention(
+                q[layer].reshape(1, n, 1, D), Kp[layer].reshape(1, n, lmax, D),
+                Vp[layer].reshape(1, n, lmax, D), attn_mask=Mp[layer].reshape(1, n, 1, lmax))
+            out_pad[layer] = o.reshape(n, D)
+
+    us_pad = timed(pad)
+    bytes_pad = n * lmax * D * 2 * es
+    del Kp, Vp, Mp
+    # one dense batch per (layer, head group), each padded to its group's
+    # capacity, gathered before timing
+    batches = []
+    for layer in range(L):
+        for g in (0, 1):   # local, global
+            h = (lab[layer] == g).nonzero().flatten()
+            if len(h) == 0:
+                continue
+            width = int(cap[layer][h].max())
+            Kg, Vg, Mg = padded(off[layer][h], ln[layer][h], width)
+            batches.append((layer, h, q[layer].reshape(n, D)[h].contiguous(), Kg, Vg, Mg, width))
+    out_grp = torch.empty(L, n, D, dtype=dt, device=dev)
+
+    def grp():
+        for layer, h, qg, Kg, Vg, Mg, width in batches:
+            m = len(h)
+            o = F.scaled_dot_product_attention(
+                qg.reshape(1, m, 1, D), Kg.reshape(1, m, width, D), Vg.reshape(1, m, width, D),
+                attn_mask=Mg.reshape(1, m, 1, width))
+            out_grp[layer].index_copy_(0, h, o.reshape(m, D))
+
+    us_grp = timed(grp)
+    bytes_grp = sum(len(b[1]) * b[6] * D * 2 * es for b in batches) / L
+    err_pad = float((out_pad.float() - out_ours).abs().max())
+    err_grp = float((out_grp.float() - out_ours).abs().max())
+    peak, peak_kind = load_peaks()
+    line = {"strategies": describe(w, P), "unit": "us per layer (attention only)",
+            "ragged_splitk": {"us": us_ours, "retained_bytes": bytes_ours,
+                              "GBps": bytes_ours / us_ours / 1e3},
+            "padding_mask_sdpa": {"us": us_pad, "bytes_read": bytes_pad,
+                                  "GBps": bytes_pad / us_pad / 1e3, "max_abs_diff": err_pad},
+            "per_group_sdpa": {"us": us_grp, "bytes_read": bytes_grp,
+                               "GBps": bytes_grp / us_grp / 1e3, "max_abs_diff": err_grp},
+            "peak_GBps": peak, "peak_kind": peak_kind,
+            "note": "baselines: torch.nn.functional.scaled_dot_product_attention on padded "
+                    "tensors (library kernels); their padded tensors are built before timing"}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -478,7 +610,12 @@ def main():
     ap.add_argument("--rho", default="1/4")
     ap.add_argument("--seqs", type=int, default=0, help="override the batch (profiling runs)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--strategies", action="store_true",
+                    help="compare decode attention with the padding and per-group strategies")
     args = ap.parse_args()
+    if args.strategies:
+        run_strategies(args)
+        return
     if args.impl == "reference":
         if int(os.environ.get("RANK", "0")) == 0:
             run_reference(args)
