@@ -194,7 +194,8 @@ AttnArgs attn_args(const hkv_config *cfg, const hkv_cache *cache, int layer, con
 }
 
 // attention CTAs: every SM filled; finishing CTAs: one warp per head, at
-// most two one-warp CTAs per SM (they fit beside the attention CTAs)
+// most kFinishCtasPerSm one-warp CTAs per SM (they fit beside the attention
+// CTAs, so they start early and trigger the next launch early)
 hkv_status attn_grid(const hkv_config *cfg, int *grid, int *finish_grid) {
   DeviceState *st;
   hkv_status s = device_state(&st);
@@ -206,7 +207,7 @@ hkv_status attn_grid(const hkv_config *cfg, int *grid, int *finish_grid) {
   *grid = g > kAttnMaxGrid ? kAttnMaxGrid : g;
   const int per = kFinishThreads / 32;
   const int f = (heads_per_layer(cfg) + per - 1) / per;
-  *finish_grid = f < 2 * st->sms ? f : 2 * st->sms;
+  *finish_grid = f < kFinishCtasPerSm * st->sms ? f : kFinishCtasPerSm * st->sms;
   return HKV_OK;
 }
 

@@ -59,9 +59,10 @@ constexpr int kAttnConsumerWarps = HKV_ATTN_CONSUMER_WARPS;
 constexpr int kAttnThreads = 32 * (kAttnConsumerWarps + 2);  // + producer + epilogue
 constexpr int kAttnMaxGrid = 4096;
 constexpr int kFinishThreads = 32;  // finishing kernel: one warp per head and CTA
-// registers of a finishing thread: two of its CTAs fit in what two
-// attention CTAs leave of an SM's 64K registers
+// registers of a finishing thread, and how many finishing CTAs an SM takes
+// beside two attention CTAs (which leave ~14.8K of its 64K registers)
 constexpr int kFinishRegs = 64;
+constexpr int kFinishCtasPerSm = 6;
 // floats of one split-K partial result: D accumulators, the running maximum
 // and the sum, padded to 16 bytes for vector access
 __host__ __device__ constexpr int attn_part_floats(int D) { return D + 4; }

@@ -102,7 +102,7 @@ extern "C" hkv_status hkv_decode_attention_noalloc(const hkv_config *cfg, const 
   if ((size_t)grid * per_cta > kPartBytes) grid = (int)(kPartBytes / per_cta);
   const int per = kFinishThreads / 32;
   int fgrid = (hpl + per - 1) / per;
-  if (fgrid > 2 * st->sms) fgrid = 2 * st->sms;
+  if (fgrid > kFinishCtasPerSm * st->sms) fgrid = kFinishCtasPerSm * st->sms;
 
   cudaStream_t s = (cudaStream_t)stream;
 
