@@ -147,8 +147,8 @@ const char *hkv_status_str(hkv_status s);
 hkv_status hkv_validate_config(const hkv_config *cfg);
 
 /* Bytes of device workspace hkv_decode_attention and hkv_decode_step need
- * for this config (split-K partial results, where each head starts in the
- * work split, and a small control block the two kernels of a call share).
+ * for this config (split-K partial results, records of the heads split
+ * between CTAs, and a small control block the two kernels of a call share).
  * The workspace must be zero-filled before its first use; every call leaves
  * it ready for the next one (after a call that reported an error, zero it
  * again). Concurrent calls must not share a workspace. Host only. */
@@ -225,14 +225,13 @@ hkv_status hkv_decode_attention(const hkv_config *cfg, const hkv_cache *cache, i
  * the paper has no counterpart to this entry point. A plain C host program
  * without a device allocator, or a plugin inside a host framework that owns
  * and budgets all device memory, may have no way to provide the workspace
- * that hkv_decode_attention takes. Here the split-K partials, the heads'
- * starts in the work split and the kernels' control block live in a fixed
- * device array inside the library (1.5 MiB: 1 MiB of partials, 512 KiB for
- * up to 65536 heads, 256 bytes), which every GPU that loads the library
+ * that hkv_decode_attention takes. Here the split-K partials, the records
+ * of heads split between CTAs and the kernels' control block live in a
+ * fixed device array inside the library (1.06 MiB: 1 MiB of partials,
+ * 64 KiB of records, 256 bytes), which every GPU that loads the library
  * holds until the process exits. Nothing in it has to start at zero: each
  * call writes what it reads. Same inputs, outputs and results as
  * hkv_decode_attention; it allocates nothing.
- *  - More than 65536 heads per layer (n_seqs * n_heads) -> HKV_ERR_CAPACITY.
  *  - The first call on a device, with that device current, looks up the
  *    array's device address and prepares the kernel; make that first call
  *    before any stream capture.

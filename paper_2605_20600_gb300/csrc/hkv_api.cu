@@ -138,28 +138,25 @@ int max_segment(const hkv_config *c) {
 
 size_t align256(size_t b) { return (b + 255) & ~(size_t)255; }
 
-// split-K partials: two slots per CTA
+// split-K partials: kAttnInlinePieces slots per CTA boundary, one overflow
+// slot per CTA
 size_t part_bytes(const hkv_config *c) {
-  return align256((size_t)kAttnMaxGrid * 2 * attn_part_floats(c->head_dim) * sizeof(float));
+  return align256((size_t)kAttnMaxGrid * kAttnInlinePieces * attn_part_floats(c->head_dim) *
+                  sizeof(float));
+}
+size_t over_bytes(const hkv_config *c) {
+  return align256((size_t)kAttnMaxGrid * attn_part_floats(c->head_dim) * sizeof(float));
 }
 
-// split-K partials: the first pieces of every head of a layer
-size_t inline_bytes(const hkv_config *c) {
-  return align256((size_t)c->n_seqs * c->n_heads * attn_inline_slots(c->head_dim) *
-                  attn_part_floats(c->head_dim) * sizeof(float));
-}
-
-// where the pieces of each head of a layer are
-size_t pieces_bytes(const hkv_config *c) {
-  return align256((size_t)c->n_seqs * c->n_heads * sizeof(int2));
-}
+// where the head split at each CTA boundary is
+size_t rec_bytes() { return align256((size_t)kAttnMaxGrid * sizeof(int4)); }
 
 constexpr size_t kCtlBytes = 256;  // AttnCtl, padded
 
 // Fills the attention launch arguments for one layer; the workspace holds
-// the split-K partials (per CTA, and inline per head), where each head's
-// pieces are and the control block the attention kernel leaves for the
-// finishing kernel.
+// the split-K partials (per CTA boundary, and overflow slots per CTA), which
+// head is split at each CTA boundary and the control block the attention
+// kernel leaves for the finishing kernel.
 AttnArgs attn_args(const hkv_config *cfg, const hkv_cache *cache, int layer, const void *q,
                    float *out, void *workspace) {
   const int hpl = cfg->n_seqs * cfg->n_heads;
@@ -173,11 +170,9 @@ AttnArgs attn_args(const hkv_config *cfg, const hkv_cache *cache, int layer, con
   a.out = out;
   unsigned char *ws = static_cast<unsigned char *>(workspace);
   a.part = reinterpret_cast<float *>(ws);
-  a.part_inline = reinterpret_cast<float *>(ws + part_bytes(cfg));
-  a.nis = attn_inline_slots(cfg->head_dim);
-  a.pieces = reinterpret_cast<int2 *>(ws + part_bytes(cfg) + inline_bytes(cfg));
-  a.ctl = reinterpret_cast<AttnCtl *>(ws + part_bytes(cfg) + inline_bytes(cfg) +
-                                      pieces_bytes(cfg));
+  a.over = reinterpret_cast<float *>(ws + part_bytes(cfg));
+  a.rec = reinterpret_cast<int4 *>(ws + part_bytes(cfg) + over_bytes(cfg));
+  a.ctl = reinterpret_cast<AttnCtl *>(ws + part_bytes(cfg) + over_bytes(cfg) + rec_bytes());
   a.err = cache->err;
   a.pos = cache->pos;
   a.nbuf = cache->nbuf;
@@ -193,21 +188,16 @@ AttnArgs attn_args(const hkv_config *cfg, const hkv_cache *cache, int layer, con
   return a;
 }
 
-// attention CTAs: every SM filled; finishing CTAs: one warp per head, at
-// most kFinishCtasPerSm one-warp CTAs per SM (they fit beside the attention
-// CTAs, so they start early and trigger the next launch early)
-hkv_status attn_grid(const hkv_config *cfg, int *grid, int *finish_grid) {
+// attention CTAs: every SM filled
+hkv_status attn_grid(const hkv_config *cfg, int *grid) {
   DeviceState *st;
   hkv_status s = device_state(&st);
   if (s != HKV_OK) return s;
   int ctas = 0;
   s = attention_ctas(st, cfg->head_dim, cfg->dtype, &ctas);
   if (s != HKV_OK) return s;
-  int g = st->sms * ctas;
+  const int g = st->sms * ctas;
   *grid = g > kAttnMaxGrid ? kAttnMaxGrid : g;
-  const int per = kFinishThreads / 32;
-  const int f = (heads_per_layer(cfg) + per - 1) / per;
-  *finish_grid = f < kFinishCtasPerSm * st->sms ? f : kFinishCtasPerSm * st->sms;
   return HKV_OK;
 }
 
@@ -256,7 +246,7 @@ hkv_status hkv_validate_config(const hkv_config *c) {
 
 size_t hkv_workspace_size(const hkv_config *c) {
   if (!c || hkv_validate_config(c) != HKV_OK) return 0;
-  return part_bytes(c) + inline_bytes(c) + pieces_bytes(c) + kCtlBytes;
+  return part_bytes(c) + over_bytes(c) + rec_bytes() + kCtlBytes;
 }
 
 hkv_status hkv_init_dense(const hkv_config *cfg, const hkv_cache *cache, hkv_stream_t stream) {
@@ -310,11 +300,11 @@ hkv_status hkv_decode_attention(const hkv_config *cfg, const hkv_cache *cache, i
   if (!q || !out || !workspace) return HKV_ERR_INVALID_ARG;
   if (!aligned16(q) || !aligned16(out) || !aligned16(workspace)) return HKV_ERR_ALIGN;
   if (ws_bytes < hkv_workspace_size(cfg)) return HKV_ERR_CAPACITY;
-  int grid = 0, fgrid = 0;
-  HKV_TRY(attn_grid(cfg, &grid, &fgrid));
+  int grid = 0;
+  HKV_TRY(attn_grid(cfg, &grid));
   const AttnArgs a = attn_args(cfg, cache, layer, q, out, workspace);
   return cuda_status(
-      launch_attention(a, cfg->head_dim, cfg->dtype, grid, fgrid, false, (cudaStream_t)stream));
+      launch_attention(a, cfg->head_dim, cfg->dtype, grid, false, (cudaStream_t)stream));
 }
 
 hkv_status hkv_decode_step(const hkv_config *cfg, const hkv_cache *cache, int layer,
@@ -329,14 +319,14 @@ hkv_status hkv_decode_step(const hkv_config *cfg, const hkv_cache *cache, int la
     return HKV_ERR_ALIGN;
   if (ws_bytes < hkv_workspace_size(cfg)) return HKV_ERR_CAPACITY;
   if (flags & ~HKV_STEP_PREFETCH) return HKV_ERR_INVALID_ARG;
-  int grid = 0, fgrid = 0;
-  HKV_TRY(attn_grid(cfg, &grid, &fgrid));
+  int grid = 0;
+  HKV_TRY(attn_grid(cfg, &grid));
   AttnArgs a = attn_args(cfg, cache, layer, q, out, workspace);
   a.k_new = k;
   a.v_new = v;
   a.prefetch = (flags & HKV_STEP_PREFETCH) ? 1 : 0;
   return cuda_status(
-      launch_attention(a, cfg->head_dim, cfg->dtype, grid, fgrid, true, (cudaStream_t)stream));
+      launch_attention(a, cfg->head_dim, cfg->dtype, grid, true, (cudaStream_t)stream));
 }
 
 hkv_status hkv_evict(const hkv_config *cfg, const hkv_cache *cache, int layer,

@@ -23,7 +23,10 @@
 //    and, fused, the new token's K/V with its last; an epilogue warp merges
 //    the consumer warps' states of each head segment and writes the output
 //    (a head wholly inside the piece) or a partial result (a split head)
-//    while the consumers stream on;
+//    while the consumers stream on. A CTA whose range starts inside a head
+//    that began in the previous CTA's range records that head and how many
+//    pieces it has; the head's first pieces go to slots of that CTA
+//    boundary, the rest to the slot of the CTA that computed them;
 //  * consumers take whole token rows with 16-byte lanes (a 256-byte bf16 row
 //    is 16 lanes), a shuffle-xor tree per row for q.k, online softmax in the
 //    log2 domain with fp32 accumulation;
@@ -33,10 +36,10 @@
 //    token (K/V row, position, query for the periodic update): nothing in
 //    the launch reads them;
 //
-// finishing kernel (one warp per head, after the attention kernel completes)
-//  * merges the partial results of each split head in index order, so the
-//    result does not depend on timing;
-//  * fused: advances each head's length and counters;
+// finishing kernel (one-warp CTAs, after the attention kernel completes)
+//  * a warp per CTA boundary merges the head split there from the pieces'
+//    slots in index order, so the result does not depend on timing;
+//  * fused: one lane per head advances the head's length and counters;
 //
 //  * programmatic dependent launch: every thread of either kernel waits for
 //    the previous kernel of the stream (griddepcontrol.wait) before it reads
@@ -233,6 +236,77 @@ struct TileIter {
   }
 };
 
+// The consumers' arithmetic on one 16-byte piece of a row.
+//  * bf16: the query stays in its packed pairs and q.k takes one
+//    mixed-precision FMA per element (a bf16 x bf16 product is exact in
+//    fp32, so this equals widening first); the scale goes on the sum;
+//  * fp32: the query is scaled when loaded;
+//  * V rows accumulate into fp32 pairs with paired FMAs.
+template <typename T>
+struct LaneMath;
+template <>
+struct LaneMath<__nv_bfloat16> {
+  static constexpr int kEPL = 8;
+  struct Q {
+    uint32_t w[4];
+  };
+  __device__ static __forceinline__ void load_q(Q &q, const uint4 &u, float) {
+    q.w[0] = u.x, q.w[1] = u.y, q.w[2] = u.z, q.w[3] = u.w;
+  }
+  __device__ static __forceinline__ void fma_pair(float &d0, float &d1, uint32_t a, uint32_t b) {
+    asm("{\n\t.reg .b16 al, ah, bl, bh;\n\t"
+        "mov.b32 {al, ah}, %2;\n\t"
+        "mov.b32 {bl, bh}, %3;\n\t"
+        "fma.rn.f32.bf16 %0, al, bl, %0;\n\t"
+        "fma.rn.f32.bf16 %1, ah, bh, %1;\n\t}"
+        : "+f"(d0), "+f"(d1)
+        : "r"(a), "r"(b));
+  }
+  __device__ static __forceinline__ float dot(const Q &q, const uint4 &k) {
+    float d0 = 0.f, d1 = 0.f;
+    fma_pair(d0, d1, q.w[0], k.x);
+    fma_pair(d0, d1, q.w[1], k.y);
+    fma_pair(d0, d1, q.w[2], k.z);
+    fma_pair(d0, d1, q.w[3], k.w);
+    return d0 + d1;
+  }
+  __device__ static __forceinline__ float score(float dot, float qscale) { return dot * qscale; }
+  __device__ static __forceinline__ float2 widen(uint32_t w) {
+    return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xFFFF0000u));
+  }
+  __device__ static __forceinline__ void add_v(float2 *acc, const uint4 &v, float pr) {
+    const float2 p2 = make_float2(pr, pr);
+    acc[0] = __ffma2_rn(widen(v.x), p2, acc[0]);
+    acc[1] = __ffma2_rn(widen(v.y), p2, acc[1]);
+    acc[2] = __ffma2_rn(widen(v.z), p2, acc[2]);
+    acc[3] = __ffma2_rn(widen(v.w), p2, acc[3]);
+  }
+};
+template <>
+struct LaneMath<float> {
+  static constexpr int kEPL = 4;
+  struct Q {
+    float f[4];
+  };
+  __device__ static __forceinline__ void load_q(Q &q, const uint4 &u, float qscale) {
+    q.f[0] = __uint_as_float(u.x) * qscale;
+    q.f[1] = __uint_as_float(u.y) * qscale;
+    q.f[2] = __uint_as_float(u.z) * qscale;
+    q.f[3] = __uint_as_float(u.w) * qscale;
+  }
+  __device__ static __forceinline__ float dot(const Q &q, const uint4 &k) {
+    const float d0 = fmaf(q.f[2], __uint_as_float(k.z), q.f[0] * __uint_as_float(k.x));
+    const float d1 = fmaf(q.f[3], __uint_as_float(k.w), q.f[1] * __uint_as_float(k.y));
+    return d0 + d1;
+  }
+  __device__ static __forceinline__ float score(float dot, float) { return dot; }
+  __device__ static __forceinline__ void add_v(float2 *acc, const uint4 &v, float pr) {
+    const float2 p2 = make_float2(pr, pr);
+    acc[0] = __ffma2_rn(make_float2(__uint_as_float(v.x), __uint_as_float(v.y)), p2, acc[0]);
+    acc[1] = __ffma2_rn(make_float2(__uint_as_float(v.z), __uint_as_float(v.w)), p2, acc[1]);
+  }
+};
+
 // what the producer must still add to a tile after its arena rows
 struct Pending {
   int h, slot_new;
@@ -257,6 +331,9 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
   __shared__ long long s_s0;
   __shared__ int s_h0, s_bad;
   __shared__ volatile int s_abort;
+#ifdef HKV_ATTN_TRACE
+  __shared__ unsigned long long t_issue[NS];
+#endif
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int nheads = p.nheads;
@@ -374,8 +451,13 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
   pit.g = st_active ? a : 0;
   pit.b = st_active ? b : 0;
   int issued = 0;
+  // the arena rows are read once per step: evict them from L2 first
+  const uint64_t stream_pol = producer ? l2_evict_first_policy() : 0;
   auto issue_old = [&](Pending &pd) {  // describe + expect + copy the arena rows
     const int stage = issued % NS;
+#ifdef HKV_ATTN_TRACE
+    t_issue[stage] = globaltimer();
+#endif
     const long long ge = pit.tile_end();
     const long long he = pit.hs + pit.hl;
     const int r0 = (int)(pit.g - pit.hs), r1 = (int)(ge - pit.hs);   // head-local rows
@@ -396,9 +478,10 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
       const uint32_t bytes = (uint32_t)n_old * RB;
       const long long row = look.off(pit.h) + r0;
       mbar_expect_tx(&full[stage], 2 * bytes);
-      bulk_g2s(dk, static_cast<const unsigned char *>(p.K) + row * RB, bytes, &full[stage]);
-      bulk_g2s(dk + TT * RB, static_cast<const unsigned char *>(p.V) + row * RB, bytes,
-               &full[stage]);
+      bulk_g2s_hint(dk, static_cast<const unsigned char *>(p.K) + row * RB, bytes, &full[stage],
+                    stream_pol);
+      bulk_g2s_hint(dk + TT * RB, static_cast<const unsigned char *>(p.V) + row * RB, bytes,
+                    &full[stage], stream_pol);
     }
     pit.advance(look);
     ++issued;
@@ -429,22 +512,43 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
   // the launch passed its checks (the workspace is free: the previous
   // finishing kernel is done)
   if (blockIdx.x == 0 && tid == 0) p.ctl->valid = 1;
+  // The head split at this CTA's boundary, if its first row lies in the
+  // previous CTA's range: the finishing kernel merges its pieces (CTAs
+  // k0 = blockIdx.x - 1 .. k0 + np - 1). Written by the epilogue warp, idle
+  // until the first segment ends (the producer is on the critical path now).
+  __shared__ int s_np;
+  if (blockIdx.x > 0 && tid == (kCW + 1) * 32) {
+    int4 r = make_int4(-1, 0, 0, 0);
+    const long long hs = tab.start[0];
+    if (st_active && hs < a && hs >= a - chunk) {
+      const long long k0 = blockIdx.x - 1;
+      const long long he = hs + tab.vlen[0];
+      r = make_int4(tab.h0, (int)((he - 1) / chunk - k0 + 1), 0, 0);
+    }
+    p.rec[blockIdx.x] = r;
+    // the inline slots of this boundary that no piece fills hold empty
+    // pieces (maximum -inf, sum 0): the finishing kernel loads all of them
+    s_np = r.x >= 0 ? r.y : 0;
+  }
 
   if (warp == 0) {
     // ---- producer ----------------------------------------------------------
     if (producer) {
+      unsigned long long t_wait = 0;
 #pragma unroll
       for (int j = 0; j < NS; ++j)
         if (j < n_pre) issue_extra(pre[j], j);
       while (!pit.done()) {
         const int stage = issued % NS;
         // the consumers are done with the tile that used this stage before
+        const unsigned long long tw = HKV_CLOCK();
         if (s_abort ||
             (issued >= NS && !mbar_wait(&empty[stage], (uint32_t)(issued / NS - 1) & 1u))) {
           s_abort = 1;
           set_err(p.err, HKV_ERR_TIMEOUT);
           break;
         }
+        t_wait += HKV_CLOCK() - tw;
         Pending pd;
         issue_old(pd);
         issue_extra(pd, stage);
@@ -459,38 +563,48 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
           mbar_arrive(&full[stage]);
         }
       }
+      HKV_TRACE_ADD(13, t_wait);
     }
   } else if (warp <= kCW) {
     // ---- consumers ---------------------------------------------------------
     const int ctid = tid - 32, cw = warp - 1;
     const int grp = lane / LPR, col = lane % LPR;
-    float q[EPL], acc[EPL];
+    using M = LaneMath<T>;
+    static_assert(M::kEPL == EPL, "lane mapping");
+    typename M::Q q;
+    float2 acc[EPL / 2];
     float m = -INFINITY, l = 0.f;
     int nseg = 0;
 #pragma unroll
-    for (int e = 0; e < EPL; ++e) acc[e] = 0.f;
+    for (int e = 0; e < EPL / 2; ++e) acc[e] = make_float2(0.f, 0.f);
 
+    unsigned long long t_full = 0, t_stall = 0, t_lat = 0;
+    long long c_comp = 0, c_last = 0;
+    int n_tiles = 0;
     for (int tile = 0;; ++tile) {
       const int stage = tile % NS;
+      const unsigned long long tw = HKV_CLOCK();
       if (!s_abort && !mbar_wait(&full[stage], (uint32_t)(tile / NS) & 1u)) {
         s_abort = 1;
         set_err(p.err, HKV_ERR_TIMEOUT);
       }
+      if (tile > 0) t_full += HKV_CLOCK() - tw;
+#ifdef HKV_ATTN_TRACE
+      const long long c_t0 = clock64();
+      if (!s_abort && !(meta[stage].flags & kDone)) t_lat += HKV_CLOCK() - t_issue[stage];
+#endif
       if (s_abort) break;
       const int flags = meta[stage].flags;
       if (flags & kDone) break;
       if (tile == 0 && ctid == 0) HKV_TRACE(3);
-      if (ctid == 0) HKV_TRACE_ADD(17, 1);
+      ++n_tiles;
       const int n = meta[stage].n;
       const unsigned char *Ks = stages + stage * S::kStageBytes;
       const unsigned char *Vs = Ks + TT * RB;
       if (flags & kFirst) {  // first tile of this head in this piece
-        Elem<T>::unpack(*reinterpret_cast<const uint4 *>(Vs + TT * RB + col * 16), q);
+        M::load_q(q, *reinterpret_cast<const uint4 *>(Vs + TT * RB + col * 16), p.qscale);
 #pragma unroll
-        for (int e = 0; e < EPL; ++e) {
-          q[e] *= p.qscale;
-          acc[e] = 0.f;
-        }
+        for (int e = 0; e < EPL / 2; ++e) acc[e] = make_float2(0.f, 0.f);
         m = -INFINITY;
         l = 0.f;
       }
@@ -500,15 +614,10 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
       for (int st = 0; st < S::kSteps; ++st) {
         const int r = st * (kCW * RPW) + cw * RPW + grp;
         float dot = 0.f;
-        if (r < n) {
-          float kf[EPL];
-          Elem<T>::unpack(*reinterpret_cast<const uint4 *>(Ks + r * RB + col * 16), kf);
-#pragma unroll
-          for (int e = 0; e < EPL; ++e) dot = fmaf(q[e], kf[e], dot);
-        }
+        if (r < n) dot = M::dot(q, *reinterpret_cast<const uint4 *>(Ks + r * RB + col * 16));
 #pragma unroll
         for (int o = LPR / 2; o >= 1; o >>= 1) dot += __shfl_xor_sync(0xFFFFFFFFu, dot, o);
-        sc[st] = r < n ? dot : -INFINITY;
+        sc[st] = r < n ? M::score(dot, p.qscale) : -INFINITY;
       }
       float mt = sc[0];
 #pragma unroll
@@ -518,21 +627,22 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
         const float corr = exp2f(m - mn);
         l *= corr;
 #pragma unroll
-        for (int e = 0; e < EPL; ++e) acc[e] *= corr;
+        for (int e = 0; e < EPL / 2; ++e) acc[e] = __fmul2_rn(acc[e], make_float2(corr, corr));
 #pragma unroll
         for (int st = 0; st < S::kSteps; ++st) {
           const int r = st * (kCW * RPW) + cw * RPW + grp;
           if (r < n) {
             const float pr = exp2f(sc[st] - mn);
             l += pr;
-            float vf[EPL];
-            Elem<T>::unpack(*reinterpret_cast<const uint4 *>(Vs + r * RB + col * 16), vf);
-#pragma unroll
-            for (int e = 0; e < EPL; ++e) acc[e] = fmaf(pr, vf[e], acc[e]);
+            M::add_v(acc, *reinterpret_cast<const uint4 *>(Vs + r * RB + col * 16), pr);
           }
         }
         m = mn;
       }
+#ifdef HKV_ATTN_TRACE
+      const long long c_t1 = clock64();
+      c_comp += c_t1 - c_t0;
+#endif
       if (flags & kLast) {  // last tile of this head in this piece: hand it over
         SegMeta sm;
         if (cw == 0 && lane == 0) {
@@ -551,9 +661,11 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
           const float s2 = m2 == -INFINITY ? 0.f : exp2f(m2 - mx);
           l = l * s1 + l2 * s2;
 #pragma unroll
-          for (int e = 0; e < EPL; ++e) {
-            const float a2 = __shfl_xor_sync(0xFFFFFFFFu, acc[e], o);
-            acc[e] = acc[e] * s1 + a2 * s2;
+          for (int e = 0; e < EPL / 2; ++e) {
+            const float ax = __shfl_xor_sync(0xFFFFFFFFu, acc[e].x, o);
+            const float ay = __shfl_xor_sync(0xFFFFFFFFu, acc[e].y, o);
+            acc[e].x = acc[e].x * s1 + ax * s2;
+            acc[e].y = acc[e].y * s1 + ay * s2;
           }
           m = mx;
         }
@@ -563,10 +675,13 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
           s_abort = 1;
           set_err(p.err, HKV_ERR_TIMEOUT);
         }
-        if (cw == 0 && lane == 0) HKV_TRACE_ADD(11, HKV_CLOCK() - tw);
+        t_stall += HKV_CLOCK() - tw;
         if (lane < LPR) {
 #pragma unroll
-          for (int e = 0; e < EPL; ++e) red_acc[cw][lane * EPL + e] = acc[e];
+          for (int e = 0; e < EPL / 2; ++e) {
+            red_acc[cw][lane * EPL + 2 * e] = acc[e].x;
+            red_acc[cw][lane * EPL + 2 * e + 1] = acc[e].y;
+          }
           if (lane == 0) {
             red_m[cw] = m;
             red_l[cw] = l;
@@ -576,12 +691,21 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
         __syncwarp();
         if (lane == 0) mbar_arrive(&epi_full);
         ++nseg;
+#ifdef HKV_ATTN_TRACE
+        c_last += clock64() - c_t1;
+#endif
       } else {
         __syncwarp();
         if (lane == 0) mbar_arrive(&empty[stage]);  // this warp is done with the stage
       }
     }
     if (ctid == 0) HKV_TRACE(4);
+    if (ctid == 0) HKV_TRACE_ADD(12, t_full);
+    if (ctid == 0) HKV_TRACE_ADD(11, t_stall);
+    if (ctid == 0) HKV_TRACE_ADD(17, n_tiles);
+    if (ctid == 0) HKV_TRACE_ADD(24, c_comp);
+    if (ctid == 0) HKV_TRACE_ADD(25, c_last);
+    if (ctid == 0) HKV_TRACE_ADD(26, t_lat);
     // tell the epilogue there is nothing more
     if (nseg > 0 && !s_abort && !mbar_wait(&epi_free, (uint32_t)(nseg - 1) & 1u)) {
       s_abort = 1;
@@ -602,15 +726,35 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
     constexpr int CPL = D / 32;
     using V = Vec<CPL>;
     constexpr int PS = attn_part_floats(D);  // floats per partial slot
-    for (int k = 0;; ++k) {
+    if (blockIdx.x > 0) {
+      __syncwarp();
+      const int np0 = s_np;  // written by lane 0 of this warp above
+      float z[CPL];
+#pragma unroll
+      for (int c = 0; c < CPL; ++c) z[c] = 0.f;
+      for (int j = np0; j < kAttnInlinePieces; ++j) {
+        float *pp = p.part + ((size_t)blockIdx.x * kAttnInlinePieces + j) * PS;
+        V::st(pp + CPL * lane, z);
+        if (lane == 0) {
+          pp[D] = -INFINITY;
+          pp[D + 1] = 0.f;
+        }
+      }
+    }
+    unsigned long long t_ew = 0, t_eb = 0, t_e1 = HKV_CLOCK();
+    int k_segs = 0;
+    for (int k = 0;; ++k, ++k_segs) {
+      const unsigned long long t_e0 = HKV_CLOCK();
+      if (k > 0) t_eb += t_e0 - t_e1;
       if (!s_abort && !mbar_wait(&epi_full, (uint32_t)k & 1u)) {
         s_abort = 1;
         set_err(p.err, HKV_ERR_TIMEOUT);
       }
+      t_e1 = HKV_CLOCK();
+      if (k > 0) t_ew += t_e1 - t_e0;
       if (s_abort) break;
       const int h = seg.h;
       if (h < 0) break;
-      if (lane == 0) HKV_TRACE_ADD(9, 1);
       const long long hs = seg.hs, he = seg.he;
       float mx = red_m[0];
 #pragma unroll
@@ -633,21 +777,16 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
 #pragma unroll
         for (int c = 0; c < CPL; ++c) A[c] /= L;
         V::st(p.out + (size_t)h * D + CPL * lane, A);
-        if (lane == 0) p.pieces[h] = make_int2(1, 0);
-      } else {
-        // Piece j of the np CTA ranges the head touches; the CTA with its
-        // first piece records np and where piece 0 sits.
+      } else {  // piece j of the head split at boundary k0 + 1
         const long long k0 = hs / chunk;
         const int j = (int)(blockIdx.x - k0);
-        const int s1 = a < hs ? 1 : 0;  // piece 0 starts inside this range
-        float *pp = j < p.nis ? p.part_inline + ((size_t)h * p.nis + j) * PS
-                              : p.part + ((size_t)blockIdx.x * 2 + s1) * PS;
+        float *pp = j < kAttnInlinePieces
+                        ? p.part + ((size_t)(k0 + 1) * kAttnInlinePieces + j) * PS
+                        : p.over + (size_t)blockIdx.x * PS;
         V::st(pp + CPL * lane, A);
         if (lane == 0) {
           pp[D] = mx;
           pp[D + 1] = L;
-          if (j == 0)
-            p.pieces[h] = make_int2((int)((he - 1) / chunk - k0 + 1), (int)(2 * k0 + s1));
         }
       }
       // Fused: the CTA whose range holds the head's last row appends the new
@@ -672,22 +811,27 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
       }
     }
     if (lane == 0) HKV_TRACE(5);
+    if (lane == 0) HKV_TRACE_ADD(14, t_eb);
+    if (lane == 0) HKV_TRACE_ADD(9, k_segs);
+    if (lane == 0) HKV_TRACE_ADD(15, t_ew);
   }
   if (tid == 0) HKV_TRACE(6);
 }
 
-// One warp per head: merge the partial results of a split head in index
-// order; fused, advance the head's counters. A head's first pieces sit in
-// inline slots of its own and the attention kernel records how many pieces
-// there are, so every load goes out at once: a head whose pieces are all
-// inline costs one round trip to memory.
+// One-warp CTAs. Warp w advances the counters of heads 32w .. 32w + 31, one
+// lane per head (fused; plain attention writes zeros for empty heads), and
+// merges the head split at CTA boundary k = w + 1, if any, from its pieces in
+// index order, so the result does not depend on timing. The record of that
+// head and the boundary's inline slots (its first pieces, or empty pieces
+// the attention kernel wrote there) load in the same round as the counters:
+// a head of at most kAttnInlinePieces pieces costs one round trip to memory.
 template <int D, typename T, bool FUSED>
 __global__ void __maxnreg__(kFinishRegs)
     finish_kernel(const AttnArgs p) {
   constexpr int CPL = D / 32;
   using V = Vec<CPL>;
   constexpr int PS = attn_part_floats(D);
-  constexpr int MB = attn_inline_slots(D);  // partial results loaded per batch
+  constexpr int NI = kAttnInlinePieces;  // pieces per batch (the first: inline)
   // Let the next kernel (the next layer's attention) start its prologue now;
   // it waits for this kernel before it reads anything written here.
   HKV_TRACE(20);
@@ -695,118 +839,126 @@ __global__ void __maxnreg__(kFinishRegs)
   pdl_wait();  // the attention kernel is complete
   HKV_TRACE(21);
   const int lane = threadIdx.x & 31;
-  const int nw = gridDim.x * (kFinishThreads / 32);
-  const int w0 = blockIdx.x * (kFinishThreads / 32) + (threadIdx.x >> 5);
-  const int nis = p.nis;
+  const int w = blockIdx.x * (kFinishThreads / 32) + (threadIdx.x >> 5);
+  const int G = p.grid;
   const int valid = p.ctl->valid;
-
-  for (int h = w0; h < p.nheads; h += nw) {
-    // One round of loads, none depending on another: where the head's pieces
-    // are, the maxima, sums and accumulators of its inline pieces and the
-    // head's counters. Inline slots past the piece count hold older data and
-    // are not used.
-    const int i = p.layer_base + h;
-    const float *rec = p.part_inline + (size_t)h * nis * PS;
-    const int2 pc = p.pieces[h];
-    float m0 = -INFINITY, l0 = 0.f;
-    if (lane < nis) {
-      m0 = __ldcg(rec + (size_t)lane * PS + D);
-      l0 = __ldcg(rec + (size_t)lane * PS + D + 1);
-    }
-    float v[MB][CPL];
-#pragma unroll
-    for (int u = 0; u < MB; ++u) {
-      if (u < nis) {
-        V::ldcg(rec + (size_t)u * PS + CPL * lane, v[u]);
-      } else {
-#pragma unroll
-        for (int c = 0; c < CPL; ++c) v[u][c] = 0.f;
-      }
-    }
-    const int len = p.len[h];
-    int nt = 0, nb = 0;
-    bool dense = true;
+  const int h = 32 * w + lane;
+  const bool hin = h < p.nheads;
+  const int i = p.layer_base + h;
+  int len = 0, nt = 0, nb = 0;
+  bool dense = true;
+  if (hin) {
+    len = p.len[h];
     if (FUSED) {
       nt = p.ntok[i];
       nb = p.nbuf[i];
       dense = p.label[i] == HKV_DENSE;
     }
-    if (!valid) return;  // the attention launch failed its checks
+  }
+  const int k = w + 1;  // the boundary between CTAs k - 1 and k
+  int4 rc = make_int4(-1, 0, 0, 0);
+  float iv[NI][CPL];
+  float im = -INFINITY, il = 0.f;  // piece `lane` (lanes < NI)
+#pragma unroll
+  for (int u = 0; u < NI; ++u)
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) iv[u][c] = 0.f;
+  const float *inl = p.part + (size_t)k * NI * PS;
+  if (k < G) {
+    rc = __ldcg(p.rec + k);
+#pragma unroll
+    for (int u = 0; u < NI; ++u) V::ldcg(inl + (size_t)u * PS + CPL * lane, iv[u]);
+    if (lane < NI) {
+      im = __ldcg(inl + (size_t)lane * PS + D);
+      il = __ldcg(inl + (size_t)lane * PS + D + 1);
+    }
+  }
 #ifdef HKV_ATTN_TRACE
-    if (g_trace && h == w0 && lane == 0 && (len + nt + nb + pc.x + (int)(m0 + l0 + v[0][0])) != 0x7fffffff)
-      HKV_TRACE_AT(23) = globaltimer();  // the first head's loads are back
+  if (g_trace && lane == 0) HKV_TRACE_AT(24) = rc.x >= 0 ? rc.y : 0;
+  if (g_trace && lane == 0 &&
+      (len + nt + nb + rc.x + valid + (int)(im + il + iv[NI - 1][0] + iv[0][0])) != 0x7fffffff)
+    HKV_TRACE_AT(23) = globaltimer();  // the loads are back
 #endif
-    if (!FUSED && len == 0) {  // an empty head (plain attention) yields zeros; it
-      float z[CPL];            // has no tiles, so its pieces are not recorded
-#pragma unroll
-      for (int c = 0; c < CPL; ++c) z[c] = 0.f;
-      V::st(p.out + (size_t)h * D + CPL * lane, z);
-      continue;
-    }
-    const int np = pc.x;
-    if (np > 1) {
-      // Merge in piece (index) order: the maximum first, then the weighted
-      // sums. Pieces past the inline ones load MB at a time.
-      auto piece = [&](int j) {
-        return j < nis ? rec + (size_t)j * PS
-                       : p.part + (size_t)(j == 0 ? pc.y : pc.y - (pc.y & 1) + 2 * j) * PS;
-      };
-      const bool all_inline = np <= nis;
-      float gm = lane < np && lane < nis ? m0 : -INFINITY;
-      for (int j = (all_inline ? 32 : (lane < nis ? lane + 32 : lane)); j < np; j += 32)
-        gm = fmaxf(gm, __ldcg(piece(j) + D));
-#pragma unroll
-      for (int o = 16; o >= 1; o >>= 1) gm = fmaxf(gm, __shfl_xor_sync(0xFFFFFFFFu, gm, o));
-      float GL = 0.f, GA[CPL];
-#pragma unroll
-      for (int c = 0; c < CPL; ++c) GA[c] = 0.f;
-      for (int j0 = 0; j0 < np; j0 += 32) {
-        float mj = -INFINITY, lj = 0.f;
-        const int j = j0 + lane;
-        if (j < np) {
-          if (j < nis) {
-            mj = m0;
-            lj = l0;
-          } else {
-            mj = __ldcg(piece(j) + D);
-            lj = __ldcg(piece(j) + D + 1);
-          }
-        }
-        // weight of piece j0 + lane (zero past the last piece)
-        const float wj = mj == -INFINITY ? 0.f : exp2f(mj - gm);
-        const float lw = lj * wj;
-        const int cnt = np - j0 < 32 ? np - j0 : 32;
-        for (int t0 = 0; t0 < cnt; t0 += MB) {
-          if (j0 + t0 >= nis) {
-#pragma unroll
-            for (int u = 0; u < MB; ++u) {
-              if (j0 + t0 + u < np) {
-                V::ldcg(piece(j0 + t0 + u) + CPL * lane, v[u]);
-              } else {
-#pragma unroll
-                for (int c = 0; c < CPL; ++c) v[u][c] = 0.f;
-              }
-            }
-          }
-#pragma unroll
-          for (int u = 0; u < MB; ++u) {
-            const float w = __shfl_sync(0xFFFFFFFFu, wj, t0 + u);
-            GL += __shfl_sync(0xFFFFFFFFu, lw, t0 + u);
-            if (j0 + t0 + u < np)  // an unused inline slot may hold anything
-#pragma unroll
-              for (int c = 0; c < CPL; ++c) GA[c] = fmaf(v[u][c], w, GA[c]);
-          }
-        }
-      }
-#pragma unroll
-      for (int c = 0; c < CPL; ++c) GA[c] /= GL;
-      V::st(p.out + (size_t)h * D + CPL * lane, GA);
-    }
-    if (FUSED && lane == 0) {  // the new token joined the head in the attention kernel
+  if (valid) {  // else the attention launch failed its checks
+    if (FUSED && hin) {  // the new token joined the head in the attention kernel
       p.len[h] = len + 1;
       p.ntok[i] = nt + 1;
       if (!dense) p.nbuf[i] = nb + 1;
     }
+    if (!FUSED && hin && len == 0) {  // an empty head has no tiles: zeros
+      float4 *o = reinterpret_cast<float4 *>(p.out + (size_t)h * D);
+#pragma unroll 4
+      for (int c = 0; c < D / 4; ++c) o[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+  }
+  if (valid && rc.x >= 0) {
+    const int hh = rc.x, np = rc.y;
+    // piece j >= NI: the overflow slot of the CTA that computed it
+    auto over = [&](int j) { return p.over + (size_t)(k - 1 + j) * PS; };
+    float m0 = im, l0 = il;  // piece `lane`
+    if (lane >= NI) {
+      m0 = -INFINITY;
+      l0 = 0.f;
+      if (lane < np) {
+        m0 = __ldcg(over(lane) + D);
+        l0 = __ldcg(over(lane) + D + 1);
+      }
+    }
+    // Merge in piece (index) order: the maximum first, then the weighted sums
+    // (inline slots past the last piece hold empty pieces: weight 0).
+    float gm = m0;
+    for (int j = lane + 32; j < np; j += 32) gm = fmaxf(gm, __ldcg(over(j) + D));
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) gm = fmaxf(gm, __shfl_xor_sync(0xFFFFFFFFu, gm, o));
+    float GL = 0.f, GA[CPL];
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) GA[c] = 0.f;
+    for (int j0 = 0; j0 < np; j0 += 32) {
+      float mj = m0, lj = l0;
+      if (j0 > 0) {
+        const int j = j0 + lane;
+        mj = -INFINITY;
+        lj = 0.f;
+        if (j < np) {
+          mj = __ldcg(over(j) + D);
+          lj = __ldcg(over(j) + D + 1);
+        }
+      }
+      // weight of piece j0 + lane (zero past the last piece)
+      const float wj = mj == -INFINITY ? 0.f : exp2f(mj - gm);
+      const float lw = lj * wj;
+      const int cnt = np - j0 < 32 ? np - j0 : 32;
+      for (int t0 = 0; t0 < cnt; t0 += NI) {
+        float v[NI][CPL];
+        if (j0 == 0 && t0 == 0) {
+#pragma unroll
+          for (int u = 0; u < NI; ++u)
+#pragma unroll
+            for (int c = 0; c < CPL; ++c) v[u][c] = iv[u][c];
+        } else {
+#pragma unroll
+          for (int u = 0; u < NI; ++u) {
+            if (j0 + t0 + u < np) {
+              V::ldcg(over(j0 + t0 + u) + CPL * lane, v[u]);
+            } else {
+#pragma unroll
+              for (int c = 0; c < CPL; ++c) v[u][c] = 0.f;
+            }
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < NI; ++u) {
+          const float wu = __shfl_sync(0xFFFFFFFFu, wj, t0 + u);
+          GL += __shfl_sync(0xFFFFFFFFu, lw, t0 + u);
+          if (j0 + t0 + u < np)
+#pragma unroll
+            for (int c = 0; c < CPL; ++c) GA[c] = fmaf(v[u][c], wu, GA[c]);
+        }
+      }
+    }
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) GA[c] /= GL;
+    V::st(p.out + (size_t)hh * D + CPL * lane, GA);
   }
   HKV_TRACE(22);
 }
@@ -855,13 +1007,19 @@ cudaError_t launch_pdl(K kernel, int grid, int threads, size_t smem, const AttnA
 }
 
 template <int D, typename T>
-cudaError_t launch_t(const AttnArgs &a, int grid, int finish_grid, bool fused, cudaStream_t s) {
+cudaError_t launch_t(AttnArgs a, int grid, bool fused, cudaStream_t s) {
+  a.grid = grid;
   cudaError_t e =
       fused ? launch_pdl(attn_kernel<D, T, true>, grid, kAttnThreads, smem_bytes<D, T>(), a, s)
             : launch_pdl(attn_kernel<D, T, false>, grid, kAttnThreads, smem_bytes<D, T>(), a, s);
   if (e != cudaSuccess) return e;
-  return fused ? launch_pdl(finish_kernel<D, T, true>, finish_grid, kFinishThreads, 0, a, s)
-               : launch_pdl(finish_kernel<D, T, false>, finish_grid, kFinishThreads, 0, a, s);
+  // a warp for every 32 heads and for every CTA boundary
+  int warps = (a.nheads + 31) / 32;
+  if (warps < grid - 1) warps = grid - 1;
+  if (warps < 1) warps = 1;
+  const int fgrid = (warps + kFinishThreads / 32 - 1) / (kFinishThreads / 32);
+  return fused ? launch_pdl(finish_kernel<D, T, true>, fgrid, kFinishThreads, 0, a, s)
+               : launch_pdl(finish_kernel<D, T, false>, fgrid, kFinishThreads, 0, a, s);
 }
 
 }  // namespace
@@ -883,13 +1041,13 @@ cudaError_t attention_prepare(int D, int dtype, int *ctas) {
   return D == 64 ? prepare_both<64, float>(ctas) : prepare_both<128, float>(ctas);
 }
 
-cudaError_t launch_attention(const AttnArgs &a, int D, int dtype, int grid, int finish_grid,
-                             bool fused, cudaStream_t s) {
+cudaError_t launch_attention(const AttnArgs &a, int D, int dtype, int grid, bool fused,
+                             cudaStream_t s) {
+  if (grid < 1 || grid > kAttnMaxGrid) return cudaErrorInvalidValue;
   if (dtype == HKV_BF16)
-    return D == 64 ? launch_t<64, __nv_bfloat16>(a, grid, finish_grid, fused, s)
-                   : launch_t<128, __nv_bfloat16>(a, grid, finish_grid, fused, s);
-  return D == 64 ? launch_t<64, float>(a, grid, finish_grid, fused, s)
-                 : launch_t<128, float>(a, grid, finish_grid, fused, s);
+    return D == 64 ? launch_t<64, __nv_bfloat16>(a, grid, fused, s)
+                   : launch_t<128, __nv_bfloat16>(a, grid, fused, s);
+  return D == 64 ? launch_t<64, float>(a, grid, fused, s) : launch_t<128, float>(a, grid, fused, s);
 }
 
 }  // namespace hkv

@@ -133,6 +133,24 @@ __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t by
       : "memory");
 }
 
+// An L2 policy that evicts the lines it is applied to first, and the bulk
+// copy above under such a policy: for data streamed once (the K/V arena in
+// decode attention), so that it does not push small, soon re-read data (the
+// kernels' records, partial results and counters) out of L2.
+__device__ __forceinline__ uint64_t l2_evict_first_policy() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+__device__ __forceinline__ void bulk_g2s_hint(void *dst, const void *src, uint32_t bytes,
+                                              uint64_t *bar, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1], %2, [%3], %4;" ::"r"(smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
+      : "memory");
+}
+
 // 16-byte asynchronous global -> shared copy (both ends 16-byte aligned) and
 // the wait for all of the thread's outstanding ones
 __device__ __forceinline__ void cp_async16(void *dst, const void *src) {

@@ -27,14 +27,18 @@ struct AttnArgs {
   const void *q;              // [nheads][D]
   const void *k_new, *v_new;  // [nheads][D] new token (fused)
   float *out;                 // [nheads][D]
-  // Partial results (attn_part_floats(D) floats each) of a head split over
-  // the ranges of CTAs k0 .. k0 + np - 1: piece j < nis in the head's inline
-  // slot part_inline[h][j], else in the CTA slots part[2 * (k0 + j) + s]
-  // (s = 1 only for a piece 0 that starts inside its CTA's range).
-  float *part;                // [grid][2][...]
-  float *part_inline;         // [nheads][nis][...]
-  int nis;                    // inline slots per head (0: none)
-  int2 *pieces;               // [nheads] {np (1: not split), 2 * k0 + s of piece 0}
+  // Partial results (attn_part_floats(D) floats each) of heads split over
+  // several CTA ranges. The head split at CTA boundary k (its first row in
+  // CTA k - 1's range, pieces in CTAs k - 1 .. k + np - 2) keeps pieces
+  // j < kAttnInlinePieces in part[k][j] and the others in over[k - 1 + j],
+  // the slot of the CTA that computed them.
+  float *part;                // [grid][kAttnInlinePieces][...]
+  float *over;                // [grid][...]
+  // For each CTA k >= 1 whose range starts inside a head whose first row
+  // lies in CTA k - 1's range: {head, np, 0, 0}; else {-1, 0, 0, 0}.
+  // Written by every launch before the finishing kernel reads it.
+  int4 *rec;                  // [grid]
+  int grid;                   // attention CTAs (set by launch_attention)
   AttnCtl *ctl;
   uint32_t *err;
   // fused append: full [L*S*H] arrays and the layer's first flat head
@@ -58,23 +62,23 @@ struct AttnArgs {
 constexpr int kAttnConsumerWarps = HKV_ATTN_CONSUMER_WARPS;
 constexpr int kAttnThreads = 32 * (kAttnConsumerWarps + 2);  // + producer + epilogue
 constexpr int kAttnMaxGrid = 4096;
-constexpr int kFinishThreads = 32;  // finishing kernel: one warp per head and CTA
-// registers of a finishing thread, and how many finishing CTAs an SM takes
-// beside two attention CTAs (which leave ~14.8K of its 64K registers)
+// finishing kernel: one-warp CTAs, each for 32 heads' counters and one CTA
+// boundary's split head; at 64 registers a thread, seven fit on an SM beside
+// two attention CTAs (which leave ~14.8K of its 64K registers)
+constexpr int kFinishThreads = 32;
 constexpr int kFinishRegs = 64;
-constexpr int kFinishCtasPerSm = 6;
 // floats of one split-K partial result: D accumulators, the running maximum
 // and the sum, padded to 16 bytes for vector access
 __host__ __device__ constexpr int attn_part_floats(int D) { return D + 4; }
+// pieces of a split head kept per CTA boundary (loaded with its record)
+constexpr int kAttnInlinePieces = 4;
 
 size_t attention_smem_bytes(int D, int dtype);
-// inline partial slots per head that the finishing kernel reads in one batch
-__host__ __device__ constexpr int attn_inline_slots(int D) { return 16 / (D / 32); }
 cudaError_t attention_prepare(int D, int dtype, int *ctas_per_sm);
-// launches the attention kernel on `grid` CTAs and the finishing kernel on
-// `finish_grid` CTAs
-cudaError_t launch_attention(const AttnArgs &a, int D, int dtype, int grid, int finish_grid,
-                             bool fused, cudaStream_t s);
+// launches the attention kernel on `grid` CTAs (at most kAttnMaxGrid) and the
+// finishing kernel behind it
+cudaError_t launch_attention(const AttnArgs &a, int D, int dtype, int grid, bool fused,
+                             cudaStream_t s);
 
 // per-head cache maintenance (append / update / repack / prefill / identify)
 struct CacheArgs {

@@ -6,7 +6,7 @@
 // framework that owns and budgets all device memory, or code on a path where
 // an allocation is not allowed (for instance because it would synchronise the
 // device in a latency-critical loop). For them the split-K partial results
-// and the per-head arrival counters live in one file-scope device array of
+// and the records of split heads live in one file-scope device array of
 // fixed size, which every GPU that loads this library holds until the process
 // exits.
 #include <cuda_runtime.h>
@@ -22,15 +22,13 @@ namespace {
 
 using namespace hkv;
 
-// Split-K partials (two per CTA, up to 1 MiB), then where the pieces of each
-// head of a layer are (up to 65536 heads), then the control block the
-// attention kernel leaves for the finishing kernel: 1.5 MiB in total. The
-// kernels write all of it before reading it, so nothing in it has to start
-// at zero.
+// Split-K partials (per CTA boundary and per CTA, up to 1 MiB), then which
+// head is split at each CTA boundary, then the control block the attention
+// kernel leaves for the finishing kernel: 1.06 MiB in total. The kernels write all of it
+// before reading it, so nothing in it has to start at zero.
 constexpr size_t kPartBytes = 1u << 20;
-constexpr int kMaxHeadsPerLayer = 65536;
-constexpr size_t kPiecesBytes = (size_t)kMaxHeadsPerLayer * sizeof(int2);
-constexpr size_t kScratchBytes = kPartBytes + kPiecesBytes + 256;
+constexpr size_t kRecBytes = (size_t)kAttnMaxGrid * sizeof(int4);
+constexpr size_t kScratchBytes = kPartBytes + kRecBytes + 256;
 
 static __device__ __align__(256) unsigned char g_scratch[kScratchBytes];
 
@@ -88,21 +86,19 @@ extern "C" hkv_status hkv_decode_attention_noalloc(const hkv_config *cfg, const 
     return HKV_ERR_ALIGN;
   if (layer < 0 || layer >= cfg->n_layers) return HKV_ERR_INVALID_ARG;
   const int hpl = cfg->n_seqs * cfg->n_heads;
-  if (hpl > kMaxHeadsPerLayer) return HKV_ERR_CAPACITY;  // piece records would not fit
 
   NoAllocDevice *st = nullptr;
   const hkv_status ss = setup(cfg->head_dim, cfg->dtype, &st);
   if (ss != HKV_OK) return ss;
   const int ctas = st->ctas[cfg->dtype == HKV_BF16 ? 1 : 0][cfg->head_dim == 128 ? 1 : 0];
 
-  // as many CTAs as the partial area holds, at most the usual grid
-  const size_t per_cta = 2 * (size_t)attn_part_floats(cfg->head_dim) * sizeof(float);
+  // as many CTAs as the partial area holds (kAttnInlinePieces slots per
+  // boundary and one overflow slot per CTA), at most the usual grid
+  const size_t per_cta =
+      (kAttnInlinePieces + 1) * (size_t)attn_part_floats(cfg->head_dim) * sizeof(float);
   int grid = st->sms * ctas;
   if (grid > kAttnMaxGrid) grid = kAttnMaxGrid;
   if ((size_t)grid * per_cta > kPartBytes) grid = (int)(kPartBytes / per_cta);
-  const int per = kFinishThreads / 32;
-  int fgrid = (hpl + per - 1) / per;
-  if (fgrid > kFinishCtasPerSm * st->sms) fgrid = kFinishCtasPerSm * st->sms;
 
   cudaStream_t s = (cudaStream_t)stream;
 
@@ -114,14 +110,14 @@ extern "C" hkv_status hkv_decode_attention_noalloc(const hkv_config *cfg, const 
   a.q = q;
   a.out = out;
   a.part = reinterpret_cast<float *>(st->scratch);
-  a.nis = 0;  // no inline slots: every piece in the CTA slots
-  a.pieces = reinterpret_cast<int2 *>(st->scratch + kPartBytes);
-  a.ctl = reinterpret_cast<AttnCtl *>(st->scratch + kPartBytes + kPiecesBytes);
+  a.over = a.part + (size_t)grid * kAttnInlinePieces * attn_part_floats(cfg->head_dim);
+  a.rec = reinterpret_cast<int4 *>(st->scratch + kPartBytes);
+  a.ctl = reinterpret_cast<AttnCtl *>(st->scratch + kPartBytes + kRecBytes);
   a.err = cache->err;
   a.arena_tokens = cache->capacity_tokens;
   a.nheads = hpl;
   a.qscale = (float)(1.4426950408889634 / sqrt((double)cfg->head_dim));
-  return launch_attention(a, cfg->head_dim, cfg->dtype, grid, fgrid, false, s) == cudaSuccess
+  return launch_attention(a, cfg->head_dim, cfg->dtype, grid, false, s) == cudaSuccess
              ? HKV_OK
              : HKV_ERR_CUDA;
 }

@@ -66,12 +66,22 @@ def test_matches_workspace_version_two_calls_in_a_row(dtype, tol):
         assert not torch.isnan(out).any()
 
 
-def test_rejects_more_heads_than_its_array_holds():
+def test_seventy_thousand_heads_match_workspace_version():
+    # the scratch array has no per-head part: any number of heads fits
+    import torch
     from paper_2605_20600_gb300 import hkv as H
-    cfg = H.make_config(n_layers=1, n_seqs=1024, n_heads=65, head_dim=64, dtype="bf16",
-                        n_cond=1, n_image=64, row_len=8, recent_w=8, local_w=8, period=8,
-                        group_at=8, global_budget=16)
-    buf = ctypes.create_string_buffer(1024)
-    a = (ctypes.addressof(buf) + 255) & ~255
-    c = H.hkv_cache(a, a, a, a, a, a, a, a, a, a, a, 100)
-    assert _noalloc(H)(ctypes.byref(cfg), ctypes.byref(c), 0, a, a, None) == H.HKV_ERR_CAPACITY
+    rng = np.random.default_rng(13)
+    lens = rng.integers(0, 4, size=70000)
+    cfg, cb, q = _ragged_cache(H, lens, 64, "bf16", seed=13)
+    st = torch.cuda.current_stream().cuda_stream
+    ws = torch.zeros(H.hkv_workspace_size(cfg), dtype=torch.uint8, device="cuda")
+    ref = torch.zeros(len(lens), 64, dtype=torch.float32, device="cuda")
+    H.hkv_decode_attention(cfg, cb.c, 1, q, ref, ws, ws.numel(), st)
+    out = torch.full_like(ref, float("nan"))
+    assert _noalloc(H)(ctypes.byref(cfg), ctypes.byref(cb.c), 1, q.data_ptr(), out.data_ptr(),
+                       st) == 0
+    torch.cuda.synchronize()
+    H.hkv_check(cb.c)
+    assert (out - ref).abs().max().item() <= 2e-3
+    assert not torch.isnan(out).any()
+    assert (out[torch.from_numpy(lens == 0).cuda()] == 0).all()
