@@ -366,25 +366,31 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
   if (!p.prefetch) pdl_wait();
 
   // ---- prologue: every thread takes a contiguous slice of the layer's heads
-  // (all of its loads in flight at once); a block scan gives each slice its
-  // first slot.
+  // (every load of a head issued before any check uses one, so a group of
+  // heads costs one round trip); a block scan gives each slice its first
+  // slot.
   const int per = (nheads + kAttnThreads - 1) / kAttnThreads;
   const int h_lo = tid * per < nheads ? tid * per : nheads;
   const int h_hi = h_lo + per < nheads ? h_lo + per : nheads;
   long long mine = 0;
   int bad = 0;
+  auto check = [&](int l, long long o, int cp, int lab, int nb) {
+    if (l < 0 || o < 0 || o + l > p.arena_tokens) bad = HKV_ERR_BOUNDS;
+    if (FUSED) {
+      if (o + cp > p.arena_tokens) bad = HKV_ERR_BOUNDS;
+      else if (l + 1 > cp) bad = bad ? bad : HKV_ERR_CAPACITY;
+      else if (lab != HKV_DENSE && nb >= p.period)
+        bad = bad ? bad : HKV_ERR_STATE;  // the periodic update is due first
+    }
+  };
 #pragma unroll 4
   for (int h = h_lo; h < h_hi; ++h) {
     const int l = p.len[h];
     const long long o = p.off[h];
-    if (l < 0 || o < 0 || o + l > p.arena_tokens) bad = HKV_ERR_BOUNDS;
-    if (FUSED) {
-      const int cp = p.cap[h];
-      if (o + cp > p.arena_tokens) bad = HKV_ERR_BOUNDS;
-      else if (l + 1 > cp) bad = bad ? bad : HKV_ERR_CAPACITY;
-      else if (p.label[p.layer_base + h] != HKV_DENSE && p.nbuf[p.layer_base + h] >= p.period)
-        bad = bad ? bad : HKV_ERR_STATE;  // the periodic update is due first
-    }
+    if (FUSED)
+      check(l, o, p.cap[h], p.label[p.layer_base + h], p.nbuf[p.layer_base + h]);
+    else
+      check(l, o, 0, 0, 0);
     mine += slot_len<TT>(l + (FUSED ? 1 : 0));
   }
   long long total;
@@ -406,7 +412,8 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
   const long long a = (long long)blockIdx.x * chunk;
   const long long b = a + chunk < total ? a + chunk : total;
   const bool st_active = a < total;
-  if (st_active && mine > 0 && slice_start <= a && a < slice_start + mine) {
+  const bool holds_a = st_active && mine > 0 && slice_start <= a && a < slice_start + mine;
+  if (holds_a) {
     long long st = slice_start;
     for (int h = h_lo; h < h_hi; ++h) {
       const long long L = slot_len<TT>(p.len[h] + (FUSED ? 1 : 0));
@@ -423,12 +430,12 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
     const int h0 = st_active ? s_h0 : 0;
     const int h = h0 + lane;
     const bool in = st_active && h < nheads;
-    const int vl = in ? p.len[h] + (FUSED ? 1 : 0) : 0;
-    const long long L = slot_len<TT>(vl);
+    const int v = in ? p.len[h] + (FUSED ? 1 : 0) : 0;
+    const long long L = slot_len<TT>(v);
     const long long incl = warp_incl_scan(L);
     tab.start[lane] = s_s0 + incl - L;
     tab.off[lane] = in ? p.off[h] : 0;
-    tab.vlen[lane] = vl;
+    tab.vlen[lane] = v;
     if (lane == 0) {
       tab.h0 = h0;
       tab.n = st_active ? (nheads - h0 < kTable ? nheads - h0 : kTable) : 0;
