@@ -322,8 +322,13 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
   extern __shared__ __align__(128) unsigned char stages[];
   __shared__ uint64_t full[NS], empty[NS];
   __shared__ uint64_t epi_full, epi_free;   // hand-over of one segment's states
-  __shared__ __align__(16) float red_acc[kCW][D];
-  __shared__ float red_m[kCW], red_l[kCW];
+  // one segment's states: every row group of every consumer warp hands over
+  // its own (the epilogue merges them), so no consumer spends a shuffle tree
+  // on it
+  constexpr int NST = kCW * RPW;
+  static_assert(NST <= 32, "a lane of the epilogue per state");
+  __shared__ __align__(16) float red_acc[NST][D];
+  __shared__ float red_m[NST], red_l[NST];
   __shared__ TileMeta meta[NS];
   __shared__ SegMeta seg;
   __shared__ HeadTable tab;
@@ -659,23 +664,6 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&empty[stage]);  // this warp is done with the stage
-#pragma unroll
-        for (int o = LPR; o < 32; o <<= 1) {  // merge the row groups of the warp
-          const float m2 = __shfl_xor_sync(0xFFFFFFFFu, m, o);
-          const float l2 = __shfl_xor_sync(0xFFFFFFFFu, l, o);
-          const float mx = fmaxf(m, m2);
-          const float s1 = m == -INFINITY ? 0.f : exp2f(m - mx);
-          const float s2 = m2 == -INFINITY ? 0.f : exp2f(m2 - mx);
-          l = l * s1 + l2 * s2;
-#pragma unroll
-          for (int e = 0; e < EPL / 2; ++e) {
-            const float ax = __shfl_xor_sync(0xFFFFFFFFu, acc[e].x, o);
-            const float ay = __shfl_xor_sync(0xFFFFFFFFu, acc[e].y, o);
-            acc[e].x = acc[e].x * s1 + ax * s2;
-            acc[e].y = acc[e].y * s1 + ay * s2;
-          }
-          m = mx;
-        }
         // the epilogue is done with the previous segment's states
         const unsigned long long tw = HKV_CLOCK();
         if (nseg > 0 && !s_abort && !mbar_wait(&epi_free, (uint32_t)(nseg - 1) & 1u)) {
@@ -683,15 +671,14 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
           set_err(p.err, HKV_ERR_TIMEOUT);
         }
         t_stall += HKV_CLOCK() - tw;
-        if (lane < LPR) {
+        {  // this row group's state
+          const int si = cw * RPW + grp;
+          float2 *dst = reinterpret_cast<float2 *>(&red_acc[si][col * EPL]);
 #pragma unroll
-          for (int e = 0; e < EPL / 2; ++e) {
-            red_acc[cw][lane * EPL + 2 * e] = acc[e].x;
-            red_acc[cw][lane * EPL + 2 * e + 1] = acc[e].y;
-          }
-          if (lane == 0) {
-            red_m[cw] = m;
-            red_l[cw] = l;
+          for (int e = 0; e < EPL / 2; ++e) dst[e] = acc[e];
+          if (col == 0) {
+            red_m[si] = m;
+            red_l[si] = l;
           }
         }
         if (cw == 0 && lane == 0) seg = sm;
@@ -763,18 +750,23 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
       const int h = seg.h;
       if (h < 0) break;
       const long long hs = seg.hs, he = seg.he;
-      float mx = red_m[0];
+      // merge the row-group states: lane s < NST weighs state s
+      const float ms = lane < NST ? red_m[lane] : -INFINITY;
+      float mx = ms;
 #pragma unroll
-      for (int w = 1; w < kCW; ++w) mx = fmaxf(mx, red_m[w]);
-      float L = 0.f, A[CPL];
+      for (int o = 16; o >= 1; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, o));
+      const float ws = ms == -INFINITY ? 0.f : exp2f(ms - mx);
+      float L = lane < NST ? red_l[lane] * ws : 0.f;
+#pragma unroll
+      for (int o = 16; o >= 1; o >>= 1) L += __shfl_xor_sync(0xFFFFFFFFu, L, o);
+      float A[CPL];
 #pragma unroll
       for (int c = 0; c < CPL; ++c) A[c] = 0.f;
 #pragma unroll
-      for (int w = 0; w < kCW; ++w) {
-        const float sw = red_m[w] == -INFINITY ? 0.f : exp2f(red_m[w] - mx);
-        L += red_l[w] * sw;
+      for (int si = 0; si < NST; ++si) {
+        const float sw = __shfl_sync(0xFFFFFFFFu, ws, si);
         float r[CPL];
-        V::lds(&red_acc[w][CPL * lane], r);
+        V::lds(&red_acc[si][CPL * lane], r);
 #pragma unroll
         for (int c = 0; c < CPL; ++c) A[c] = fmaf(r[c], sw, A[c]);
       }
