@@ -88,10 +88,10 @@ __device__ unsigned long long *g_trace = nullptr;  // [layer][kAttnMaxGrid][32],
   do {                                               \
     if (g_trace) HKV_TRACE_AT(slot) = globaltimer(); \
   } while (0)
-#define HKV_TRACE_ADD(slot, v)              \
-  do {                                      \
-    if (g_trace) HKV_TRACE_AT(slot) += (v); \
-  } while (0)
+#define HKV_TRACE_ADD(slot, v)             \
+  do {                                     \
+    if (g_trace) HKV_TRACE_AT(slot) = (v); \
+  } while (0)  // one writer per slot and launch: a plain store
 #define HKV_CLOCK() globaltimer()
 #else
 #define HKV_TRACE(slot) \
@@ -873,7 +873,7 @@ __global__ void __maxnreg__(kFinishRegs)
     }
   }
 #ifdef HKV_ATTN_TRACE
-  if (g_trace && lane == 0) HKV_TRACE_AT(24) = rc.x >= 0 ? rc.y : 0;
+  if (g_trace && lane == 0) HKV_TRACE_AT(27) = rc.x >= 0 ? rc.y : 0;
   if (g_trace && lane == 0 &&
       (len + nt + nb + rc.x + valid + (int)(im + il + iv[NI - 1][0] + iv[0][0])) != 0x7fffffff)
     HKV_TRACE_AT(23) = globaltimer();  // the loads are back
