@@ -857,25 +857,28 @@ __global__ void __maxnreg__(kFinishRegs)
   const int k = w + 1;  // the boundary between CTAs k - 1 and k
   int4 rc = make_int4(-1, 0, 0, 0);
   float iv[NI][CPL];
-  float im = -INFINITY, il = 0.f;  // piece `lane` (lanes < NI)
+  float im[NI], il[NI];  // maxima and sums of the inline pieces (every lane)
 #pragma unroll
-  for (int u = 0; u < NI; ++u)
+  for (int u = 0; u < NI; ++u) {
+    im[u] = -INFINITY;
+    il[u] = 0.f;
 #pragma unroll
     for (int c = 0; c < CPL; ++c) iv[u][c] = 0.f;
+  }
   const float *inl = p.part + (size_t)k * NI * PS;
   if (k < G) {
     rc = __ldcg(p.rec + k);
 #pragma unroll
-    for (int u = 0; u < NI; ++u) V::ldcg(inl + (size_t)u * PS + CPL * lane, iv[u]);
-    if (lane < NI) {
-      im = __ldcg(inl + (size_t)lane * PS + D);
-      il = __ldcg(inl + (size_t)lane * PS + D + 1);
+    for (int u = 0; u < NI; ++u) {
+      V::ldcg(inl + (size_t)u * PS + CPL * lane, iv[u]);
+      im[u] = __ldcg(inl + (size_t)u * PS + D);
+      il[u] = __ldcg(inl + (size_t)u * PS + D + 1);
     }
   }
 #ifdef HKV_ATTN_TRACE
   if (g_trace && lane == 0) HKV_TRACE_AT(27) = rc.x >= 0 ? rc.y : 0;
   if (g_trace && lane == 0 &&
-      (len + nt + nb + rc.x + valid + (int)(im + il + iv[NI - 1][0] + iv[0][0])) != 0x7fffffff)
+      (len + nt + nb + rc.x + valid + (int)(im[0] + il[NI - 1] + iv[NI - 1][0] + iv[0][0])) != 0x7fffffff)
     HKV_TRACE_AT(23) = globaltimer();  // the loads are back
 #endif
   if (valid) {  // else the attention launch failed its checks
@@ -890,18 +893,40 @@ __global__ void __maxnreg__(kFinishRegs)
       for (int c = 0; c < D / 4; ++c) o[c] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
   }
-  if (valid && rc.x >= 0) {
+  if (valid && rc.x >= 0 && rc.y <= NI) {
+    // at most NI pieces, all inline (the slots past the last piece hold empty
+    // pieces: weight 0): every lane merges them in piece order with no
+    // exchange, the largest maximum first, then the weighted sums
+    float gm = im[0];
+#pragma unroll
+    for (int u = 1; u < NI; ++u) gm = fmaxf(gm, im[u]);
+    float GL = 0.f, GA[CPL];
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) GA[c] = 0.f;
+#pragma unroll
+    for (int u = 0; u < NI; ++u) {
+      const float wu = im[u] == -INFINITY ? 0.f : exp2f(im[u] - gm);
+      GL += il[u] * wu;
+#pragma unroll
+      for (int c = 0; c < CPL; ++c) GA[c] = fmaf(iv[u][c], wu, GA[c]);
+    }
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) GA[c] /= GL;
+    V::st(p.out + (size_t)rc.x * D + CPL * lane, GA);
+  } else if (valid && rc.x >= 0) {
     const int hh = rc.x, np = rc.y;
     // piece j >= NI: the overflow slot of the CTA that computed it
     auto over = [&](int j) { return p.over + (size_t)(k - 1 + j) * PS; };
-    float m0 = im, l0 = il;  // piece `lane`
-    if (lane >= NI) {
-      m0 = -INFINITY;
-      l0 = 0.f;
-      if (lane < np) {
-        m0 = __ldcg(over(lane) + D);
-        l0 = __ldcg(over(lane) + D + 1);
+    float m0 = -INFINITY, l0 = 0.f;  // piece `lane`
+#pragma unroll
+    for (int u = 0; u < NI; ++u)
+      if (lane == u) {
+        m0 = im[u];
+        l0 = il[u];
       }
+    if (lane >= NI && lane < np) {
+      m0 = __ldcg(over(lane) + D);
+      l0 = __ldcg(over(lane) + D + 1);
     }
     // Merge in piece (index) order: the maximum first, then the weighted sums
     // (inline slots past the last piece hold empty pieces: weight 0).
