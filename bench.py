@@ -72,12 +72,13 @@ def describe(w, n_steps_window):
             f"period of P decode steps x L layers")
 
 
-def profiled_traffic(workload, bytes_per_launch, n_heads):
+def profiled_traffic(workload, bytes_per_launch):
     """DRAM bytes per decode step from the committed ncu summary: the
     attention kernel's measured traffic ratio to its algorithmic bytes, scaled
-    to this launch, plus the finishing kernel's bytes per head. None for
-    another kernel instantiation (the capture is of the Lumina-1024 shape:
-    D = 128, bf16) or when the kernel source has changed since the capture."""
+    to this launch, plus the finishing kernel's bytes per launch (set by the
+    grid: one CTA boundary's record and slots per warp). None for another
+    kernel instantiation (the capture is of the Lumina-1024 shape: D = 128,
+    bf16) or when the kernel source has changed since the capture."""
     if workload != "lumina1024":
         return None
     import hashlib
@@ -87,13 +88,13 @@ def profiled_traffic(workload, bytes_per_launch, n_heads):
         vals = {}
         for line in open(path):
             k, _, v = line.strip().partition(": ")
-            if k in ("source_sha256", "attn_traffic_ratio", "finish_traffic_bytes_per_head"):
+            if k in ("source_sha256", "attn_traffic_ratio", "finish_traffic_bytes_per_launch"):
                 vals[k] = v
         with open(src, "rb") as f:
             if hashlib.sha256(f.read()).hexdigest() != vals["source_sha256"]:
                 return None
         return (float(vals["attn_traffic_ratio"]) * bytes_per_launch
-                + float(vals["finish_traffic_bytes_per_head"]) * n_heads)
+                + float(vals["finish_traffic_bytes_per_launch"]))
     except (OSError, KeyError, ValueError):
         return None
 
@@ -446,7 +447,7 @@ def run_ours(args):
             "global_head_fraction": float((labels == 1).mean()),
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak,
-                         "traffic": profiled_traffic(w.name, bytes_per_launch, S * Hh),
+                         "traffic": profiled_traffic(w.name, bytes_per_launch),
                          "kernel": "hkv_decode_step: attn_kernel<fused> + finish_kernel<fused>",
                          "bytes_per_launch": bytes_per_launch, "launch_us": attn_us,
                          # the first step of the period, per layer (what a
