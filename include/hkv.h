@@ -276,6 +276,24 @@ hkv_status hkv_repack(const hkv_config *cfg, const hkv_cache *dense, const hkv_c
  * error word (HKV_OK if none), or HKV_ERR_CUDA if the stream failed. */
 hkv_status hkv_check(const hkv_cache *cache, hkv_stream_t stream);
 
+/* Copies one layer's cache state to host memory, for a checkpoint or for
+ * comparing the cache with a reference at any step (the paper has no
+ * counterpart). For the layer's S*H heads, in flat order s*H + h: label,
+ * len, nbuf and ntok (host arrays of S*H entries each, any of them NULL to
+ * skip), and the positions of every head's live tokens, head after head, in
+ * the order they sit in the head's segment (pos_out: host int32 array of
+ * pos_capacity entries, or NULL). *pos_count (if not NULL) receives the
+ * layer's live token count, the entries written to pos_out. Host memory may
+ * be pageable. Synchronises the stream; the work queued before it on the
+ * stream is included.
+ *  - pos_out given and pos_capacity below the live token count ->
+ *    HKV_ERR_CAPACITY (nothing written to pos_out);
+ *  - a segment with len < 0 or outside the arena -> HKV_ERR_BOUNDS. */
+hkv_status hkv_export_state(const hkv_config *cfg, const hkv_cache *cache, int layer,
+                            uint8_t *label_out, int32_t *len_out, int32_t *nbuf_out,
+                            int32_t *ntok_out, int32_t *pos_out, int64_t pos_capacity,
+                            int64_t *pos_count, hkv_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -1,12 +1,15 @@
 // Host side of the HeadKV C-ABI (include/hkv.h): argument validation, fault
-// injection for tests, per-device launch setup, and the kernel launches.
+// injection for tests, per-device launch setup, the kernel launches, and the
+// state export.
 #include <cuda_runtime.h>
 #include <math.h>
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
 
+#include <algorithm>
 #include <mutex>
+#include <vector>
 
 #include "hkv.h"
 #include "hkv_kernels.h"
@@ -404,6 +407,54 @@ hkv_status hkv_repack(const hkv_config *cfg, const hkv_cache *dense, const hkv_c
   return cuda_status(launch_repack(cache_args(dense), cache_args(ragged), method_args(cfg),
                                    layer * hpl, hpl, cfg->head_dim, cfg->dtype, smem,
                                    (cudaStream_t)stream));
+}
+
+hkv_status hkv_export_state(const hkv_config *cfg, const hkv_cache *cache, int layer,
+                            uint8_t *label_out, int32_t *len_out, int32_t *nbuf_out,
+                            int32_t *ntok_out, int32_t *pos_out, int64_t pos_capacity,
+                            int64_t *pos_count, hkv_stream_t stream) {
+  HKV_TRY(injected("export_state"));
+  HKV_TRY(hkv_validate_config(cfg));
+  if (!cache || !cache->off || !cache->len || !cache->nbuf || !cache->ntok || !cache->label ||
+      (pos_out && !cache->pos) || pos_capacity < 0)
+    return HKV_ERR_INVALID_ARG;
+  if (layer < 0 || layer >= cfg->n_layers) return HKV_ERR_INVALID_ARG;
+  const int hpl = heads_per_layer(cfg);
+  const size_t base = (size_t)layer * hpl;
+  cudaStream_t s = (cudaStream_t)stream;
+  std::vector<int64_t> off(hpl);
+  std::vector<int32_t> len(hpl);
+  auto d2h = [&](void *dst, const void *src, size_t bytes) {
+    return cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToHost, s) == cudaSuccess;
+  };
+  bool ok = d2h(off.data(), cache->off + base, hpl * sizeof(int64_t)) &&
+            d2h(len.data(), cache->len + base, hpl * sizeof(int32_t));
+  if (label_out) ok = ok && d2h(label_out, cache->label + base, hpl * sizeof(uint8_t));
+  if (nbuf_out) ok = ok && d2h(nbuf_out, cache->nbuf + base, hpl * sizeof(int32_t));
+  if (ntok_out) ok = ok && d2h(ntok_out, cache->ntok + base, hpl * sizeof(int32_t));
+  if (!ok || cudaStreamSynchronize(s) != cudaSuccess) return HKV_ERR_CUDA;
+  if (len_out) std::copy(len.begin(), len.end(), len_out);
+  int64_t total = 0, lo = INT64_MAX, hi = 0;
+  for (int h = 0; h < hpl; ++h) {
+    if (len[h] < 0 || off[h] < 0 || off[h] + len[h] > cache->capacity_tokens) return HKV_ERR_BOUNDS;
+    total += len[h];
+    if (len[h] > 0) {
+      lo = std::min(lo, off[h]);
+      hi = std::max(hi, off[h] + (int64_t)len[h]);
+    }
+  }
+  if (pos_count) *pos_count = total;
+  if (!pos_out || total == 0) return HKV_OK;
+  if (pos_capacity < total) return HKV_ERR_CAPACITY;
+  // one copy of the span the layer's live tokens occupy, then packed
+  std::vector<int32_t> span((size_t)(hi - lo));
+  if (!d2h(span.data(), cache->pos + lo, span.size() * sizeof(int32_t)) ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return HKV_ERR_CUDA;
+  int64_t w = 0;
+  for (int h = 0; h < hpl; ++h)
+    for (int j = 0; j < len[h]; ++j) pos_out[w++] = span[(size_t)(off[h] - lo + j)];
+  return HKV_OK;
 }
 
 hkv_status hkv_check(const hkv_cache *cache, hkv_stream_t stream) {

@@ -77,6 +77,8 @@ _SIGNATURES = {
                               POINTER(c_int64), c_void_p], c_int),
     "hkv_repack": ([POINTER(hkv_config), POINTER(hkv_cache), POINTER(hkv_cache), c_int, c_void_p], c_int),
     "hkv_check": ([POINTER(hkv_cache), c_void_p], c_int),
+    "hkv_export_state": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p, c_void_p, c_void_p,
+                          c_void_p, c_void_p, c_int64, POINTER(c_int64), c_void_p], c_int),
 }
 
 
@@ -179,3 +181,24 @@ def hkv_repack(cfg, dense, ragged, layer, stream=0) -> None:
 
 def hkv_check(cache, stream=0) -> None:
     _call("check", ctypes.byref(cache), stream)
+
+
+def hkv_export_state(cfg, cache, layer, stream=0):
+    """One layer's state on the host: numpy arrays label, len, nbuf, ntok
+    (S*H each) and the live positions of every head, packed head after head
+    (a list of arrays, one per head)."""
+    import numpy as np
+    n = cfg.n_seqs * cfg.n_heads
+    label = np.zeros(n, np.uint8)
+    ln = np.zeros(n, np.int32)
+    nbuf = np.zeros(n, np.int32)
+    ntok = np.zeros(n, np.int32)
+    count = c_int64(0)
+    _call("export_state", ctypes.byref(cfg), ctypes.byref(cache), layer, label.ctypes.data,
+          ln.ctypes.data, nbuf.ctypes.data, ntok.ctypes.data, None, 0, ctypes.byref(count), stream)
+    pos = np.zeros(max(int(count.value), 1), np.int32)
+    _call("export_state", ctypes.byref(cfg), ctypes.byref(cache), layer, None, None, None, None,
+          pos.ctypes.data, pos.size, ctypes.byref(count), stream)
+    split = np.cumsum(ln)[:-1]
+    return {"label": label, "len": ln, "nbuf": nbuf, "ntok": ntok,
+            "pos": np.split(pos[:int(count.value)], split)}

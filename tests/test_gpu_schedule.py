@@ -146,3 +146,60 @@ def test_model_shapes_two_layers_two_seqs(name, rho, fused):
         budget = O.global_budget(w.rho, w.n_image) if labels[i] == 1 else w.recent_w
         assert poss[w.n_image - 1][i].size == w.n_cond + budget + t_r.nbuf
     assert worst <= TOL[w.dtype], worst
+
+
+def test_export_state_matches_the_cache():
+    """hkv_export_state returns the layer's counters, labels and live
+    positions (segment order) as the cache arrays hold them, through the
+    dense phase, grouping and compressed decode."""
+    from paper_2605_20600_gb300 import hkv as H
+    from paper_2605_20600_gb300.engine import Engine
+    from paper_2605_20600_gb300.runner import generate
+    from synth.gpu import DeviceSynth
+    from _gpu_util import cfg_of
+    w = configs.TINY
+    eng = Engine(cfg_of(H, w), "cuda")
+    n = w.n_seqs * w.n_heads
+    seen = []
+
+    def on_step(t, out):
+        if t % 29 != 3 and t != w.group_at - 1 and t != w.n_image - 1:
+            return
+        cc = eng.cache
+        for layer in range(w.n_layers):
+            st = H.hkv_export_state(eng.cfg, cc.c, layer)
+            sl = slice(layer * n, (layer + 1) * n)
+            for k in ("label", "len", "nbuf", "ntok"):
+                assert np.array_equal(st[k], getattr(cc, k)[sl].cpu().numpy()), (t, k)
+            off, ln = cc.off[sl].cpu().numpy(), cc.len[sl].cpu().numpy()
+            pos = cc.pos.cpu().numpy()
+            for h in range(n):
+                assert np.array_equal(st["pos"][h], pos[off[h]: off[h] + ln[h]]), (t, h)
+        seen.append(t)
+
+    generate(eng, DeviceSynth(w, "cuda"), on_step=on_step)
+    eng.check()
+    assert len(seen) >= 8 and w.group_at - 1 in seen
+
+
+def test_export_state_capacity():
+    import ctypes
+    from paper_2605_20600_gb300 import hkv as H
+    from paper_2605_20600_gb300.engine import Engine
+    from _gpu_util import cfg_of
+    w = configs.TINY
+    eng = Engine(cfg_of(H, w), "cuda")
+    cc = eng.cache
+    cc.len.fill_(3)
+    cc.off.copy_(cc.off.new_tensor(list(range(0, 8 * 40, 40))))
+    out = np.zeros(23, np.int32)
+    cnt = ctypes.c_int64(0)
+    f = H.lib().hkv_export_state
+    args = (ctypes.byref(eng.cfg), ctypes.byref(cc.c), 0, None, None, None, None)
+    assert f(*args, out.ctypes.data, 23, ctypes.byref(cnt), None) == H.HKV_ERR_CAPACITY
+    assert cnt.value == 24
+    big = np.zeros(24, np.int32)
+    assert f(*args, big.ctypes.data, 24, ctypes.byref(cnt), None) == 0
+    assert np.array_equal(big, cc.pos.cpu().numpy()[np.add.outer(np.arange(0, 320, 40), np.arange(3)).ravel()])
+    cc.len[2] = -1
+    assert f(*args, None, 0, ctypes.byref(cnt), None) == H.HKV_ERR_BOUNDS
