@@ -601,6 +601,84 @@ def run_strategies(args):
     print(json.dumps(line), flush=True)
 
 
+def run_grouping(args):
+    """--grouping: the grouping token's step (image token E - 1, every layer,
+    on the uncompressed cache) with the head types decided two ways: a decode
+    step followed by hkv_identify_heads (a second pass over every head's
+    dense keys), or hkv_decode_step_identify (the decision taken in the
+    step's own pass). Each way is one CUDA graph of the L layers, replayed
+    after restoring the counters the step advances (the rows it writes are
+    the same every time); the labels of the two ways are compared."""
+    import torch
+
+    from paper_2605_20600_gb300 import hkv as H
+    from paper_2605_20600_gb300.engine import Engine, torch_dtype
+    from paper_2605_20600_gb300.runner import generate
+    from synth.gpu import DeviceSynth
+
+    dev = torch.device("cuda", 0)
+    w = workload(args)
+    L, S, Hh, D, E = w.n_layers, w.n_seqs, w.n_heads, w.head_dim, w.group_at
+    cfg = H.make_config(n_layers=L, n_seqs=S, n_heads=Hh, head_dim=D, dtype=w.dtype,
+                        n_cond=w.n_cond, n_image=w.n_image, row_len=w.row_len,
+                        recent_w=w.recent_w, local_w=w.w_loc, period=w.period, group_at=E,
+                        rho=w.rho, tau=w.tau, r_s=w.r_s)
+    eng = Engine(cfg, dev)
+    synth = DeviceSynth(w, dev)
+    generate(eng, synth, last_step=E - 2)                   # the dense phase up to E - 2
+    dt = torch_dtype(cfg)
+    q = torch.empty(L, S, Hh, D, dtype=dt, device=dev)
+    k, v = torch.empty_like(q), torch.empty_like(q)
+    synth.image(q, k, v, 0, L, E - 1, 1)
+    out = torch.empty(L, S, Hh, D, dtype=torch.float32, device=dev)
+    c = eng.dense
+    saved = [x.clone() for x in (c.len, c.nbuf, c.ntok)]
+
+    def restore():
+        for x, y in zip((c.len, c.nbuf, c.ntok), saved):
+            x.copy_(y)
+
+    def separate():
+        for layer in range(L):
+            eng.step(layer, q[layer], k[layer], v[layer], out[layer])
+            eng.identify(layer, q[layer])
+
+    def fused():
+        for layer in range(L):
+            eng.step_identify(layer, q[layer], k[layer], v[layer], out[layer])
+
+    res, labels = {}, {}
+    for name, fn in (("separate", separate), ("fused", fused)):
+        restore()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            fn()
+        times = []
+        for rep in range(args.warmup + args.steps):
+            restore()
+            eng.labels.fill_(H.HKV_DENSE)
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            g.replay()
+            e1.record()
+            torch.cuda.synchronize()
+            if rep >= args.warmup:
+                times.append(e0.elapsed_time(e1) * 1000.0)
+        eng.check()
+        labels[name] = eng.labels.cpu().numpy().copy()
+        res[name] = {"us_per_layer": statistics.median(times) / L,
+                     "global_fraction": float((labels[name] == H.HKV_GLOBAL).mean())}
+    dense_bytes = (eng.dense.len.sum().item() + L * S * Hh) * D * 2 * (2 if w.dtype == "bf16" else 4)
+    line = {"grouping": f"{w.name}: image token E-1 = {E - 1}, {L} layers x {S * Hh} heads",
+            "unit": "us per layer (median of steps)", **res,
+            "labels_differ": int((labels["separate"] != labels["fused"]).sum()),
+            "dense_kv_bytes_per_step": dense_bytes,
+            "note": "separate: hkv_decode_step then hkv_identify_heads; fused: "
+                    "hkv_decode_step_identify; one CUDA graph of all layers each"}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -613,9 +691,14 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--strategies", action="store_true",
                     help="compare decode attention with the padding and per-group strategies")
+    ap.add_argument("--grouping", action="store_true",
+                    help="time the grouping step with identification separate and fused")
     args = ap.parse_args()
     if args.strategies:
         run_strategies(args)
+        return
+    if args.grouping:
+        run_grouping(args)
         return
     if args.impl == "reference":
         if int(os.environ.get("RANK", "0")) == 0:

@@ -211,6 +211,23 @@ hkv_status hkv_decode_step(const hkv_config *cfg, const hkv_cache *cache, int la
                            const void *q, const void *k, const void *v, float *out,
                            void *workspace, size_t ws_bytes, int flags, hkv_stream_t stream);
 
+/* hkv_decode_step fused with the head-type identification of Sec. 4,
+ * Step 2, for the grouping step (image token E - 1) on the uncompressed
+ * cache: besides everything hkv_decode_step does, each head's attention
+ * mass on its newest local_w - 1 tokens (the new one included) is
+ * accumulated with the softmax sum, and label_out[i] (device, [L*S*H], flat
+ * head index i) becomes HKV_LOCAL iff that mass is at least tau of the
+ * total, i.e. iff fewer than local_w tokens, counted back from the newest,
+ * carry tau of the attention; else HKV_GLOBAL. Same decision as
+ * hkv_identify_heads over the same cache (which also reports n_h; this
+ * does not). A head of another label than HKV_DENSE sets HKV_ERR_STATE in
+ * the error word and the step is not taken; label_out NULL ->
+ * HKV_ERR_INVALID_ARG. */
+hkv_status hkv_decode_step_identify(const hkv_config *cfg, const hkv_cache *cache, int layer,
+                                    const void *q, const void *k, const void *v, float *out,
+                                    uint8_t *label_out, void *workspace, size_t ws_bytes,
+                                    int flags, hkv_stream_t stream);
+
 /* Eq. 1 for one new query per head over that head's live tokens (any mix
  * of lengths): out[s][h][:] = softmax(q k^T / sqrt(d)) V, fp32 accumulation,
  * written in fp32 ([S][H][head_dim]). Split-K over the layer's total token

@@ -307,13 +307,16 @@ hkv_status hkv_decode_attention(const hkv_config *cfg, const hkv_cache *cache, i
   HKV_TRY(attn_grid(cfg, &grid));
   const AttnArgs a = attn_args(cfg, cache, layer, q, out, workspace);
   return cuda_status(
-      launch_attention(a, cfg->head_dim, cfg->dtype, grid, false, (cudaStream_t)stream));
+      launch_attention(a, cfg->head_dim, cfg->dtype, grid, false, false, (cudaStream_t)stream));
 }
 
-hkv_status hkv_decode_step(const hkv_config *cfg, const hkv_cache *cache, int layer,
-                           const void *q, const void *k, const void *v, float *out,
-                           void *workspace, size_t ws_bytes, int flags, hkv_stream_t stream) {
-  HKV_TRY(injected("decode_step"));
+namespace {
+
+hkv_status decode_step(const char *name, const hkv_config *cfg, const hkv_cache *cache, int layer,
+                       const void *q, const void *k, const void *v, float *out,
+                       uint8_t *label_out, void *workspace, size_t ws_bytes, int flags,
+                       hkv_stream_t stream) {
+  HKV_TRY(injected(name));
   HKV_TRY(hkv_validate_config(cfg));
   HKV_TRY(check_cache(cache));
   if (layer < 0 || layer >= cfg->n_layers) return HKV_ERR_INVALID_ARG;
@@ -328,8 +331,29 @@ hkv_status hkv_decode_step(const hkv_config *cfg, const hkv_cache *cache, int la
   a.k_new = k;
   a.v_new = v;
   a.prefetch = (flags & HKV_STEP_PREFETCH) ? 1 : 0;
-  return cuda_status(
-      launch_attention(a, cfg->head_dim, cfg->dtype, grid, true, (cudaStream_t)stream));
+  a.label_out = label_out;
+  a.w_loc = cfg->local_w;
+  a.tau = (float)cfg->tau;
+  return cuda_status(launch_attention(a, cfg->head_dim, cfg->dtype, grid, true,
+                                      label_out != nullptr, (cudaStream_t)stream));
+}
+
+}  // namespace
+
+hkv_status hkv_decode_step(const hkv_config *cfg, const hkv_cache *cache, int layer,
+                           const void *q, const void *k, const void *v, float *out,
+                           void *workspace, size_t ws_bytes, int flags, hkv_stream_t stream) {
+  return decode_step("decode_step", cfg, cache, layer, q, k, v, out, nullptr, workspace, ws_bytes,
+                     flags, stream);
+}
+
+hkv_status hkv_decode_step_identify(const hkv_config *cfg, const hkv_cache *cache, int layer,
+                                    const void *q, const void *k, const void *v, float *out,
+                                    uint8_t *label_out, void *workspace, size_t ws_bytes,
+                                    int flags, hkv_stream_t stream) {
+  if (!label_out) return HKV_ERR_INVALID_ARG;
+  return decode_step("decode_step_identify", cfg, cache, layer, q, k, v, out, label_out,
+                     workspace, ws_bytes, flags, stream);
 }
 
 hkv_status hkv_evict(const hkv_config *cfg, const hkv_cache *cache, int layer,

@@ -136,6 +136,8 @@ constexpr int kFirst = 1, kLast = 2, kDone = 4;
 
 struct TileMeta {           // producer -> consumers, one per stage
   int h, n, flags;          // head, rows, kFirst | kLast | kDone
+  int recent0;              // identification: rows from here on are among the
+                            // head's newest w_loc - 1
   long long hs, he;         // the head's rows in the index space
 };
 
@@ -313,7 +315,7 @@ struct Pending {
   bool first, has_new;
 };
 
-template <int D, typename T, bool FUSED>
+template <int D, typename T, bool FUSED, bool IDENT>
 __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p) {
   using S = AttnShape<D, T>;
   constexpr int LPR = S::kLPR, EPL = S::kEPL, RPW = S::kRPW, TT = S::kTT;
@@ -329,6 +331,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
   static_assert(NST <= 32, "a lane of the epilogue per state");
   __shared__ __align__(16) float red_acc[NST][D];
   __shared__ float red_m[NST], red_l[NST];
+  __shared__ float red_r[IDENT ? NST : 1];  // identification: mass of the newest rows
   __shared__ TileMeta meta[NS];
   __shared__ SegMeta seg;
   __shared__ HeadTable tab;
@@ -386,6 +389,8 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
       else if (l + 1 > cp) bad = bad ? bad : HKV_ERR_CAPACITY;
       else if (lab != HKV_DENSE && nb >= p.period)
         bad = bad ? bad : HKV_ERR_STATE;  // the periodic update is due first
+      else if (IDENT && lab != HKV_DENSE)
+        bad = bad ? bad : HKV_ERR_STATE;  // identification reads the dense cache's row order
     }
   };
 #pragma unroll 4
@@ -486,6 +491,10 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
     mt.flags = (pd.first ? kFirst : 0) | (ge == (b < he ? b : he) ? kLast : 0);
     mt.hs = pit.hs;
     mt.he = he;
+    if (IDENT) {
+      const long long r0n = he - (p.w_loc - 1) - pit.g;  // first of the newest rows, tile-local
+      mt.recent0 = r0n < 0 ? 0 : (int)(r0n < TT ? r0n : TT);
+    }
     if (n_old > 0) {
       const uint32_t bytes = (uint32_t)n_old * RB;
       const long long row = look.off(pit.h) + r0;
@@ -585,7 +594,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
     static_assert(M::kEPL == EPL, "lane mapping");
     typename M::Q q;
     float2 acc[EPL / 2];
-    float m = -INFINITY, l = 0.f;
+    float m = -INFINITY, l = 0.f, lr = 0.f;  // lr: identification's newest-row mass
     int nseg = 0;
 #pragma unroll
     for (int e = 0; e < EPL / 2; ++e) acc[e] = make_float2(0.f, 0.f);
@@ -619,7 +628,9 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
         for (int e = 0; e < EPL / 2; ++e) acc[e] = make_float2(0.f, 0.f);
         m = -INFINITY;
         l = 0.f;
+        lr = 0.f;
       }
+      const int recent0 = IDENT ? meta[stage].recent0 : 0;
 
       float sc[S::kSteps];
 #pragma unroll
@@ -638,6 +649,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
       if (mn != -INFINITY) {
         const float corr = exp2f(m - mn);
         l *= corr;
+        if (IDENT) lr *= corr;
 #pragma unroll
         for (int e = 0; e < EPL / 2; ++e) acc[e] = __fmul2_rn(acc[e], make_float2(corr, corr));
 #pragma unroll
@@ -646,6 +658,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
           if (r < n) {
             const float pr = exp2f(sc[st] - mn);
             l += pr;
+            if (IDENT && r >= recent0) lr += pr;
             M::add_v(acc, *reinterpret_cast<const uint4 *>(Vs + r * RB + col * 16), pr);
           }
         }
@@ -679,6 +692,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
           if (col == 0) {
             red_m[si] = m;
             red_l[si] = l;
+            if (IDENT) red_r[si] = lr;
           }
         }
         if (cw == 0 && lane == 0) seg = sm;
@@ -732,6 +746,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
         if (lane == 0) {
           pp[D] = -INFINITY;
           pp[D + 1] = 0.f;
+          pp[D + 2] = 0.f;
         }
       }
     }
@@ -757,8 +772,12 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
       for (int o = 16; o >= 1; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, o));
       const float ws = ms == -INFINITY ? 0.f : exp2f(ms - mx);
       float L = lane < NST ? red_l[lane] * ws : 0.f;
+      float LR = IDENT && lane < NST ? red_r[lane] * ws : 0.f;
 #pragma unroll
-      for (int o = 16; o >= 1; o >>= 1) L += __shfl_xor_sync(0xFFFFFFFFu, L, o);
+      for (int o = 16; o >= 1; o >>= 1) {
+        L += __shfl_xor_sync(0xFFFFFFFFu, L, o);
+        if (IDENT) LR += __shfl_xor_sync(0xFFFFFFFFu, LR, o);
+      }
       float A[CPL];
 #pragma unroll
       for (int c = 0; c < CPL; ++c) A[c] = 0.f;
@@ -776,6 +795,10 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
 #pragma unroll
         for (int c = 0; c < CPL; ++c) A[c] /= L;
         V::st(p.out + (size_t)h * D + CPL * lane, A);
+        // Sec. 4 Step 2: local iff the newest w_loc - 1 tokens hold a share
+        // tau of the attention
+        if (IDENT && lane == 0)
+          p.label_out[p.layer_base + h] = LR >= p.tau * L ? HKV_LOCAL : HKV_GLOBAL;
       } else {  // piece j of the head split at boundary k0 + 1
         const long long k0 = hs / chunk;
         const int j = (int)(blockIdx.x - k0);
@@ -786,6 +809,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
         if (lane == 0) {
           pp[D] = mx;
           pp[D + 1] = L;
+          if (IDENT) pp[D + 2] = LR;
         }
       }
       // Fused: the CTA whose range holds the head's last row appends the new
@@ -824,8 +848,8 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p)
 // head and the boundary's inline slots (its first pieces, or empty pieces
 // the attention kernel wrote there) load in the same round as the counters:
 // a head of at most kAttnInlinePieces pieces costs one round trip to memory.
-template <int D, typename T, bool FUSED>
-__global__ void __maxnreg__(kFinishRegs)
+template <int D, typename T, bool FUSED, bool IDENT>
+__global__ void __maxnreg__(IDENT ? kFinishRegs + 16 : kFinishRegs)
     finish_kernel(const AttnArgs p) {
   constexpr int CPL = D / 32;
   using V = Vec<CPL>;
@@ -858,10 +882,12 @@ __global__ void __maxnreg__(kFinishRegs)
   int4 rc = make_int4(-1, 0, 0, 0);
   float iv[NI][CPL];
   float im[NI], il[NI];  // maxima and sums of the inline pieces (every lane)
+  float ir[IDENT ? NI : 1];  // identification: their newest-row masses
 #pragma unroll
   for (int u = 0; u < NI; ++u) {
     im[u] = -INFINITY;
     il[u] = 0.f;
+    if (IDENT) ir[u] = 0.f;
 #pragma unroll
     for (int c = 0; c < CPL; ++c) iv[u][c] = 0.f;
   }
@@ -873,6 +899,7 @@ __global__ void __maxnreg__(kFinishRegs)
       V::ldcg(inl + (size_t)u * PS + CPL * lane, iv[u]);
       im[u] = __ldcg(inl + (size_t)u * PS + D);
       il[u] = __ldcg(inl + (size_t)u * PS + D + 1);
+      if (IDENT) ir[u] = __ldcg(inl + (size_t)u * PS + D + 2);
     }
   }
 #ifdef HKV_ATTN_TRACE
@@ -900,33 +927,38 @@ __global__ void __maxnreg__(kFinishRegs)
     float gm = im[0];
 #pragma unroll
     for (int u = 1; u < NI; ++u) gm = fmaxf(gm, im[u]);
-    float GL = 0.f, GA[CPL];
+    float GL = 0.f, GR = 0.f, GA[CPL];
 #pragma unroll
     for (int c = 0; c < CPL; ++c) GA[c] = 0.f;
 #pragma unroll
     for (int u = 0; u < NI; ++u) {
       const float wu = im[u] == -INFINITY ? 0.f : exp2f(im[u] - gm);
       GL += il[u] * wu;
+      if (IDENT) GR += ir[u] * wu;
 #pragma unroll
       for (int c = 0; c < CPL; ++c) GA[c] = fmaf(iv[u][c], wu, GA[c]);
     }
 #pragma unroll
     for (int c = 0; c < CPL; ++c) GA[c] /= GL;
     V::st(p.out + (size_t)rc.x * D + CPL * lane, GA);
+    if (IDENT && lane == 0)  // Sec. 4 Step 2, as in the attention kernel
+      p.label_out[p.layer_base + rc.x] = GR >= p.tau * GL ? HKV_LOCAL : HKV_GLOBAL;
   } else if (valid && rc.x >= 0) {
     const int hh = rc.x, np = rc.y;
     // piece j >= NI: the overflow slot of the CTA that computed it
     auto over = [&](int j) { return p.over + (size_t)(k - 1 + j) * PS; };
-    float m0 = -INFINITY, l0 = 0.f;  // piece `lane`
+    float m0 = -INFINITY, l0 = 0.f, r0 = 0.f;  // piece `lane`
 #pragma unroll
     for (int u = 0; u < NI; ++u)
       if (lane == u) {
         m0 = im[u];
         l0 = il[u];
+        if (IDENT) r0 = ir[u];
       }
     if (lane >= NI && lane < np) {
       m0 = __ldcg(over(lane) + D);
       l0 = __ldcg(over(lane) + D + 1);
+      if (IDENT) r0 = __ldcg(over(lane) + D + 2);
     }
     // Merge in piece (index) order: the maximum first, then the weighted sums
     // (inline slots past the last piece hold empty pieces: weight 0).
@@ -934,23 +966,25 @@ __global__ void __maxnreg__(kFinishRegs)
     for (int j = lane + 32; j < np; j += 32) gm = fmaxf(gm, __ldcg(over(j) + D));
 #pragma unroll
     for (int o = 16; o >= 1; o >>= 1) gm = fmaxf(gm, __shfl_xor_sync(0xFFFFFFFFu, gm, o));
-    float GL = 0.f, GA[CPL];
+    float GL = 0.f, GR = 0.f, GA[CPL];
 #pragma unroll
     for (int c = 0; c < CPL; ++c) GA[c] = 0.f;
     for (int j0 = 0; j0 < np; j0 += 32) {
-      float mj = m0, lj = l0;
+      float mj = m0, lj = l0, rj = r0;
       if (j0 > 0) {
         const int j = j0 + lane;
         mj = -INFINITY;
-        lj = 0.f;
+        lj = rj = 0.f;
         if (j < np) {
           mj = __ldcg(over(j) + D);
           lj = __ldcg(over(j) + D + 1);
+          if (IDENT) rj = __ldcg(over(j) + D + 2);
         }
       }
       // weight of piece j0 + lane (zero past the last piece)
       const float wj = mj == -INFINITY ? 0.f : exp2f(mj - gm);
       const float lw = lj * wj;
+      const float rw = IDENT ? rj * wj : 0.f;
       const int cnt = np - j0 < 32 ? np - j0 : 32;
       for (int t0 = 0; t0 < cnt; t0 += NI) {
         float v[NI][CPL];
@@ -974,6 +1008,7 @@ __global__ void __maxnreg__(kFinishRegs)
         for (int u = 0; u < NI; ++u) {
           const float wu = __shfl_sync(0xFFFFFFFFu, wj, t0 + u);
           GL += __shfl_sync(0xFFFFFFFFu, lw, t0 + u);
+          if (IDENT) GR += __shfl_sync(0xFFFFFFFFu, rw, t0 + u);
           if (j0 + t0 + u < np)
 #pragma unroll
             for (int c = 0; c < CPL; ++c) GA[c] = fmaf(v[u][c], wu, GA[c]);
@@ -983,6 +1018,8 @@ __global__ void __maxnreg__(kFinishRegs)
 #pragma unroll
     for (int c = 0; c < CPL; ++c) GA[c] /= GL;
     V::st(p.out + (size_t)hh * D + CPL * lane, GA);
+    if (IDENT && lane == 0)
+      p.label_out[p.layer_base + hh] = GR >= p.tau * GL ? HKV_LOCAL : HKV_GLOBAL;
   }
   HKV_TRACE(22);
 }
@@ -992,23 +1029,24 @@ size_t smem_bytes() {
   return (size_t)AttnShape<D, T>::kNS * AttnShape<D, T>::kStageBytes;
 }
 
-template <int D, typename T, bool F>
+template <int D, typename T, bool F, bool I>
 cudaError_t prepare_t(int *ctas) {
   const size_t smem = smem_bytes<D, T>();
-  cudaError_t e = cudaFuncSetAttribute(attn_kernel<D, T, F>,
+  cudaError_t e = cudaFuncSetAttribute(attn_kernel<D, T, F, I>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas, attn_kernel<D, T, F>, kAttnThreads,
-                                                       smem);
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas, attn_kernel<D, T, F, I>,
+                                                       kAttnThreads, smem);
 }
 
 template <int D, typename T>
-cudaError_t prepare_both(int *ctas) {
-  int a = 0, b = 0;
-  cudaError_t e = prepare_t<D, T, false>(&a);
-  if (e != cudaSuccess) return e;
-  e = prepare_t<D, T, true>(&b);
+cudaError_t prepare_all(int *ctas) {
+  int a = 0, b = 0, c = 0;
+  cudaError_t e = prepare_t<D, T, false, false>(&a);
+  if (e == cudaSuccess) e = prepare_t<D, T, true, false>(&b);
+  if (e == cudaSuccess) e = prepare_t<D, T, true, true>(&c);
   *ctas = a < b ? a : b;
+  if (c < *ctas) *ctas = c;
   if (*ctas > HKV_ATTN_MAX_CTAS_PER_SM) *ctas = HKV_ATTN_MAX_CTAS_PER_SM;
   return e;
 }
@@ -1030,20 +1068,24 @@ cudaError_t launch_pdl(K kernel, int grid, int threads, size_t smem, const AttnA
   return cudaLaunchKernelEx(&cfg, kernel, a);
 }
 
-template <int D, typename T>
-cudaError_t launch_t(AttnArgs a, int grid, bool fused, cudaStream_t s) {
-  a.grid = grid;
-  cudaError_t e =
-      fused ? launch_pdl(attn_kernel<D, T, true>, grid, kAttnThreads, smem_bytes<D, T>(), a, s)
-            : launch_pdl(attn_kernel<D, T, false>, grid, kAttnThreads, smem_bytes<D, T>(), a, s);
+template <int D, typename T, bool F, bool I>
+cudaError_t launch_both(const AttnArgs &a, int grid, cudaStream_t s) {
+  cudaError_t e = launch_pdl(attn_kernel<D, T, F, I>, grid, kAttnThreads, smem_bytes<D, T>(), a, s);
   if (e != cudaSuccess) return e;
   // a warp for every 32 heads and for every CTA boundary
   int warps = (a.nheads + 31) / 32;
   if (warps < grid - 1) warps = grid - 1;
   if (warps < 1) warps = 1;
   const int fgrid = (warps + kFinishThreads / 32 - 1) / (kFinishThreads / 32);
-  return fused ? launch_pdl(finish_kernel<D, T, true>, fgrid, kFinishThreads, 0, a, s)
-               : launch_pdl(finish_kernel<D, T, false>, fgrid, kFinishThreads, 0, a, s);
+  return launch_pdl(finish_kernel<D, T, F, I>, fgrid, kFinishThreads, 0, a, s);
+}
+
+template <int D, typename T>
+cudaError_t launch_t(AttnArgs a, int grid, bool fused, bool identify, cudaStream_t s) {
+  a.grid = grid;
+  if (!fused) return launch_both<D, T, false, false>(a, grid, s);
+  return identify ? launch_both<D, T, true, true>(a, grid, s)
+                  : launch_both<D, T, true, false>(a, grid, s);
 }
 
 }  // namespace
@@ -1061,17 +1103,18 @@ size_t attention_smem_bytes(int D, int dtype) {
 }
 
 cudaError_t attention_prepare(int D, int dtype, int *ctas) {
-  if (dtype == HKV_BF16) return D == 64 ? prepare_both<64, __nv_bfloat16>(ctas) : prepare_both<128, __nv_bfloat16>(ctas);
-  return D == 64 ? prepare_both<64, float>(ctas) : prepare_both<128, float>(ctas);
+  if (dtype == HKV_BF16) return D == 64 ? prepare_all<64, __nv_bfloat16>(ctas) : prepare_all<128, __nv_bfloat16>(ctas);
+  return D == 64 ? prepare_all<64, float>(ctas) : prepare_all<128, float>(ctas);
 }
 
 cudaError_t launch_attention(const AttnArgs &a, int D, int dtype, int grid, bool fused,
-                             cudaStream_t s) {
+                             bool identify, cudaStream_t s) {
   if (grid < 1 || grid > kAttnMaxGrid) return cudaErrorInvalidValue;
   if (dtype == HKV_BF16)
-    return D == 64 ? launch_t<64, __nv_bfloat16>(a, grid, fused, s)
-                   : launch_t<128, __nv_bfloat16>(a, grid, fused, s);
-  return D == 64 ? launch_t<64, float>(a, grid, fused, s) : launch_t<128, float>(a, grid, fused, s);
+    return D == 64 ? launch_t<64, __nv_bfloat16>(a, grid, fused, identify, s)
+                   : launch_t<128, __nv_bfloat16>(a, grid, fused, identify, s);
+  return D == 64 ? launch_t<64, float>(a, grid, fused, identify, s)
+                 : launch_t<128, float>(a, grid, fused, identify, s);
 }
 
 }  // namespace hkv

@@ -52,6 +52,11 @@ struct AttnArgs {
   float qscale;               // log2(e) / sqrt(D)
   int prefetch;               // read the layer's cache before waiting for the
                               // previous kernel (its writes do not touch it)
+  // identification fused into the step (Sec. 4, Step 2): a head is local iff
+  // its newest w_loc - 1 tokens hold at least tau of its attention
+  uint8_t *label_out;         // [L*S*H]
+  int w_loc;
+  float tau;
 };
 
 // decode attention CTA: one producer warp (TMA), consumer warps, one
@@ -76,9 +81,10 @@ constexpr int kAttnInlinePieces = 4;
 size_t attention_smem_bytes(int D, int dtype);
 cudaError_t attention_prepare(int D, int dtype, int *ctas_per_sm);
 // launches the attention kernel on `grid` CTAs (at most kAttnMaxGrid) and the
-// finishing kernel behind it
+// finishing kernel behind it; identify (fused only): also the Step 2 label of
+// every head into label_out
 cudaError_t launch_attention(const AttnArgs &a, int D, int dtype, int grid, bool fused,
-                             cudaStream_t s);
+                             bool identify, cudaStream_t s);
 
 // per-head cache maintenance (append / update / repack / prefill / identify)
 struct CacheArgs {

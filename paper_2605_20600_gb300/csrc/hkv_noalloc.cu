@@ -117,7 +117,7 @@ extern "C" hkv_status hkv_decode_attention_noalloc(const hkv_config *cfg, const 
   a.arena_tokens = cache->capacity_tokens;
   a.nheads = hpl;
   a.qscale = (float)(1.4426950408889634 / sqrt((double)cfg->head_dim));
-  return launch_attention(a, cfg->head_dim, cfg->dtype, grid, false, s) == cudaSuccess
+  return launch_attention(a, cfg->head_dim, cfg->dtype, grid, false, false, s) == cudaSuccess
              ? HKV_OK
              : HKV_ERR_CUDA;
 }

@@ -102,6 +102,13 @@ class Engine:
         return t > E and (t - E) % P == 0
 
     # Step 2
+    def step_identify(self, layer: int, q, k, v, out) -> None:
+        """The decode step of the grouping token with the head types (Sec. 4,
+        Step 2) decided in the same pass, into self.labels (no n_h)."""
+        flags = H.HKV_STEP_PREFETCH if self.cfg.n_layers >= 2 else 0
+        H.hkv_decode_step_identify(self.cfg, self.cache.c, layer, q, k, v, out, self.labels, self.ws,
+                                   self.ws_bytes, flags, self.stream())
+
     def identify(self, layer: int, q) -> None:
         H.hkv_identify_heads(self.cfg, self.dense.c, layer, q, self.labels, self.n_h, self.stream())
 

@@ -70,6 +70,9 @@ _SIGNATURES = {
                               c_size_t, c_void_p], c_int),
     "hkv_decode_step": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p, c_void_p, c_void_p,
                          c_void_p, c_void_p, c_size_t, c_int, c_void_p], c_int),
+    "hkv_decode_step_identify": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p, c_void_p,
+                                  c_void_p, c_void_p, c_void_p, c_void_p, c_size_t, c_int, c_void_p],
+                                 c_int),
     "hkv_evict": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p], c_int),
     "hkv_identify_heads": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p, c_void_p, c_void_p,
                             c_void_p], c_int),
@@ -157,6 +160,12 @@ def hkv_decode_step(cfg, cache, layer, q, k, v, out, workspace, ws_bytes, flags=
                     stream=0) -> None:
     _call("decode_step", ctypes.byref(cfg), ctypes.byref(cache), layer, _p(q), _p(k), _p(v), _p(out),
           _p(workspace), ws_bytes, flags, stream)
+
+
+def hkv_decode_step_identify(cfg, cache, layer, q, k, v, out, label_out, workspace, ws_bytes,
+                             flags=0, stream=0) -> None:
+    _call("decode_step_identify", ctypes.byref(cfg), ctypes.byref(cache), layer, _p(q), _p(k), _p(v),
+          _p(out), _p(label_out), _p(workspace), ws_bytes, flags, stream)
 
 
 def hkv_evict(cfg, cache, layer, stream=0) -> None:

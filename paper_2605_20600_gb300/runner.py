@@ -14,7 +14,8 @@ from .engine import Engine, torch_dtype
 
 
 def generate(engine: Engine, provider, *, last_step: int | None = None, on_step=None,
-             before_compress=None, fused: bool = True, first_step: int = 0) -> None:
+             before_compress=None, fused: bool = True, first_step: int = 0,
+             identify: str | None = None) -> None:
     """Runs image tokens first_step..last_step (default N-1) for every layer.
 
     fused: per layer and step, hkv_evict when the update is due and then
@@ -22,7 +23,15 @@ def generate(engine: Engine, provider, *, last_step: int | None = None, on_step=
     on_step(t, out) receives out [L][S][H][D] (fp32, device) after step t.
     before_compress(engine) runs after grouping, before budgets and repack.
     first_step > 0 continues a generation (the prefill is skipped).
+    identify: "fused" decides the head types inside the grouping token's
+    decode step (fused path only; no n_h), "separate" runs
+    hkv_identify_heads after it (labels and n_h). Default: fused when the
+    path is fused.
     """
+    if identify is None:
+        identify = "fused" if fused else "separate"
+    if identify not in ("fused", "separate") or (identify == "fused" and not fused):
+        raise ValueError(f"identify={identify!r} with fused={fused}")
     cfg = engine.cfg
     L, S, H, D, C = cfg.n_layers, cfg.n_seqs, cfg.n_heads, cfg.head_dim, cfg.n_cond
     E = cfg.group_at
@@ -45,11 +54,14 @@ def generate(engine: Engine, provider, *, last_step: int | None = None, on_step=
             if fused:
                 if due:
                     engine.evict(layer)
-                engine.step(layer, q[layer], k[layer], v[layer], out[layer])
+                if t == E - 1 and identify == "fused":
+                    engine.step_identify(layer, q[layer], k[layer], v[layer], out[layer])
+                else:
+                    engine.step(layer, q[layer], k[layer], v[layer], out[layer])
             else:
                 engine.append(layer, q[layer], k[layer], v[layer])
                 engine.attend(layer, q[layer], out[layer])
-            if t == E - 1:
+            if t == E - 1 and identify == "separate":
                 engine.identify(layer, q[layer])
         if on_step is not None:
             on_step(t, out)

@@ -47,7 +47,7 @@ def fake_cache(H, **kw):
 
 def test_every_declared_symbol_is_exported(H):
     names = declared_functions()
-    assert len(names) == 15
+    assert len(names) == 16
     for n in names:
         assert hasattr(H.lib(), n), n
     assert set(names) >= {"hkv_identify_heads", "hkv_allocate_budgets", "hkv_append_evict",
@@ -132,6 +132,10 @@ def test_null_and_misaligned_arguments(H):
                                 0, ctypes.byref(cnt), None) == 1
     assert lib.hkv_export_state(ctypes.byref(cfg), ctypes.byref(c), 0, None, None, None, None, 16,
                                 -1, ctypes.byref(cnt), None) == 1
+    assert lib.hkv_decode_step_identify(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, 16, 16, None,
+                                        16, 1 << 30, 0, None) == 1
+    assert lib.hkv_decode_step_identify(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, 16, 16, 16,
+                                        16, 8, 0, None) == 3
     nopos = fake_cache(H, pos=None)
     assert lib.hkv_export_state(ctypes.byref(cfg), ctypes.byref(nopos), 0, None, None, None, None,
                                 16, 8, ctypes.byref(cnt), None) == 1
@@ -139,7 +143,7 @@ def test_null_and_misaligned_arguments(H):
 
 @pytest.mark.parametrize("name", ["decode_attention", "append_evict", "identify_heads",
                                   "allocate_budgets", "repack", "prefill", "init_dense", "check",
-                                  "decode_step", "evict", "export_state"])
+                                  "decode_step", "evict", "export_state", "decode_step_identify"])
 def test_fault_injection_returns_the_code(H, name, monkeypatch):
     cfg = tiny_cfg(H)
     c = fake_cache(H)
@@ -156,6 +160,8 @@ def test_fault_injection_returns_the_code(H, name, monkeypatch):
         "check": lambda: lib.hkv_check(ctypes.byref(c), None),
         "decode_step": lambda: lib.hkv_decode_step(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, 16, 16, 16, 1 << 30, 0, None),
         "evict": lambda: lib.hkv_evict(ctypes.byref(cfg), ctypes.byref(c), 0, None),
+        "decode_step_identify": lambda: lib.hkv_decode_step_identify(
+            ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, 16, 16, 16, 16, 1 << 30, 0, None),
         "export_state": lambda: lib.hkv_export_state(ctypes.byref(cfg), ctypes.byref(c), 0, None, None,
                                                      None, None, None, 0, None, None),
     }

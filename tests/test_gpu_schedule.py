@@ -63,7 +63,8 @@ def test_hand_worked_grid_on_gpu(fused):
                      for h in range(2)]
         outs[t] = out.cpu().numpy()[0, 0]
 
-    generate(eng, HandProvider(heads, c["n_cond"], "cuda"), on_step=on_step, fused=fused)
+    generate(eng, HandProvider(heads, c["n_cond"], "cuda"), on_step=on_step, fused=fused,
+             identify="separate")
     eng.check()
     labels, nh = eng.labels.cpu().numpy(), eng.n_h.cpu().numpy()
     hp = O.HeadParams(n_cond=c["n_cond"], n_image=c["n_image"], recent_w=c["recent_w"],
@@ -86,13 +87,37 @@ def test_hand_worked_grid_on_gpu(fused):
             assert np.abs(outs[t][h] - tr.outputs[t]).max() < 1e-5, (hd["name"], t)
 
 
-@pytest.mark.parametrize("fused", [True, False])
-def test_tiny_every_step_every_head(fused):
+def test_hand_worked_grid_fused_identification():
+    """The grouping step's decode with the head types decided in the same
+    pass gives the hand-worked labels (4x4 grid, D = 2, integer keys)."""
+    from paper_2605_20600_gb300 import hkv as H
+    from paper_2605_20600_gb300.engine import Engine
+    from paper_2605_20600_gb300.runner import generate
+    case, heads = load_hand()
+    c = case["config"]
+    cfg = H.make_config(n_layers=1, n_seqs=1, n_heads=2, head_dim=c["head_dim"], dtype="fp32",
+                        n_cond=c["n_cond"], n_image=c["n_image"], row_len=c["row_len"],
+                        recent_w=c["recent_w"], local_w=c["local_w"], period=c["period"],
+                        group_at=c["group_at"], global_budget=c["global_budget"], tau=c["tau"],
+                        r_s=c["r_s"])
+    eng = Engine(cfg, "cuda")
+    generate(eng, HandProvider(heads, c["n_cond"], "cuda"), last_step=c["group_at"] - 1,
+             fused=True, identify="fused")
+    eng.check()
+    labels = eng.labels.cpu().numpy()
+    for h, hd in enumerate(heads):
+        assert int(labels[h]) == hd["expected"]["label"], hd["name"]
+
+
+@pytest.mark.parametrize("fused,identify", [(True, "separate"), (False, "separate"),
+                                            (True, "fused")])
+def test_tiny_every_step_every_head(fused, identify):
     w = configs.TINY
     N = w.n_image
     heads = [(0, 0, h) for h in range(w.n_heads)]
     outs, poss, labels, nh, eng = run_gpu(w, out_steps=range(N), pos_steps=range(N),
-                                          pos_heads=[flat(w, *x) for x in heads], fused=fused)
+                                          pos_heads=[flat(w, *x) for x in heads], fused=fused,
+                                          identify=identify)
     lab = oracle_labels(w, [0], [0])
     ties = check_labels(w, labels, nh, lab, "tiny")
     assert not ties
@@ -116,20 +141,25 @@ def sampled_steps(w, rng, extra=12):
     return sorted(x for x in s if 0 <= x < N)
 
 
-REDUCED = [("lumina768", "1/4", True), ("lumina1024", "1/4", True), ("lumina1024", "1/6", True),
-           ("lumina1024", "1/8", True), ("llamagen_xl", "1/6", True), ("janus_pro_7b", "1/8", True),
-           ("lumina1024", "1/8", False), ("llamagen_xl", "1/6", False)]
+REDUCED = [("lumina768", "1/4", True, "separate"), ("lumina1024", "1/4", True, "separate"),
+           ("lumina1024", "1/6", True, "separate"), ("lumina1024", "1/8", True, "separate"),
+           ("llamagen_xl", "1/6", True, "separate"), ("janus_pro_7b", "1/8", True, "separate"),
+           ("lumina1024", "1/8", False, "separate"), ("llamagen_xl", "1/6", False, "separate"),
+           # the head types decided inside the grouping token's decode step
+           ("lumina1024", "1/4", True, "fused"), ("llamagen_xl", "1/6", True, "fused"),
+           ("janus_pro_7b", "1/8", True, "fused")]
 
 
-@pytest.mark.parametrize("name,rho,fused", REDUCED)
-def test_model_shapes_two_layers_two_seqs(name, rho, fused):
+@pytest.mark.parametrize("name,rho,fused,identify", REDUCED)
+def test_model_shapes_two_layers_two_seqs(name, rho, fused, identify):
     from fractions import Fraction
     w = configs.ALL[name].with_(n_layers=2, n_seqs=2, rho=Fraction(rho))
     rng = np.random.default_rng(42)
     steps = sampled_steps(w, rng)
     heads = [(s, l, h) for l in range(w.n_layers) for s in range(w.n_seqs) for h in range(w.n_heads)]
     outs, poss, labels, nh, eng = run_gpu(w, out_steps=steps, pos_steps=steps,
-                                          pos_heads=[flat(w, *x) for x in heads], fused=fused)
+                                          pos_heads=[flat(w, *x) for x in heads], fused=fused,
+                                          identify=identify)
     lab = oracle_labels(w, range(w.n_layers), range(w.n_seqs))
     ties = check_labels(w, labels, nh, lab, name)
     assert len(ties) <= 2, ties
