@@ -31,6 +31,10 @@ namespace hkv {
 namespace {
 
 constexpr int NT = kCacheThreads;
+// update kernels resident per SM that the register budget allows (48
+// registers a thread, no spills): a layer of many short heads (one CTA each)
+// then runs in fewer waves; shared memory may allow fewer
+constexpr int kUpdCtasPerSm = 5;
 
 // Phase timestamps per head of the update for latency studies; compiled out
 // by default.
@@ -81,20 +85,29 @@ struct UpdSmem {
   int *aux;                  // [max_len] class, then keep flag, then rank
   float *qbar;               // [D]
   int *hist;                 // [512]
+  int stage_rows;            // rows a warp stages per pass of the score phase
 };
 
+// Rows a warp stages per pass of the score phase: 32, or fewer when every
+// warp's share of the longest segment is smaller (short segments then leave
+// room for more CTAs per SM).
+__host__ __device__ constexpr int stage_rows(int max_len) {
+  return max_len >= NT ? 32 : (max_len + NT / 32 - 1) / (NT / 32) < 1 ? 1 : (max_len + NT / 32 - 1) / (NT / 32);
+}
+
 // the query ring (P rows of es-byte elements); after q-bar it is the score
-// stage: NT/32 warps x 32 rows of D * es + 16 bytes
-__host__ __device__ constexpr size_t ring_bytes(int P, int D, int es) {
-  return (size_t)P * D * es > (size_t)(NT / 32) * 32 * (D * es + 16)
+// stage: NT/32 warps x stage_rows rows of D * es + 16 bytes
+__host__ __device__ constexpr size_t ring_bytes(int P, int D, int es, int max_len) {
+  return (size_t)P * D * es > (size_t)(NT / 32) * stage_rows(max_len) * (D * es + 16)
              ? (size_t)P * D * es
-             : (size_t)(NT / 32) * 32 * (D * es + 16);
+             : (size_t)(NT / 32) * stage_rows(max_len) * (D * es + 16);
 }
 
 __device__ __forceinline__ UpdSmem carve(unsigned char *dyn, int max_len, int D, int P, int es) {
   UpdSmem u;
   u.ring = dyn;
-  u.keys = reinterpret_cast<unsigned long long *>(dyn + ring_bytes(P, D, es));
+  u.stage_rows = stage_rows(max_len);
+  u.keys = reinterpret_cast<unsigned long long *>(dyn + ring_bytes(P, D, es, max_len));
   u.ps = reinterpret_cast<int *>(u.keys + max_len);
   u.aux = u.ps + max_len;
   u.qbar = reinterpret_cast<float *>(u.aux + max_len);
@@ -250,9 +263,10 @@ __device__ int select_evictions(const SegRef &sg, int label, const MethodArgs &m
     // sums its row in the fixed order.
     constexpr int RS = LPR + 1;  // row stride in 16-byte pieces
     const int warp = tid >> 5, lane = tid & 31;
-    unsigned char *stage = u.ring + (size_t)warp * 32 * RS * 16;
-    for (int base = warp * 32; base < sg.len; base += (NT / 32) * 32) {
-      const int nrows = sg.len - base < 32 ? sg.len - base : 32;
+    const int SR = u.stage_rows;
+    unsigned char *stage = u.ring + (size_t)warp * SR * RS * 16;
+    for (int base = warp * SR; base < sg.len; base += (NT / 32) * SR) {
+      const int nrows = sg.len - base < SR ? sg.len - base : SR;
       for (int w = lane; w < nrows * LPR; w += 32) {
         const int rr = w / LPR, pc = w % LPR;
         cp_async16(stage + (rr * RS + pc) * 16, sg.sk + (size_t)(base + rr) * RB + pc * 16);
@@ -418,7 +432,7 @@ __device__ int update_in_place(const SegRef &sg, int label, const MethodArgs &m,
 }
 
 template <int D, typename T>
-__global__ void __launch_bounds__(NT)
+__global__ void __launch_bounds__(NT, kUpdCtasPerSm)
     evict_kernel(const CacheArgs c, const MethodArgs m, int layer_base, int max_len) {
   constexpr int RB = D * (int)sizeof(T);
   extern __shared__ __align__(16) unsigned char dyn[];
@@ -456,7 +470,7 @@ __global__ void __launch_bounds__(NT)
 }
 
 template <int D, typename T>
-__global__ void __launch_bounds__(NT)
+__global__ void __launch_bounds__(NT, kUpdCtasPerSm)
     append_evict_kernel(const CacheArgs c, const MethodArgs m, int layer_base, const void *q,
                         const void *k, const void *v, int max_len) {
   constexpr int RB = D * (int)sizeof(T);
@@ -518,7 +532,7 @@ __global__ void __launch_bounds__(NT)
 }
 
 template <int D, typename T>
-__global__ void __launch_bounds__(NT)
+__global__ void __launch_bounds__(NT, kUpdCtasPerSm)
     repack_kernel(const CacheArgs dn, const CacheArgs rg, const MethodArgs m, int layer_base,
                   int max_len) {
   constexpr int RB = D * (int)sizeof(T);
@@ -830,17 +844,28 @@ cudaError_t pdl_launch(void (*kernel)(KArgs...), int grid, int block, size_t sme
   return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
 
+size_t smem_of(int max_len, int D, int P, int es) {
+  // the query ring / score stage; keys (8 B), positions (4 B), class/flag/
+  // rank (4 B) per row; q-bar; two 256-bin histograms
+  return ring_bytes(P, D, es, max_len) + (size_t)max_len * 16 + (size_t)D * 4 + 512 * 4 + 64;
+}
+
+// the longest segment a launch with `smem` bytes takes (the inverse of
+// smem_of, which grows with max_len)
 int max_len_of(size_t smem, int D, int P, int es) {
-  return (int)((smem - ring_bytes(P, D, es) - (size_t)D * 4 - 512 * 4 - 64) / 16);
+  int lo = 0, hi = 1 << 20;
+  while (lo < hi) {
+    const int mid = lo + (hi - lo + 1) / 2;
+    if (smem_of(mid, D, P, es) <= smem) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
 }
 
 }  // namespace
 
 size_t update_smem_bytes(int max_len, int D, int P, int dtype) {
-  // the query ring / score stage; keys (8 B), positions (4 B), class/flag/
-  // rank (4 B) per row; q-bar; two 256-bin histograms
-  return ring_bytes(P, D, dtype == HKV_BF16 ? 2 : 4) + (size_t)max_len * 16 + (size_t)D * 4 +
-         512 * 4 + 64;
+  return smem_of(max_len, D, P, dtype == HKV_BF16 ? 2 : 4);
 }
 
 cudaError_t update_prepare(int D, int dtype, size_t smem) {
