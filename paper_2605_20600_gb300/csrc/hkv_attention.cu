@@ -58,14 +58,29 @@
 namespace hkv {
 namespace {
 
-// Tuning knobs (compile time): bytes of K per pipeline stage, stages, a cap
+// Tuning knobs (compile time), per head dimension: consumer warps, bytes of
+// K per pipeline stage and stages (measured: rows of 256 B stream best with 7
+// consumer warps over 10.5 KB tiles in 4 stages; rows of 128 B, whose short
+// heads come many to a CTA, with 8 warps over 8 KB tiles in 5 stages); a cap
 // on resident CTAs per SM used to size the grid, and tiles loaded before the
 // wait for the previous kernel (prefetch).
-#ifndef HKV_ATTN_TILE_BYTES
-#define HKV_ATTN_TILE_BYTES 10752
+#ifndef HKV_ATTN_CW_D128
+#define HKV_ATTN_CW_D128 7
 #endif
-#ifndef HKV_ATTN_STAGES
-#define HKV_ATTN_STAGES 4
+#ifndef HKV_ATTN_TILE_BYTES_D128
+#define HKV_ATTN_TILE_BYTES_D128 10752
+#endif
+#ifndef HKV_ATTN_STAGES_D128
+#define HKV_ATTN_STAGES_D128 4
+#endif
+#ifndef HKV_ATTN_CW_D64
+#define HKV_ATTN_CW_D64 8
+#endif
+#ifndef HKV_ATTN_TILE_BYTES_D64
+#define HKV_ATTN_TILE_BYTES_D64 8192
+#endif
+#ifndef HKV_ATTN_STAGES_D64
+#define HKV_ATTN_STAGES_D64 5
 #endif
 #ifndef HKV_ATTN_MAX_CTAS_PER_SM
 #define HKV_ATTN_MAX_CTAS_PER_SM 2
@@ -74,9 +89,6 @@ namespace {
 #define HKV_ATTN_PRE_TILES 3
 #endif
 
-static_assert(HKV_ATTN_PRE_TILES >= 0 && HKV_ATTN_PRE_TILES <= HKV_ATTN_STAGES, "prefetch depth");
-
-constexpr int kCW = kAttnConsumerWarps;
 
 // Phase timestamps and counters per CTA for latency studies; compiled out by
 // default.
@@ -106,20 +118,24 @@ __device__ unsigned long long *g_trace = nullptr;  // [layer][kAttnMaxGrid][32],
 
 template <int D, typename T>
 struct AttnShape {
+  static constexpr int kCW = D == 64 ? HKV_ATTN_CW_D64 : HKV_ATTN_CW_D128;  // consumer warps
+  static constexpr int kThreads = 32 * (kCW + 2);  // + producer + epilogue
   static constexpr int kES = sizeof(T);
   static constexpr int kRB = D * kES;             // bytes per token row
   static constexpr int kLPR = kRB / 16;           // lanes per row
   static constexpr int kEPL = 16 / kES;           // elements per lane
   static constexpr int kRPW = 32 / kLPR;          // rows per warp step
-  static constexpr int kTT = HKV_ATTN_TILE_BYTES / kRB;   // rows per tile
+  static constexpr int kTT =                      // rows per tile
+      (D == 64 ? HKV_ATTN_TILE_BYTES_D64 : HKV_ATTN_TILE_BYTES_D128) / kRB;
   static constexpr int kSteps = kTT / (kCW * kRPW);
-  static constexpr int kNS = HKV_ATTN_STAGES;     // pipeline stages
+  static constexpr int kNS = D == 64 ? HKV_ATTN_STAGES_D64 : HKV_ATTN_STAGES_D128;  // stages
   static constexpr int kStageBytes = 2 * kTT * kRB + kRB;   // K, V, q row
   static constexpr int kMinChunk = 2 * kTT;       // fewest indices per CTA range
   static_assert(kLPR >= 1 && kLPR <= 32 && 32 % kLPR == 0, "row mapping");
   static_assert(kSteps >= 1 && kTT % (kCW * kRPW) == 0, "tile mapping");
   static_assert(D <= kCW * 32 && D % 32 == 0, "output channels");
   static_assert(kStageBytes % 16 == 0, "TMA alignment");
+  static_assert(HKV_ATTN_PRE_TILES >= 0 && HKV_ATTN_PRE_TILES <= kNS, "prefetch depth");
 };
 
 constexpr int kTable = 32;  // heads of a CTA's range kept in smem
@@ -316,8 +332,9 @@ struct Pending {
 };
 
 template <int D, typename T, bool FUSED, bool IDENT>
-__global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnArgs p) {
+__global__ void __launch_bounds__(AttnShape<D, T>::kThreads, 2) attn_kernel(const AttnArgs p) {
   using S = AttnShape<D, T>;
+  constexpr int kCW = S::kCW, kAttnThreads = S::kThreads;
   constexpr int LPR = S::kLPR, EPL = S::kEPL, RPW = S::kRPW, TT = S::kTT;
   constexpr int RB = S::kRB, NS = S::kNS;
 
@@ -1036,7 +1053,7 @@ cudaError_t prepare_t(int *ctas) {
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas, attn_kernel<D, T, F, I>,
-                                                       kAttnThreads, smem);
+                                                       AttnShape<D, T>::kThreads, smem);
 }
 
 template <int D, typename T>
@@ -1070,7 +1087,8 @@ cudaError_t launch_pdl(K kernel, int grid, int threads, size_t smem, const AttnA
 
 template <int D, typename T, bool F, bool I>
 cudaError_t launch_both(const AttnArgs &a, int grid, cudaStream_t s) {
-  cudaError_t e = launch_pdl(attn_kernel<D, T, F, I>, grid, kAttnThreads, smem_bytes<D, T>(), a, s);
+  cudaError_t e = launch_pdl(attn_kernel<D, T, F, I>, grid, AttnShape<D, T>::kThreads,
+                             smem_bytes<D, T>(), a, s);
   if (e != cudaSuccess) return e;
   // a warp for every 32 heads and for every CTA boundary
   int warps = (a.nheads + 31) / 32;

@@ -59,13 +59,8 @@ struct AttnArgs {
   float tau;
 };
 
-// decode attention CTA: one producer warp (TMA), consumer warps, one
-// epilogue warp (merges, outputs, partial results)
-#ifndef HKV_ATTN_CONSUMER_WARPS
-#define HKV_ATTN_CONSUMER_WARPS 7
-#endif
-constexpr int kAttnConsumerWarps = HKV_ATTN_CONSUMER_WARPS;
-constexpr int kAttnThreads = 32 * (kAttnConsumerWarps + 2);  // + producer + epilogue
+// decode attention CTAs: one producer warp (TMA), consumer warps, one
+// epilogue warp (merges, outputs, partial results); at most kAttnMaxGrid
 constexpr int kAttnMaxGrid = 4096;
 // finishing kernel: one-warp CTAs, each for 32 heads' counters and one CTA
 // boundary's split head; at 64 registers a thread, seven fit on an SM beside
