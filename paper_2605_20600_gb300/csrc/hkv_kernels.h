@@ -62,10 +62,14 @@ struct AttnArgs {
 // decode attention CTAs: one producer warp (TMA), consumer warps, one
 // epilogue warp (merges, outputs, partial results); at most kAttnMaxGrid
 constexpr int kAttnMaxGrid = 4096;
-// finishing kernel: one-warp CTAs, each for 32 heads' counters and one CTA
-// boundary's split head; at 64 registers a thread, seven fit on an SM beside
-// two attention CTAs (which leave ~14.8K of its 64K registers)
-constexpr int kFinishThreads = 32;
+// finishing kernel: CTAs of two warps, each warp for 32 heads' counters and
+// one CTA boundary's split head; at 64 registers a thread, two such CTAs fit
+// on an SM beside two attention CTAs (measured: one-warp CTAs 1 % slower,
+// four-warp CTAs, one per SM, 10 % slower)
+#ifndef HKV_FINISH_THREADS
+#define HKV_FINISH_THREADS 64
+#endif
+constexpr int kFinishThreads = HKV_FINISH_THREADS;
 constexpr int kFinishRegs = 64;
 // floats of one split-K partial result: D accumulators, the running maximum
 // and the sum, padded to 16 bytes for vector access
