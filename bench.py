@@ -284,10 +284,13 @@ def run_ours(args):
                          f"mean {per_head * 1e3:.1f} ms per head-period, projected to all heads "
                          f"on {workers} processes"}
 
+    redistribute = args.budget == "redistribute"
     cfg = H.make_config(n_layers=L, n_seqs=S, n_heads=Hh, head_dim=D, dtype=w.dtype,
                         n_cond=w.n_cond, n_image=w.n_image, row_len=w.row_len,
                         recent_w=w.recent_w, local_w=w.w_loc, period=P, group_at=w.group_at,
-                        rho=w.rho, tau=w.tau, r_s=w.r_s)
+                        rho=w.rho, tau=w.tau, r_s=w.r_s,
+                        budget_mode=H.HKV_BUDGET_REDISTRIBUTE if redistribute else
+                        H.HKV_BUDGET_PAPER)
     eng = Engine(cfg, dev)
     synth = DeviceSynth(w, dev)
     generate(eng, synth, last_step=t0 - 1)      # dense phase, grouping, compression, decode
@@ -443,7 +446,9 @@ def run_ours(args):
             "metric": METRIC, "value": value, "unit": "image tokens/s", "n_gpus": world,
             "steps": K, "warmup": W, "ms_per_step": ms / K, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-            "config": bench_config(w, world),
+            "config": {**bench_config(w, world),
+                       **({"budget": "redistributed (aggregate-preserving), arena "
+                                     f"{eng.total_tokens} tokens"} if redistribute else {})},
             "global_head_fraction": float((labels == 1).mean()),
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak,
@@ -691,6 +696,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--strategies", action="store_true",
                     help="compare decode attention with the padding and per-group strategies")
+    ap.add_argument("--budget", default="paper", choices=["paper", "redistribute"],
+                    help="budget rule: the paper's, or local heads' unused tokens to global heads")
     ap.add_argument("--grouping", action="store_true",
                     help="time the grouping step with identification separate and fused")
     args = ap.parse_args()

@@ -86,6 +86,9 @@ enum { HKV_LOCAL = 0, HKV_GLOBAL = 1, HKV_DENSE = 255 };
  *                (Appendix, More Implementation Details)
  *  global_budget B_g = floor(rho * N) image tokens kept by a global head
  *                (Sec. 5.1); must be >= recent_w
+ *  budget_mode   HKV_BUDGET_PAPER (0) or HKV_BUDGET_REDISTRIBUTE (1): the
+ *                rule hkv_allocate_budgets applies (below); the update calls
+ *                size their scratch for the longest segment it allows
  *  tau           accumulation threshold, 0.9 in the paper (Step 2)
  *  r_s           long/near split ratio, 0.5 in the paper (Eq. 5)
  */
@@ -95,9 +98,21 @@ typedef struct {
   int32_t n_cond, n_image, row_len;
   int32_t recent_w, local_w, period, group_at;
   int32_t global_budget;
-  int32_t reserved;
+  int32_t budget_mode;
   double tau, r_s;
 } hkv_config;
+
+/* budget rules (hkv_config.budget_mode) */
+enum {
+  HKV_BUDGET_PAPER = 0,      /* Sec. 5.1: B_g (global) or w (local) */
+  /* not in the paper, aggregate-preserving: within each (sequence, layer)
+   * group of H heads the (H - n_g)(B_g - w) image tokens the local heads do
+   * not use go to its n_g global heads in equal shares, the remainder one
+   * token each to the global heads of lowest head index; the group then
+   * keeps H * B_g image tokens, as if every head kept B_g. A group without
+   * global heads keeps the paper's budgets. */
+  HKV_BUDGET_REDISTRIBUTE = 1
+};
 
 /*
  * A KV cache: one arena holding every head's segment back to back.
@@ -143,7 +158,8 @@ const char *hkv_status_str(hkv_status s);
 
 /* Checks a config: sizes positive, head_dim in {64, 128}, dtype known,
  * recent_w <= global_budget <= n_image, period <= group_at <= n_image,
- * 0 < tau <= 1, 0 <= r_s <= 1. Host only. */
+ * 0 < tau <= 1, 0 <= r_s <= 1, budget_mode one of HKV_BUDGET_*. Host
+ * only. */
 hkv_status hkv_validate_config(const hkv_config *cfg);
 
 /* Bytes of device workspace hkv_decode_attention and hkv_decode_step need
@@ -170,7 +186,8 @@ hkv_status hkv_prefill(const hkv_config *cfg, const hkv_cache *cache, int layer,
  * Sec. 3; periodic update, Sec. 4):
  *  1. for a compressed head whose buffer holds P tokens, run the update
  *     first: a local head keeps its conditioning and newest w tokens
- *     (Eq. 3); a global head whose history exceeds B_g - w evicts the excess
+ *     (Eq. 3); a global head whose history exceeds its budget (cap - C - P
+ *     - w: B_g - w under the paper's budgets) evicts the excess
  *     by STE (Eqs. 4-6: long/near split by r_s, scores from the P buffered
  *     queries, the lowest floor(M/2) / M - floor(M/2) of each subset
  *     evicted, older first on equal score); the segment shrinks in place by
@@ -270,20 +287,24 @@ hkv_status hkv_identify_heads(const hkv_config *cfg, const hkv_cache *cache, int
                               hkv_stream_t stream);
 
 /* Sec. 5.1 budgets for all L*S*H heads from their labels: budget = B_g
- * (global) or w (local) image tokens, cap = C + budget + P, off = exclusive
- * prefix sum of cap (tokens). Writes budget, cap, off (device) and the
+ * (global) or w (local) image tokens (or the redistributed budgets, per
+ * cfg->budget_mode), cap = C + budget + P, off = exclusive prefix sum of cap
+ * (tokens). The periodic update reads each global head's history budget
+ * from its capacity (cap - C - P - w). Writes budget, cap, off (device) and the
  * arena size in tokens to *total_tokens (host); synchronises the stream.
  * A label other than HKV_LOCAL / HKV_GLOBAL yields HKV_ERR_STATE. */
 hkv_status hkv_allocate_budgets(const hkv_config *cfg, const uint8_t *label, int32_t *budget,
                                 int32_t *cap, int64_t *off, int64_t *total_tokens,
                                 hkv_stream_t stream);
 
+
 /* Head-aware compression of one layer after grouping (Step 3): copies
  * every head of the dense cache into its segment of the ragged cache (whose
  * off, cap and label arrays the caller filled from hkv_allocate_budgets and
  * hkv_identify_heads) and applies the first update there: local heads keep
  * the conditioning and newest w tokens; global heads keep a history of at
- * most B_g - w tokens chosen by STE with the P latest queries. Sets len,
+ * most cap - C - P - w tokens (B_g - w under the paper's budgets) chosen by
+ * STE with the P latest queries. Sets len,
  * nbuf = 0 and ntok on the ragged side. The two caches share the qbuf ring
  * layout; the ragged cache's qbuf must be the dense cache's qbuf. */
 hkv_status hkv_repack(const hkv_config *cfg, const hkv_cache *dense, const hkv_cache *ragged,

@@ -117,12 +117,38 @@ def head_budget(label: int, B_g: int, w: int) -> int:
     return B_g if label == GLOBAL else w
 
 
-def arena_layout(labels, n_cond: int, B_g: int, w: int, P: int):
+def redistributed_budgets(group_labels, B_g: int, w: int) -> np.ndarray:
+    """Budget variant (not in the paper; aggregate-preserving): within one
+    (sequence, layer) group of H heads, the image tokens the local heads do
+    not use, (H - n_g)(B_g - w), go to its n_g global heads in equal shares,
+    the remainder one token each to the global heads of lowest index, so the
+    group keeps H * B_g image tokens as if every head had B_g. A group
+    without global heads keeps the paper's budgets."""
+    lab = np.asarray(group_labels).reshape(-1)
+    glob = np.flatnonzero(lab == GLOBAL)
+    budget = np.array([head_budget(int(x), B_g, w) for x in lab], dtype=np.int64)
+    if glob.size == 0:
+        return budget
+    extra = (lab.size - glob.size) * (B_g - w)
+    share, rem = divmod(extra, glob.size)
+    budget[glob] += share
+    budget[glob[:rem]] += 1
+    return budget
+
+
+def arena_layout(labels, n_cond: int, B_g: int, w: int, P: int, group: int = 0):
     """Per-head budget, capacity (C + budget + P buffered tokens) and the
     exclusive prefix sum of capacities (segment offsets, in tokens) for heads
-    in the given order. Returns (budget, cap, off, total)."""
+    in the given order. group > 0: the redistributed budgets over
+    consecutive groups of that many heads (one (sequence, layer) each).
+    Returns (budget, cap, off, total)."""
     labels = np.asarray(labels).reshape(-1)
-    budget = np.array([head_budget(int(x), B_g, w) for x in labels], dtype=np.int64)
+    if group > 0:
+        budget = np.concatenate([redistributed_budgets(labels[i: i + group], B_g, w)
+                                 for i in range(0, labels.size, group)]) if labels.size else \
+            np.zeros(0, np.int64)
+    else:
+        budget = np.array([head_budget(int(x), B_g, w) for x in labels], dtype=np.int64)
     cap = n_cond + budget + P
     off = np.zeros_like(cap)
     if cap.size:

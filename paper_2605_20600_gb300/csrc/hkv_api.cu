@@ -123,7 +123,6 @@ MethodArgs method_args(const hkv_config *cfg) {
   m.w = cfg->recent_w;
   m.w_loc = cfg->local_w;
   m.P = cfg->period;
-  m.hist_budget = cfg->global_budget - cfg->recent_w;
   m.r_s = cfg->r_s;
   m.tau = (float)cfg->tau;
   return m;
@@ -133,9 +132,18 @@ int heads_per_layer(const hkv_config *c) { return c->n_seqs * c->n_heads; }
 
 // longest segment any call may see: a dense head (C + E) or a compressed
 // global head right before its update (C + B_g + P)
+// the longest segment the config allows: the dense cache at grouping, or a
+// global head's C + budget + P tokens (never more than C + N); a
+// redistributed budget reaches B_g + (H - 1)(B_g - w) for a group of one
+// global head
 int max_segment(const hkv_config *c) {
   const int a = c->n_cond + c->group_at;
-  const int b = c->n_cond + c->global_budget + c->period;
+  long long bud = c->global_budget;
+  if (c->budget_mode == HKV_BUDGET_REDISTRIBUTE)
+    bud += (long long)(c->n_heads - 1) * (c->global_budget - c->recent_w);
+  long long kept = bud + c->period;
+  if (kept > c->n_image) kept = c->n_image;
+  const int b = c->n_cond + (int)kept;
   return a > b ? a : b;
 }
 
@@ -244,6 +252,11 @@ hkv_status hkv_validate_config(const hkv_config *c) {
   if ((long long)c->n_cond + c->n_image + c->period > (1ll << 24)) return HKV_ERR_SHAPE;
   if (!(c->tau > 0.0 && c->tau <= 1.0) || !(c->r_s >= 0.0 && c->r_s <= 1.0))
     return HKV_ERR_INVALID_ARG;
+  if (c->budget_mode != HKV_BUDGET_PAPER && c->budget_mode != HKV_BUDGET_REDISTRIBUTE)
+    return HKV_ERR_INVALID_ARG;
+  // a capacity (C + budget + P) stays an int32
+  if ((long long)c->n_cond + (long long)c->n_heads * c->global_budget + c->period > 0x7fffffffLL)
+    return HKV_ERR_SHAPE;
   return HKV_OK;
 }
 
@@ -400,7 +413,9 @@ hkv_status hkv_allocate_budgets(const hkv_config *cfg, const uint8_t *label, int
   const int n = cfg->n_layers * heads_per_layer(cfg);
   cudaStream_t s = (cudaStream_t)stream;
   if (launch_budgets(label, budget, cap, off, n, cfg->n_cond, cfg->global_budget, cfg->recent_w,
-                     cfg->period, s) != cudaSuccess)
+                     cfg->period,
+                     cfg->budget_mode == HKV_BUDGET_REDISTRIBUTE ? cfg->n_heads : 0,
+                     s) != cudaSuccess)
     return HKV_ERR_CUDA;
   int64_t last_off = 0;
   int32_t last_cap = 0;

@@ -99,7 +99,7 @@ struct CacheArgs {
 };
 
 struct MethodArgs {
-  int C, w, w_loc, P, hist_budget;  // hist_budget = B_g - w
+  int C, w, w_loc, P;  // a global head's history budget comes from its capacity
   double r_s;
   float tau;
 };
@@ -126,7 +126,8 @@ cudaError_t launch_init_dense(const CacheArgs &c, int nheads_total, int seg_toke
 cudaError_t launch_identify(const CacheArgs &c, const MethodArgs &m, int layer_base, int nheads,
                             const void *q, uint8_t *label_out, int32_t *nh_out, int D, int dtype,
                             int max_len, cudaStream_t s);
+// group > 0: the aggregate-preserving budgets over groups of that many heads
 cudaError_t launch_budgets(const uint8_t *label, int32_t *budget, int32_t *cap, int64_t *off,
-                           int n, int C, int B_g, int w, int P, cudaStream_t s);
+                           int n, int C, int B_g, int w, int P, int group, cudaStream_t s);
 
 }  // namespace hkv

@@ -212,9 +212,12 @@ __device__ int select_evictions(const SegRef &sg, int label, const MethodArgs &m
   }
   const int NH = block_sum(nh, sh);  // history candidates (Eq. 2)
   HKV_UTRACE(1);
+  // the head's history budget, B_g - w with the paper's budgets, from the
+  // capacity its segment was given (C + budget + P)
+  const int hist_budget = sg.dst_cap - C - m.P - m.w > 0 ? sg.dst_cap - C - m.P - m.w : 0;
   int M = 0;
   if (label == HKV_LOCAL) M = NH;    // Eq. 3: no history
-  else if (NH > m.hist_budget) M = NH - m.hist_budget;
+  else if (NH > hist_budget) M = NH - hist_budget;
 
   if (label == HKV_GLOBAL && M > 0) {
     // Eq. 5: the floor(NH r_s) oldest history tokens are long-range
@@ -737,8 +740,13 @@ __global__ void __launch_bounds__(NT)
   }
 }
 
+// Sec. 5.1 budgets (group = 0), or the aggregate-preserving variant over
+// consecutive groups of `group` heads, one (sequence, layer) each: the
+// (group - n_g)(B_g - w) tokens the local heads leave go to the group's n_g
+// global heads in equal shares, the remainder one each to the global heads
+// of lowest index.
 __global__ void budgets_kernel(const uint8_t *label, int32_t *budget, int32_t *cap, int64_t *off,
-                               int n, int C, int B_g, int w, int P) {
+                               int n, int C, int B_g, int w, int P, int group) {
   __shared__ long long scratch[33];
   pdl_wait();
   pdl_launch_dependents();
@@ -753,6 +761,17 @@ __global__ void budgets_kernel(const uint8_t *label, int32_t *budget, int32_t *c
       if (lb == HKV_GLOBAL) bg = B_g;
       else if (lb == HKV_LOCAL) bg = w;
       else bad = 1;
+      if (group > 0 && lb == HKV_GLOBAL) {
+        const int g0 = i / group * group;
+        int ng = 0, rank = 0;
+        for (int j = g0; j < g0 + group && j < n; ++j) {
+          const bool gl = label[j] == HKV_GLOBAL;
+          ng += gl;
+          rank += gl && j < i;
+        }
+        const long long extra = (long long)(group - ng) * (B_g - w);
+        bg += (int)(extra / ng) + (rank < extra % ng ? 1 : 0);
+      }
       cp = (long long)C + bg + P;
       budget[i] = bg;
       cap[i] = (int32_t)cp;
@@ -929,8 +948,8 @@ cudaError_t launch_identify(const CacheArgs &c, const MethodArgs &m, int layer_b
 }
 
 cudaError_t launch_budgets(const uint8_t *label, int32_t *budget, int32_t *cap, int64_t *off,
-                           int n, int C, int B_g, int w, int P, cudaStream_t s) {
-  return pdl_launch(budgets_kernel, 1, 1024, 0, s, label, budget, cap, off, n, C, B_g, w, P);
+                           int n, int C, int B_g, int w, int P, int group, cudaStream_t s) {
+  return pdl_launch(budgets_kernel, 1, 1024, 0, s, label, budget, cap, off, n, C, B_g, w, P, group);
 }
 
 }  // namespace hkv

@@ -2,6 +2,7 @@
 the C-ABI with snapshots, oracle runs of sampled heads in a spawn pool."""
 from __future__ import annotations
 
+import dataclasses
 import multiprocessing as mp
 import os
 
@@ -11,11 +12,12 @@ from oracle import headkv as O
 from synth import configs, gen
 
 
-def cfg_of(H, w: configs.Workload):
+def cfg_of(H, w: configs.Workload, budget_mode=0):
     return H.make_config(n_layers=w.n_layers, n_seqs=w.n_seqs, n_heads=w.n_heads,
                          head_dim=w.head_dim, dtype=w.dtype, n_cond=w.n_cond, n_image=w.n_image,
                          row_len=w.row_len, recent_w=w.recent_w, local_w=w.w_loc,
-                         period=w.period, group_at=w.group_at, rho=w.rho, tau=w.tau, r_s=w.r_s)
+                         period=w.period, group_at=w.group_at, rho=w.rho, tau=w.tau, r_s=w.r_s,
+                         budget_mode=budget_mode)
 
 
 def flat(w, s, l, h):
@@ -23,7 +25,7 @@ def flat(w, s, l, h):
 
 
 def run_gpu(w, *, out_steps=(), pos_steps=(), pos_heads=(), last_step=None, fused=True,
-            out_heads=None, identify="separate"):
+            out_heads=None, identify="separate", budget_mode=0):
     """One generation on the GPU. Returns outputs {t: [L,S,H,D] fp32, or
     {(s, l, h): [D]} for out_heads}, positions {t: {flat head: sorted
     positions}}, labels, n_h (None when the identification is fused into
@@ -34,7 +36,7 @@ def run_gpu(w, *, out_steps=(), pos_steps=(), pos_heads=(), last_step=None, fuse
     from paper_2605_20600_gb300.runner import generate
     from synth.gpu import DeviceSynth
 
-    eng = Engine(cfg_of(H, w), "cuda")
+    eng = Engine(cfg_of(H, w, budget_mode), "cuda")
     out_steps, pos_steps = set(out_steps), set(pos_steps)
     outs, poss = {}, {}
 
@@ -64,19 +66,24 @@ def run_gpu(w, *, out_steps=(), pos_steps=(), pos_heads=(), last_step=None, fuse
 
 
 def _oracle_job(args):
-    w, s, l, h, label, record, record_pos = args
+    w, s, l, h, label, record, record_pos, budget = args
     pe, cq = gen.pe_table(w), gen.q_coef(w)
     hi = gen.HeadInputs(w, s, l, h, pe, cq)
     hp = O.HeadParams.of(w)
+    if budget is not None and label == O.GLOBAL:   # a per-head budget (redistributed)
+        hp = dataclasses.replace(hp, global_budget=budget)
     tr = O.run_head(hp, hi.q, hi.k, hi.v, label=label, record=record, record_pos=record_pos)
     return (s, l, h), tr
 
 
-def oracle_heads(w, heads, labels=None, record=(), record_pos=()):
+def oracle_heads(w, heads, labels=None, record=(), record_pos=(), budgets=None):
     """Oracle traces of the given (s, l, h) heads; labels (flat array) are
-    injected when given. Runs in a spawn pool (safe after CUDA init)."""
+    injected when given, and so are per-head image-token budgets (flat
+    array, used for global heads). Runs in a spawn pool (safe after CUDA
+    init)."""
     jobs = [(w, s, l, h, None if labels is None else int(labels[flat(w, s, l, h)]),
-             tuple(record), tuple(record_pos)) for (s, l, h) in heads]
+             tuple(record), tuple(record_pos),
+             None if budgets is None else int(budgets[flat(w, s, l, h)])) for (s, l, h) in heads]
     if len(jobs) <= 2:
         return dict(map(_oracle_job, jobs))
     n = min(len(jobs), os.cpu_count() or 1, 16)

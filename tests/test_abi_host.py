@@ -68,7 +68,7 @@ def test_status_strings(H):
 @pytest.mark.parametrize("change,code", [
     (dict(head_dim=96), 2), (dict(dtype=5), 1), (dict(period=32), 2), (dict(global_budget=8), 2),
     (dict(global_budget=65), 2), (dict(group_at=65), 2), (dict(n_seqs=0), 2), (dict(tau=0.0), 1),
-    (dict(r_s=1.5), 1),
+    (dict(r_s=1.5), 1), (dict(budget_mode=2), 1),
 ])
 def test_validate_config_rejects(H, change, code):
     cfg = tiny_cfg(H)

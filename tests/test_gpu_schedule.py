@@ -233,3 +233,62 @@ def test_export_state_capacity():
     assert np.array_equal(big, cc.pos.cpu().numpy()[np.add.outer(np.arange(0, 320, 40), np.arange(3)).ravel()])
     cc.len[2] = -1
     assert f(*args, None, 0, ctypes.byref(cnt), None) == H.HKV_ERR_BOUNDS
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_budgets_match_the_oracle(mode):
+    """hkv_allocate_budgets against the oracle's arena layout, both budget
+    rules (cfg.budget_mode), on the Lumina-1024 head count with random labels (one group all
+    local, one all global)."""
+    import torch
+    from paper_2605_20600_gb300 import hkv as H
+    from _gpu_util import cfg_of
+    w = configs.LUMINA_1024
+    cfg = cfg_of(H, w, mode)
+    n = w.n_layers * w.n_seqs * w.n_heads
+    rng = np.random.default_rng(5 + mode)
+    lab = rng.integers(0, 2, n).astype(np.uint8)
+    lab[: w.n_heads] = 0
+    lab[w.n_heads: 2 * w.n_heads] = 1
+    dev = torch.device("cuda")
+    lab_t = torch.from_numpy(lab).to(dev)
+    budget = torch.empty(n, dtype=torch.int32, device=dev)
+    cap = torch.empty(n, dtype=torch.int32, device=dev)
+    off = torch.empty(n, dtype=torch.int64, device=dev)
+    total = H.hkv_allocate_budgets(cfg, lab_t, budget, cap, off)
+    B_g = O.global_budget(w.rho, w.n_image)
+    ob, ocap, ooff, ototal = O.arena_layout(lab, w.n_cond, B_g, w.recent_w, w.period,
+                                            group=w.n_heads if mode else 0)
+    assert np.array_equal(budget.cpu().numpy(), ob)
+    assert np.array_equal(cap.cpu().numpy(), ocap)
+    assert np.array_equal(off.cpu().numpy(), ooff)
+    assert total == ototal
+
+
+@pytest.mark.parametrize("name,rho", [("lumina1024", "1/8"), ("llamagen_xl", "1/6")])
+def test_model_shapes_redistributed_budgets(name, rho):
+    """The aggregate-preserving budgets through the whole path: every global
+    head runs STE with its own history budget; positions exact against the
+    oracle with the same per-head budgets, outputs within tolerance."""
+    from fractions import Fraction
+    w = configs.ALL[name].with_(n_layers=2, n_seqs=2, rho=Fraction(rho))
+    rng = np.random.default_rng(43)
+    steps = sampled_steps(w, rng)
+    heads = [(s, l, h) for l in range(w.n_layers) for s in range(w.n_seqs) for h in range(w.n_heads)]
+    outs, poss, labels, nh, eng = run_gpu(w, out_steps=steps, pos_steps=steps,
+                                          pos_heads=[flat(w, *x) for x in heads], budget_mode=1)
+    lab = oracle_labels(w, range(w.n_layers), range(w.n_seqs))
+    check_labels(w, labels, nh, lab, name)
+    B_g = O.global_budget(w.rho, w.n_image)
+    budgets = O.arena_layout(labels, w.n_cond, B_g, w.recent_w, w.period, group=w.n_heads)[0]
+    assert np.array_equal(eng.budget.cpu().numpy(), budgets)
+    assert (budgets[labels == 1] > B_g).any()          # some global head gained tokens
+    tr = oracle_heads(w, heads, labels, record=steps, record_pos=steps, budgets=budgets)
+    worst = 0.0
+    for (s, l, h) in heads:
+        t_r, i = tr[(s, l, h)], flat(w, s, l, h)
+        for t in steps:
+            assert np.array_equal(poss[t][i], t_r.pos_at[t]), (name, s, l, h, t)
+            worst = max(worst, float(np.abs(outs[t][l, s, h] - t_r.outputs[t]).max()))
+        assert poss[w.n_image - 1][i].size == w.n_cond + int(budgets[i]) + t_r.nbuf
+    assert worst <= TOL[w.dtype], worst
