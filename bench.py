@@ -684,6 +684,71 @@ def run_grouping(args):
     print(json.dumps(line), flush=True)
 
 
+def run_labels(args):
+    """--labels: how the head types of Step 2 depend on the threshold tau and
+    on when the grouping is taken (an analogue, on the synthetic inputs, of
+    the paper's grouping-accuracy study): the dense phase runs to a late
+    step, and at the paper's grouping token E - 1 and at that late token the
+    heads of every layer are identified (hkv_identify_heads) with tau in
+    {0.85, 0.9, 0.95}. Reports the share of global heads and the agreement of
+    the labels between the two points and between thresholds."""
+    import torch
+
+    from paper_2605_20600_gb300 import hkv as H
+    from paper_2605_20600_gb300.engine import Engine, torch_dtype
+    from paper_2605_20600_gb300.runner import generate
+    from synth.gpu import DeviceSynth
+
+    dev = torch.device("cuda", 0)
+    w = workload(args)
+    L, S, Hh, D, E, N = w.n_layers, w.n_seqs, w.n_heads, w.head_dim, w.group_at, w.n_image
+    late = min(N, 4 * E)
+    wl = w.with_(group_at=late)
+    def mk(tau):
+        return H.make_config(n_layers=L, n_seqs=S, n_heads=Hh, head_dim=D, dtype=w.dtype,
+                             n_cond=w.n_cond, n_image=N, row_len=w.row_len, recent_w=w.recent_w,
+                             local_w=w.w_loc, period=w.period, group_at=late, rho=w.rho,
+                             tau=tau, r_s=w.r_s)
+
+    cfg = mk(w.tau)
+    eng = Engine(cfg, dev)
+    synth = DeviceSynth(wl, dev)
+    dt = torch_dtype(cfg)
+    q = torch.empty(L, S, Hh, D, dtype=dt, device=dev)
+    k, v = torch.empty_like(q), torch.empty_like(q)
+    n = L * S * Hh
+    taus = (0.85, 0.9, 0.95)
+    labels = {}
+
+    def on_step(t, out):
+        if t not in (E - 1, late - 1):
+            return
+        synth.image(q, k, v, 0, L, t, 1)
+        for tau in taus:
+            c = mk(tau)
+            lab = torch.empty(n, dtype=torch.uint8, device=dev)
+            nh = torch.empty(n, dtype=torch.int32, device=dev)
+            for layer in range(L):
+                H.hkv_identify_heads(c, eng.dense.c, layer, q[layer], lab, nh, eng.stream())
+            labels[(t, tau)] = lab.cpu().numpy()
+
+    generate(eng, synth, last_step=late - 1, on_step=on_step, identify="separate")
+    eng.check()
+    g = lambda x: float((x == H.HKV_GLOBAL).mean())
+    agree = lambda a, b: float((a == b).mean())
+    line = {"labels": describe(w, w.period), "heads": n, "early_token": E - 1,
+            "late_token": late - 1,
+            "global_fraction": {str(tau): {"early": g(labels[(E - 1, tau)]),
+                                           "late": g(labels[(late - 1, tau)])} for tau in taus},
+            "early_late_agreement": {str(tau): agree(labels[(E - 1, tau)], labels[(late - 1, tau)])
+                                     for tau in taus},
+            "tau_agreement_early": {f"{a}-{b}": agree(labels[(E - 1, a)], labels[(E - 1, b)])
+                                    for a, b in ((0.85, 0.9), (0.9, 0.95), (0.85, 0.95))},
+            "note": "synthetic inputs (per-head query scale drawn log-uniform); the paper's "
+                    "grouping accuracy is against its models' own attention maps"}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -700,7 +765,12 @@ def main():
                     help="budget rule: the paper's, or local heads' unused tokens to global heads")
     ap.add_argument("--grouping", action="store_true",
                     help="time the grouping step with identification separate and fused")
+    ap.add_argument("--labels", action="store_true",
+                    help="head-type shares and stability over tau and early/late grouping")
     args = ap.parse_args()
+    if args.labels:
+        run_labels(args)
+        return
     if args.strategies:
         run_strategies(args)
         return

@@ -1,0 +1,34 @@
+"""Head-type identification (Sec. 4, Step 2) on the GPU against the oracle
+away from the paper's setting: the threshold tau swept over {0.85, 0.95}
+(the paper uses 0.9 and reports 0.85-0.95 in its grouping-accuracy study),
+and the grouping taken late in the generation instead of at the paper's
+early step E. Labels must match except declared near-ties; n_h within one."""
+import numpy as np
+import pytest
+
+from synth import configs
+
+from _gpu_util import check_labels, oracle_labels, run_gpu
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.mark.parametrize("name,tau", [("lumina768", 0.85), ("lumina768", 0.95),
+                                      ("llamagen_xl", 0.85), ("janus_pro_7b", 0.95)])
+def test_tau_sweep_labels(name, tau):
+    w = configs.ALL[name].with_(n_layers=2, n_seqs=2, tau=tau)
+    _, _, labels, nh, _ = run_gpu(w, last_step=w.group_at - 1)
+    lab = oracle_labels(w, range(w.n_layers), range(w.n_seqs))
+    ties = check_labels(w, labels, nh, lab, f"{name} tau={tau}")
+    assert len(ties) <= 2, ties
+
+
+@pytest.mark.parametrize("name,late", [("llamagen_xl", 400), ("lumina768", 1200)])
+def test_late_grouping_labels(name, late):
+    w = configs.ALL[name].with_(n_layers=2, n_seqs=2, group_at=late)
+    _, _, labels, nh, _ = run_gpu(w, last_step=w.group_at - 1)
+    lab = oracle_labels(w, range(w.n_layers), range(w.n_seqs))
+    ties = check_labels(w, labels, nh, lab, f"{name} E={late}")
+    assert len(ties) <= 2, ties
+    g = float((np.asarray(labels) == 1).mean())
+    assert 0.0 < g < 1.0, g
