@@ -91,6 +91,25 @@ def grouping_count(q, K, tau: float):
     return n_h, cum
 
 
+def grouping_count_multi(Q, K, tau: float):
+    """Multi-query variant of Step 2 (not in the paper): the P buffered
+    queries Q [P, d] (oldest first, the last is the current token's) each
+    attend over the cache as it stood at their own step (query p of P sees
+    the oldest len(K) - (P - 1 - p) keys), their attention is averaged, and
+    the average is accumulated backward from the current position as in
+    grouping_count. Returns (n_h, cum)."""
+    P, n = Q.shape[0], K.shape[0]
+    pbar = np.zeros(n, dtype=np.float64)
+    for p in range(P):
+        m = n - (P - 1 - p)
+        pbar[:m] += attention_weights(Q[p], K[:m])
+    pbar /= P
+    cum = np.cumsum(pbar[::-1])
+    hit = np.nonzero(cum >= tau)[0]
+    n_h = int(hit[0]) + 1 if hit.size else int(cum.size)
+    return n_h, cum
+
+
 def classify(n_h: int, w_loc: int) -> int:
     """Local head iff fewer than w_loc tokens carry tau of the attention."""
     return LOCAL if n_h < w_loc else GLOBAL

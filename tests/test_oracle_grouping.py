@@ -76,3 +76,47 @@ def test_tiny_generator_gives_intended_head_types():
         labels.append(tr.label_computed)
         assert tr.margin > 1e-3
     assert labels == [0, 0, 0, 0, 1, 1, 1, 1]
+
+
+# Multi-query variant (not in the paper): P buffered queries, each over the
+# cache as it stood at its own step, attention averaged.
+
+def test_multi_query_with_one_query_is_step_2():
+    rng = np.random.default_rng(11)
+    for n in (5, 40, 300):
+        K = rng.normal(size=(n, 16))
+        q = rng.normal(size=16) * 3
+        a = O.grouping_count(q, K, 0.9)
+        b = O.grouping_count_multi(q[None, :], K, 0.9)
+        assert a[0] == b[0] and np.array_equal(a[1], b[1])
+
+
+def test_multi_query_uniform_closed_form():
+    # zero queries: query p spreads 1/m_p over its m_p = n - (P-1-p) keys, so
+    # key j (0-based) gets (1/P) * sum over the queries that see it of 1/m_p
+    n, P, tau = 20, 4, 0.9
+    K = np.random.default_rng(2).normal(size=(n, 8))
+    _, cum = O.grouping_count_multi(np.zeros((P, 8)), K, tau)
+    pbar = np.zeros(n)
+    for p in range(P):
+        m = n - (P - 1 - p)
+        pbar[:m] += 1.0 / m
+    pbar /= P
+    assert np.allclose(cum, np.cumsum(pbar[::-1]), rtol=0, atol=1e-15)
+    assert abs(cum[-1] - 1.0) < 1e-15
+    # the newest key is seen by the current query only: mass 1/(P n)
+    assert abs(cum[0] - 1.0 / (P * n)) < 1e-15
+
+
+def test_multi_query_older_queries_do_not_see_newer_keys():
+    # the current query attends only to the newest key; an older query sees
+    # every key but the newest and puts its mass on the oldest: the average
+    # is half on each end
+    D, n = 8, 10
+    K = np.zeros((n, D))
+    K[-1, 0] = 40 * math.sqrt(D)
+    K[0, 1] = 40 * math.sqrt(D)
+    Q = np.zeros((2, D)); Q[1, 0] = 1.0; Q[0, 1] = 1.0
+    n_h, cum = O.grouping_count_multi(Q, K, 0.9)
+    assert abs(cum[0] - 0.5) < 1e-12 and abs(cum[-2] - 0.5) < 1e-12
+    assert n_h == n            # tau needs the oldest key too: global for any w_loc <= n
