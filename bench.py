@@ -690,8 +690,11 @@ def run_labels(args):
     the paper's grouping-accuracy study): the dense phase runs to a late
     step, and at the paper's grouping token E - 1 and at that late token the
     heads of every layer are identified (hkv_identify_heads) with tau in
-    {0.85, 0.9, 0.95}. Reports the share of global heads and the agreement of
-    the labels between the two points and between thresholds."""
+    {0.85, 0.9, 0.95}, and at tau = 0.9 also by the multi-query variant
+    (hkv_identify_heads_multi). Reports the share of global heads, the
+    agreement of the labels between the two points, between thresholds and
+    between the two identifications, and the device time of each
+    identification over all layers."""
     import torch
 
     from paper_2605_20600_gb300 import hkv as H
@@ -718,7 +721,7 @@ def run_labels(args):
     k, v = torch.empty_like(q), torch.empty_like(q)
     n = L * S * Hh
     taus = (0.85, 0.9, 0.95)
-    labels = {}
+    labels, times = {}, {}
 
     def on_step(t, out):
         if t not in (E - 1, late - 1):
@@ -731,6 +734,22 @@ def run_labels(args):
             for layer in range(L):
                 H.hkv_identify_heads(c, eng.dense.c, layer, q[layer], lab, nh, eng.stream())
             labels[(t, tau)] = lab.cpu().numpy()
+        c = mk(w.tau)
+        lab = torch.empty(n, dtype=torch.uint8, device=dev)
+        nh = torch.empty(n, dtype=torch.int32, device=dev)
+        for kind in ("single", "multi"):
+            for rep in range(3):  # the last of three repetitions is timed
+                ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+                ev[0].record()
+                for layer in range(L):
+                    if kind == "single":
+                        H.hkv_identify_heads(c, eng.dense.c, layer, q[layer], lab, nh, eng.stream())
+                    else:
+                        H.hkv_identify_heads_multi(c, eng.dense.c, layer, lab, nh, eng.stream())
+                ev[1].record()
+            torch.cuda.synchronize()
+            labels[(t, kind)] = lab.cpu().numpy()
+            times[(t, kind)] = ev[0].elapsed_time(ev[1]) * 1e3 / L
 
     generate(eng, synth, last_step=late - 1, on_step=on_step, identify="separate")
     eng.check()
@@ -744,6 +763,17 @@ def run_labels(args):
                                      for tau in taus},
             "tau_agreement_early": {f"{a}-{b}": agree(labels[(E - 1, a)], labels[(E - 1, b)])
                                     for a, b in ((0.85, 0.9), (0.9, 0.95), (0.85, 0.95))},
+            "multi_query": {
+                "queries": w.period,
+                "global_fraction": {"early": g(labels[(E - 1, "multi")]),
+                                    "late": g(labels[(late - 1, "multi")])},
+                "early_late_agreement": agree(labels[(E - 1, "multi")], labels[(late - 1, "multi")]),
+                "agreement_with_single": {"early": agree(labels[(E - 1, "multi")], labels[(E - 1, "single")]),
+                                          "late": agree(labels[(late - 1, "multi")], labels[(late - 1, "single")])},
+                "us_per_layer": {"single_early": times[(E - 1, "single")],
+                                 "multi_early": times[(E - 1, "multi")],
+                                 "single_late": times[(late - 1, "single")],
+                                 "multi_late": times[(late - 1, "multi")]}},
             "note": "synthetic inputs (per-head query scale drawn log-uniform); the paper's "
                     "grouping accuracy is against its models' own attention maps"}
     print(json.dumps(line), flush=True)

@@ -286,6 +286,26 @@ hkv_status hkv_identify_heads(const hkv_config *cfg, const hkv_cache *cache, int
                               const void *q, uint8_t *label_out, int32_t *nh_out,
                               hkv_stream_t stream);
 
+/* A variant of Sec. 4, Step 2 that the paper does not have: the decision
+ * from the attention of several recent queries instead of the current one.
+ * For each head of one layer of an HKV_DENSE cache, the newest
+ * Pe = min(period, ntok) queries of the cache's query ring (written by the
+ * decode steps; the newest is the current token's) each attend over the keys
+ * that existed at their own step: the p-th oldest (p = 0 .. Pe-1) over the
+ * oldest len - (Pe - 1 - p) keys. Their softmax rows are averaged, the
+ * average is accumulated backward from the newest token until tau is
+ * reached, n_h is the number of tokens needed, and the head is HKV_LOCAL iff
+ * n_h < w_loc. With period = 1 this is hkv_identify_heads. Call it after the
+ * grouping token's decode step, like hkv_identify_heads. Writes
+ * label_out[i] and, if non-null, nh_out[i] for the layer's heads (device
+ * arrays of [L*S*H]).
+ *  - a head with another label than HKV_DENSE, or with ntok = 0 (no query
+ *    buffered yet): HKV_ERR_STATE in the error word, head not decided;
+ *  - len above n_cond + group_at: HKV_ERR_CAPACITY in the error word;
+ *  - label_out NULL or layer out of range: HKV_ERR_INVALID_ARG. */
+hkv_status hkv_identify_heads_multi(const hkv_config *cfg, const hkv_cache *cache, int layer,
+                                    uint8_t *label_out, int32_t *nh_out, hkv_stream_t stream);
+
 /* Sec. 5.1 budgets for all L*S*H heads from their labels: budget = B_g
  * (global) or w (local) image tokens (or the redistributed budgets, per
  * cfg->budget_mode), cap = C + budget + P, off = exclusive prefix sum of cap

@@ -10,7 +10,11 @@ Compression for Efficient Autoregressive Image Generation" (HeadKV):
   attention          Eq. 1 (Sec. 3), fp64 brute force
   grouping_count     Sec. 4 Step 2 (threshold-based attention accumulation)
   classify           Sec. 4 Step 2 (local iff the count is below w_loc)
+  grouping_count_multi  a variant of Step 2 not in the paper: the buffered
+                     queries' attention averaged, each over its own prefix
   global_budget      Sec. 5.1 Implementation Details (rho * N tokens)
+  redistributed_budgets  a budget variant not in the paper: local heads'
+                     unused tokens shared among the group's global heads
   arena_layout       Sec. 5.1 (local heads keep w, global heads rho*N) and
                      Sec. 4 Efficient Cache Update (room for P buffered tokens)
   ste_partition      Eq. 5 (long/near split by r_s)

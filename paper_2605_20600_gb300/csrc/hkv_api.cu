@@ -404,6 +404,25 @@ hkv_status hkv_identify_heads(const hkv_config *cfg, const hkv_cache *cache, int
                                      (cudaStream_t)stream));
 }
 
+hkv_status hkv_identify_heads_multi(const hkv_config *cfg, const hkv_cache *cache, int layer,
+                                    uint8_t *label_out, int32_t *nh_out, hkv_stream_t stream) {
+  HKV_TRY(injected("identify_heads_multi"));
+  HKV_TRY(hkv_validate_config(cfg));
+  HKV_TRY(check_cache(cache));
+  if (layer < 0 || layer >= cfg->n_layers) return HKV_ERR_INVALID_ARG;
+  if (!label_out) return HKV_ERR_INVALID_ARG;
+  DeviceState *st;
+  HKV_TRY(device_state(&st));
+  const int max_len = cfg->n_cond + cfg->group_at;
+  const size_t upd = update_smem_bytes(max_segment(cfg), cfg->head_dim, cfg->period, cfg->dtype);
+  const size_t need = identify_multi_smem_bytes(max_len, cfg->period);
+  HKV_TRY(update_ready(st, cfg->head_dim, cfg->dtype, upd > need ? upd : need));
+  const int hpl = heads_per_layer(cfg);
+  return cuda_status(launch_identify_multi(cache_args(cache), method_args(cfg), layer * hpl, hpl,
+                                           label_out, nh_out, cfg->head_dim, cfg->dtype, max_len,
+                                           (cudaStream_t)stream));
+}
+
 hkv_status hkv_allocate_budgets(const hkv_config *cfg, const uint8_t *label, int32_t *budget,
                                 int32_t *cap, int64_t *off, int64_t *total_tokens,
                                 hkv_stream_t stream) {

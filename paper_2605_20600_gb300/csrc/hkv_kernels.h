@@ -126,6 +126,13 @@ cudaError_t launch_init_dense(const CacheArgs &c, int nheads_total, int seg_toke
 cudaError_t launch_identify(const CacheArgs &c, const MethodArgs &m, int layer_base, int nheads,
                             const void *q, uint8_t *label_out, int32_t *nh_out, int D, int dtype,
                             int max_len, cudaStream_t s);
+// multi-query Step 2 over the ring's newest min(P, ntok) queries (the
+// kernel needs identify_multi_smem_bytes(max_len, P) of shared memory, at
+// most what update_prepare enabled)
+size_t identify_multi_smem_bytes(int max_len, int P);
+cudaError_t launch_identify_multi(const CacheArgs &c, const MethodArgs &m, int layer_base,
+                                  int nheads, uint8_t *label_out, int32_t *nh_out, int D,
+                                  int dtype, int max_len, cudaStream_t s);
 // group > 0: the aggregate-preserving budgets over groups of that many heads
 cudaError_t launch_budgets(const uint8_t *label, int32_t *budget, int32_t *cap, int64_t *off,
                            int n, int C, int B_g, int w, int P, int group, cudaStream_t s);

@@ -740,6 +740,182 @@ __global__ void __launch_bounds__(NT)
   }
 }
 
+// Block-wide max (MAX) or sum of N floats per thread, returned to every
+// thread in place; red holds N values per warp, bc the N results.
+// Consecutive calls are safe: each reads its operands before the next call
+// writes them.
+template <bool MAX, int N>
+__device__ __forceinline__ void block_all(float (&v)[N], float *red, float *bc) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+#pragma unroll
+  for (int b = 0; b < N; ++b) {
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) {
+      const float u = __shfl_xor_sync(0xFFFFFFFFu, v[b], o);
+      v[b] = MAX ? fmaxf(v[b], u) : v[b] + u;
+    }
+    if (lane == 0) red[b * nw + warp] = v[b];
+  }
+  __syncthreads();
+  if (threadIdx.x < N) {
+    const int b = threadIdx.x;
+    float a = red[b * nw];
+    for (int w = 1; w < nw; ++w) a = MAX ? fmaxf(a, red[b * nw + w]) : a + red[b * nw + w];
+    bc[b] = a;
+  }
+  __syncthreads();
+#pragma unroll
+  for (int b = 0; b < N; ++b) v[b] = bc[b];
+}
+
+// queries of the multi-query identification handled per pass over the keys:
+// 8 for rings of at least kIdQB8From queries, else 4 (measured on a GB300:
+// 8 is 17 % faster on 65-query rings over 628 keys, 4 is 26-33 % faster on
+// 24-query rings over 101-164 keys, where the fewer registers of 4 give
+// more CTAs per SM)
+constexpr int kIdQB8From = 48;
+__host__ __device__ constexpr int id_qb(int P) { return P >= kIdQB8From ? 8 : 4; }
+
+// Multi-query variant of Step 2 (not in the paper): the newest Pe = min(P,
+// ntok) queries of the ring each attend over the keys that existed at their
+// own step (the p-th oldest of them over the oldest len - (Pe - 1 - p)
+// keys), their normalised attention rows are averaged, and the average is
+// accumulated backward from the newest token until tau, as in
+// identify_kernel. One CTA per head; each pass over the keys serves QB
+// queries (every key row loaded once per pass, dotted with all of them).
+template <int D, typename T, int QB>
+__global__ void __launch_bounds__(NT)
+    identify_multi_kernel(const CacheArgs c, const MethodArgs m, int layer_base,
+                          uint8_t *label_out, int32_t *nh_out, float qscale, int max_len) {
+  constexpr int RB = D * (int)sizeof(T);
+  constexpr int EPL = Elem<T>::kPerPiece;
+  constexpr int LPR = RB / 16;
+  constexpr int RPW = 32 / LPR;
+  constexpr int NW = NT / 32;
+  extern __shared__ float e[];      // [QB][max_len] the pass's logits, then weights
+  float *pbar = e + QB * max_len;  // [max_len] summed weights of all queries
+  __shared__ float red[QB * NW];
+  __shared__ float s_b[QB];
+  __shared__ float fscan[33];
+  __shared__ int s_nh;
+  pdl_wait();
+  pdl_launch_dependents();
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int hl = blockIdx.x, i = layer_base + hl;
+  const int len = c.len[i];
+  const int ntok = c.ntok[i];
+  const long long off = c.off[i];
+  if (c.label[i] != HKV_DENSE || ntok <= 0) {  // in position order, with buffered queries
+    if (tid == 0) set_err(c.err, HKV_ERR_STATE);
+    return;
+  }
+  if (off < 0 || len <= 0 || off + len > c.arena_tokens) {
+    if (tid == 0) set_err(c.err, HKV_ERR_BOUNDS);
+    return;
+  }
+  if (len > max_len) {
+    if (tid == 0) set_err(c.err, HKV_ERR_CAPACITY);
+    return;
+  }
+  const int Pe = min(m.P, min(ntok, len));
+  const int grp = lane / LPR, col = lane % LPR;
+  const unsigned char *K = static_cast<const unsigned char *>(c.K) + off * RB;
+  const unsigned char *ring = static_cast<const unsigned char *>(c.qbuf) + (size_t)i * m.P * RB;
+  for (int r = tid; r < len; r += NT) pbar[r] = 0.f;
+  for (int p0 = 0; p0 < Pe; p0 += QB) {
+    // query p0 + b sees mq[b] keys (0 past the newest query)
+    int mq[QB];
+    float qf[QB][EPL];
+#pragma unroll
+    for (int b = 0; b < QB; ++b) {
+      const int p = p0 + b;
+      mq[b] = p < Pe ? len - (Pe - 1 - p) : 0;
+      if (p < Pe) {
+        const int slot = (ntok - Pe + p) % m.P;
+        Elem<T>::unpack(*reinterpret_cast<const uint4 *>(ring + (size_t)slot * RB + col * 16),
+                        qf[b]);
+      }
+#pragma unroll
+      for (int x = 0; x < EPL; ++x) qf[b][x] = p < Pe ? qf[b][x] * qscale : 0.f;
+    }
+    const int mmax = len - max(0, Pe - 1 - (p0 + QB - 1));  // keys of the pass's newest query
+    for (int r0 = warp * RPW; r0 < mmax; r0 += NW * RPW) {  // logits (log2 units)
+      const int r = r0 + grp;
+      float dot[QB];
+#pragma unroll
+      for (int b = 0; b < QB; ++b) dot[b] = 0.f;
+      if (r < mmax) {
+        float kf[EPL];
+        Elem<T>::unpack(*reinterpret_cast<const uint4 *>(K + (size_t)r * RB + col * 16), kf);
+#pragma unroll
+        for (int b = 0; b < QB; ++b)
+#pragma unroll
+          for (int x = 0; x < EPL; ++x) dot[b] = fmaf(qf[b][x], kf[x], dot[b]);
+      }
+#pragma unroll
+      for (int b = 0; b < QB; ++b) {
+#pragma unroll
+        for (int o = LPR / 2; o >= 1; o >>= 1) dot[b] += __shfl_xor_sync(0xFFFFFFFFu, dot[b], o);
+        if (col == 0 && r < mq[b]) e[b * max_len + r] = dot[b];
+      }
+    }
+    __syncthreads();
+    float acc[QB];
+#pragma unroll
+    for (int b = 0; b < QB; ++b) acc[b] = -INFINITY;
+    for (int r = tid; r < mmax; r += NT)
+#pragma unroll
+      for (int b = 0; b < QB; ++b)
+        if (r < mq[b]) acc[b] = fmaxf(acc[b], e[b * max_len + r]);
+    block_all<true, QB>(acc, red, s_b);
+    float mx[QB];
+#pragma unroll
+    for (int b = 0; b < QB; ++b) {
+      mx[b] = acc[b];
+      acc[b] = 0.f;
+    }
+    for (int r = tid; r < mmax; r += NT)
+#pragma unroll
+      for (int b = 0; b < QB; ++b)
+        if (r < mq[b]) {
+          const float x = exp2f(e[b * max_len + r] - mx[b]);
+          e[b * max_len + r] = x;
+          acc[b] += x;
+        }
+    block_all<false, QB>(acc, red, s_b);
+#pragma unroll
+    for (int b = 0; b < QB; ++b) acc[b] = 1.f / acc[b];  // unused past the newest query
+    for (int r = tid; r < mmax; r += NT) {
+      float s = pbar[r];
+#pragma unroll
+      for (int b = 0; b < QB; ++b)
+        if (r < mq[b]) s = fmaf(e[b * max_len + r], acc[b], s);
+      pbar[r] = s;
+    }
+    __syncthreads();  // e is rewritten by the next pass
+  }
+  float tot[1] = {0.f};
+  for (int r = tid; r < len; r += NT) tot[0] += pbar[r];
+  block_all<false, 1>(tot, red, s_b);
+  const float thr = tot[0] * m.tau;
+  if (tid == 0) s_nh = len;
+  __syncthreads();
+  float running = 0.f;  // backward cumulative mass from the newest token
+  for (int base = 0; base < len; base += NT) {
+    const int jb = base + tid;  // jb-th newest token (0 = current)
+    const float x = jb < len ? pbar[len - 1 - jb] : 0.f;
+    float t;
+    const float cum = running + block_excl_scan<float>(x, fscan, &t) + x;
+    if (jb < len && cum >= thr) atomicMin(&s_nh, jb + 1);
+    running += t;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    label_out[i] = s_nh < m.w_loc ? HKV_LOCAL : HKV_GLOBAL;
+    if (nh_out) nh_out[i] = s_nh;
+  }
+}
+
 // Sec. 5.1 budgets (group = 0), or the aggregate-preserving variant over
 // consecutive groups of `group` heads, one (sequence, layer) each: the
 // (group - n_g)(B_g - w) tokens the local heads leave go to the group's n_g
@@ -808,6 +984,12 @@ cudaError_t prepare_t(size_t smem) {
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(identify_kernel<D, T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(identify_multi_kernel<D, T, 4>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(identify_multi_kernel<D, T, 8>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   // all of an SM's L1 as shared memory, so that every head of a layer (one
   // CTA each) is resident at once
   if (e == cudaSuccess)
@@ -945,6 +1127,27 @@ cudaError_t launch_identify(const CacheArgs &c, const MethodArgs &m, int layer_b
                return pdl_launch(identify_kernel<kD, kT>, nheads, NT, smem, s, c, m, layer_base,
                                  q, label_out, nh_out, qscale, max_len));
   return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_identify_multi(const CacheArgs &c, const MethodArgs &m, int layer_base,
+                                  int nheads, uint8_t *label_out, int32_t *nh_out, int D,
+                                  int dtype, int max_len, cudaStream_t s) {
+  const float qscale = (float)(1.4426950408889634 / sqrt((double)D));
+  const size_t smem = identify_multi_smem_bytes(max_len, m.P);
+  if (id_qb(m.P) == 8) {
+    HKV_DISPATCH(D, dtype,
+                 return pdl_launch(identify_multi_kernel<kD, kT, 8>, nheads, NT, smem, s, c, m,
+                                   layer_base, label_out, nh_out, qscale, max_len));
+  } else {
+    HKV_DISPATCH(D, dtype,
+                 return pdl_launch(identify_multi_kernel<kD, kT, 4>, nheads, NT, smem, s, c, m,
+                                   layer_base, label_out, nh_out, qscale, max_len));
+  }
+  return cudaErrorInvalidValue;
+}
+
+size_t identify_multi_smem_bytes(int max_len, int P) {
+  return (size_t)(id_qb(P) + 1) * 4 * max_len;
 }
 
 cudaError_t launch_budgets(const uint8_t *label, int32_t *budget, int32_t *cap, int64_t *off,

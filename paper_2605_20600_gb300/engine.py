@@ -112,6 +112,11 @@ class Engine:
     def identify(self, layer: int, q) -> None:
         H.hkv_identify_heads(self.cfg, self.dense.c, layer, q, self.labels, self.n_h, self.stream())
 
+    def identify_multi(self, layer: int) -> None:
+        """Step 2 from the ring's recent queries (a variant the paper does not
+        have): labels and n_h."""
+        H.hkv_identify_heads_multi(self.cfg, self.dense.c, layer, self.labels, self.n_h, self.stream())
+
     # Step 3: budgets, arena, repack of every layer
     def compress(self, labels=None) -> None:
         if labels is not None:

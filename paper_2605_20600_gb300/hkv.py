@@ -77,6 +77,8 @@ _SIGNATURES = {
     "hkv_evict": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p], c_int),
     "hkv_identify_heads": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p, c_void_p, c_void_p,
                             c_void_p], c_int),
+    "hkv_identify_heads_multi": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p, c_void_p,
+                                  c_void_p], c_int),
     "hkv_allocate_budgets": ([POINTER(hkv_config), c_void_p, c_void_p, c_void_p, c_void_p,
                               POINTER(c_int64), c_void_p], c_int),
     "hkv_repack": ([POINTER(hkv_config), POINTER(hkv_cache), POINTER(hkv_cache), c_int, c_void_p], c_int),
@@ -175,6 +177,11 @@ def hkv_evict(cfg, cache, layer, stream=0) -> None:
 
 def hkv_identify_heads(cfg, cache, layer, q, label_out, nh_out=None, stream=0) -> None:
     _call("identify_heads", ctypes.byref(cfg), ctypes.byref(cache), layer, _p(q), _p(label_out),
+          _p(nh_out), stream)
+
+
+def hkv_identify_heads_multi(cfg, cache, layer, label_out, nh_out=None, stream=0) -> None:
+    _call("identify_heads_multi", ctypes.byref(cfg), ctypes.byref(cache), layer, _p(label_out),
           _p(nh_out), stream)
 
 

@@ -25,12 +25,13 @@ def generate(engine: Engine, provider, *, last_step: int | None = None, on_step=
     first_step > 0 continues a generation (the prefill is skipped).
     identify: "fused" decides the head types inside the grouping token's
     decode step (fused path only; no n_h), "separate" runs
-    hkv_identify_heads after it (labels and n_h). Default: fused when the
-    path is fused.
+    hkv_identify_heads after it (labels and n_h), "multi" runs
+    hkv_identify_heads_multi after it (the recent queries' averaged
+    attention; labels and n_h). Default: fused when the path is fused.
     """
     if identify is None:
         identify = "fused" if fused else "separate"
-    if identify not in ("fused", "separate") or (identify == "fused" and not fused):
+    if identify not in ("fused", "separate", "multi") or (identify == "fused" and not fused):
         raise ValueError(f"identify={identify!r} with fused={fused}")
     cfg = engine.cfg
     L, S, H, D, C = cfg.n_layers, cfg.n_seqs, cfg.n_heads, cfg.head_dim, cfg.n_cond
@@ -63,6 +64,8 @@ def generate(engine: Engine, provider, *, last_step: int | None = None, on_step=
                 engine.attend(layer, q[layer], out[layer])
             if t == E - 1 and identify == "separate":
                 engine.identify(layer, q[layer])
+            elif t == E - 1 and identify == "multi":
+                engine.identify_multi(layer)
         if on_step is not None:
             on_step(t, out)
         if t == E - 1:

@@ -61,7 +61,7 @@ def run_gpu(w, *, out_steps=(), pos_steps=(), pos_heads=(), last_step=None, fuse
              identify=identify)
     torch.cuda.synchronize()
     eng.check()
-    nh = eng.n_h.cpu().numpy() if identify == "separate" else None
+    nh = eng.n_h.cpu().numpy() if identify in ("separate", "multi") else None
     return outs, poss, eng.labels.cpu().numpy(), nh, eng
 
 
@@ -92,8 +92,9 @@ def oracle_heads(w, heads, labels=None, record=(), record_pos=(), budgets=None):
 
 
 def label_job(args):
-    """Oracle grouping for heads of one (s, l): (label, n_h, margin) per head."""
-    w, s, l, heads = args
+    """Oracle grouping for heads of one (s, l): (label, n_h, margin) per head;
+    multi: from the newest min(P, E) queries (grouping_count_multi)."""
+    w, s, l, heads, multi = args
     pe, cq = gen.pe_table(w), gen.q_coef(w)
     hp = O.HeadParams.of(w)
     res = []
@@ -101,13 +102,17 @@ def label_job(args):
         hi = gen.HeadInputs(w, s, l, h, pe, cq)
         t = w.group_at - 1
         K = hi.k[: w.n_cond + t + 1]
-        n_h, cum = O.grouping_count(hi.q[t], K, w.tau)
+        if multi:
+            Q = hi.q[max(0, t + 1 - w.period): t + 1]
+            n_h, cum = O.grouping_count_multi(Q, K, w.tau)
+        else:
+            n_h, cum = O.grouping_count(hi.q[t], K, w.tau)
         res.append((O.classify(n_h, w.w_loc), n_h, O.label_margin(cum, w.tau, w.w_loc)))
     return (s, l), res
 
 
-def oracle_labels(w, layers, seqs):
-    jobs = [(w, s, l, tuple(range(w.n_heads))) for l in layers for s in seqs]
+def oracle_labels(w, layers, seqs, multi=False):
+    jobs = [(w, s, l, tuple(range(w.n_heads)), multi) for l in layers for s in seqs]
     n = min(len(jobs), os.cpu_count() or 1, 16)
     with mp.get_context("spawn").Pool(n) as pool:
         return dict(pool.map(label_job, jobs, chunksize=1))

@@ -47,7 +47,7 @@ def fake_cache(H, **kw):
 
 def test_every_declared_symbol_is_exported(H):
     names = declared_functions()
-    assert len(names) == 16
+    assert len(names) == 17
     for n in names:
         assert hasattr(H.lib(), n), n
     assert set(names) >= {"hkv_identify_heads", "hkv_allocate_budgets", "hkv_append_evict",
@@ -114,6 +114,9 @@ def test_null_and_misaligned_arguments(H):
     assert lib.hkv_append_evict(ctypes.byref(cfg), ctypes.byref(bad), 0, 16, 16, 16, None) == 8
     nul = fake_cache(H, err=None)
     assert lib.hkv_identify_heads(ctypes.byref(cfg), ctypes.byref(nul), 0, 16, 16, None, None) == 1
+    assert lib.hkv_identify_heads_multi(ctypes.byref(cfg), ctypes.byref(nul), 0, 16, None, None) == 1
+    assert lib.hkv_identify_heads_multi(ctypes.byref(cfg), ctypes.byref(c), 0, None, None, None) == 1
+    assert lib.hkv_identify_heads_multi(ctypes.byref(cfg), ctypes.byref(c), 2, 16, None, None) == 1
     small = fake_cache(H, capacity_tokens=10)
     assert lib.hkv_init_dense(ctypes.byref(cfg), ctypes.byref(small), None) == 3
     other = fake_cache(H, qbuf=c.qbuf + 256)
@@ -143,7 +146,8 @@ def test_null_and_misaligned_arguments(H):
 
 @pytest.mark.parametrize("name", ["decode_attention", "append_evict", "identify_heads",
                                   "allocate_budgets", "repack", "prefill", "init_dense", "check",
-                                  "decode_step", "evict", "export_state", "decode_step_identify"])
+                                  "decode_step", "evict", "export_state", "decode_step_identify",
+                                  "identify_heads_multi"])
 def test_fault_injection_returns_the_code(H, name, monkeypatch):
     cfg = tiny_cfg(H)
     c = fake_cache(H)
@@ -153,6 +157,7 @@ def test_fault_injection_returns_the_code(H, name, monkeypatch):
         "decode_attention": lambda: lib.hkv_decode_attention(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, 16, 1 << 30, None),
         "append_evict": lambda: lib.hkv_append_evict(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, 16, None),
         "identify_heads": lambda: lib.hkv_identify_heads(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, None, None),
+        "identify_heads_multi": lambda: lib.hkv_identify_heads_multi(ctypes.byref(cfg), ctypes.byref(c), 0, 16, None, None),
         "allocate_budgets": lambda: lib.hkv_allocate_budgets(ctypes.byref(cfg), 16, 16, 16, 16, None, None),
         "repack": lambda: lib.hkv_repack(ctypes.byref(cfg), ctypes.byref(c), ctypes.byref(c), 0, None),
         "prefill": lambda: lib.hkv_prefill(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, None),

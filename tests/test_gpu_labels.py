@@ -2,7 +2,9 @@
 away from the paper's setting: the threshold tau swept over {0.85, 0.95}
 (the paper uses 0.9 and reports 0.85-0.95 in its grouping-accuracy study),
 and the grouping taken late in the generation instead of at the paper's
-early step E. Labels must match except declared near-ties; n_h within one."""
+early step E; and the multi-query variant (the newest P queries' averaged
+attention, each query over the keys of its own step). Labels must match
+except declared near-ties; n_h within one."""
 import numpy as np
 import pytest
 
@@ -32,3 +34,26 @@ def test_late_grouping_labels(name, late):
     assert len(ties) <= 2, ties
     g = float((np.asarray(labels) == 1).mean())
     assert 0.0 < g < 1.0, g
+
+
+@pytest.mark.parametrize("name", ["lumina768", "lumina1024", "llamagen_xl", "janus_pro_7b"])
+def test_multi_query_labels(name):
+    w = configs.ALL[name].with_(n_layers=2, n_seqs=2)
+    _, _, labels, nh, _ = run_gpu(w, last_step=w.group_at - 1, identify="multi")
+    lab = oracle_labels(w, range(w.n_layers), range(w.n_seqs), multi=True)
+    ties = check_labels(w, labels, nh, lab, f"{name} multi")
+    assert len(ties) <= 2, ties
+    # every margin is far from tau here, so n_h was compared for every head
+    assert min(m for res in lab.values() for (_, _, m) in res) > 1e-3
+
+
+@pytest.mark.parametrize("name", ["llamagen_xl", "lumina768"])
+def test_multi_query_labels_grouping_at_the_period(name):
+    """E = P: every image token's query counts, the oldest over only the
+    conditioning tokens and itself."""
+    w0 = configs.ALL[name]
+    w = w0.with_(n_layers=1, n_seqs=2, group_at=w0.period)
+    _, _, labels, nh, _ = run_gpu(w, last_step=w.group_at - 1, identify="multi")
+    lab = oracle_labels(w, range(w.n_layers), range(w.n_seqs), multi=True)
+    ties = check_labels(w, labels, nh, lab, f"{name} E=P multi")
+    assert len(ties) <= 2, ties

@@ -110,7 +110,7 @@ def test_hand_worked_grid_fused_identification():
 
 
 @pytest.mark.parametrize("fused,identify", [(True, "separate"), (False, "separate"),
-                                            (True, "fused")])
+                                            (True, "fused"), (True, "multi")])
 def test_tiny_every_step_every_head(fused, identify):
     w = configs.TINY
     N = w.n_image
@@ -118,7 +118,7 @@ def test_tiny_every_step_every_head(fused, identify):
     outs, poss, labels, nh, eng = run_gpu(w, out_steps=range(N), pos_steps=range(N),
                                           pos_heads=[flat(w, *x) for x in heads], fused=fused,
                                           identify=identify)
-    lab = oracle_labels(w, [0], [0])
+    lab = oracle_labels(w, [0], [0], multi=identify == "multi")
     ties = check_labels(w, labels, nh, lab, "tiny")
     assert not ties
     assert labels.tolist() == [0, 0, 0, 0, 1, 1, 1, 1]
@@ -147,7 +147,9 @@ REDUCED = [("lumina768", "1/4", True, "separate"), ("lumina1024", "1/4", True, "
            ("lumina1024", "1/8", False, "separate"), ("llamagen_xl", "1/6", False, "separate"),
            # the head types decided inside the grouping token's decode step
            ("lumina1024", "1/4", True, "fused"), ("llamagen_xl", "1/6", True, "fused"),
-           ("janus_pro_7b", "1/8", True, "fused")]
+           ("janus_pro_7b", "1/8", True, "fused"),
+           # the head types from the recent queries' averaged attention
+           ("lumina768", "1/4", True, "multi"), ("janus_pro_7b", "1/8", True, "multi")]
 
 
 @pytest.mark.parametrize("name,rho,fused,identify", REDUCED)
@@ -160,7 +162,7 @@ def test_model_shapes_two_layers_two_seqs(name, rho, fused, identify):
     outs, poss, labels, nh, eng = run_gpu(w, out_steps=steps, pos_steps=steps,
                                           pos_heads=[flat(w, *x) for x in heads], fused=fused,
                                           identify=identify)
-    lab = oracle_labels(w, range(w.n_layers), range(w.n_seqs))
+    lab = oracle_labels(w, range(w.n_layers), range(w.n_seqs), multi=identify == "multi")
     ties = check_labels(w, labels, nh, lab, name)
     assert len(ties) <= 2, ties
     g = float((labels == 1).mean())
