@@ -12,12 +12,19 @@ Compression for Efficient Autoregressive Image Generation" (HeadKV):
   classify           Sec. 4 Step 2 (local iff the count is below w_loc)
   grouping_count_multi  a variant of Step 2 not in the paper: the buffered
                      queries' attention averaged, each over its own prefix
+  grid_d2, count_order_2d, grouping_count_2d, grouping_count_multi_2d
+                     a variant of Step 2 not in the paper: the count runs
+                     outward from the current token by distance on the image
+                     grid instead of backward in raster order
   global_budget      Sec. 5.1 Implementation Details (rho * N tokens)
   redistributed_budgets  a budget variant not in the paper: local heads'
                      unused tokens shared among the group's global heads
   arena_layout       Sec. 5.1 (local heads keep w, global heads rho*N) and
                      Sec. 4 Efficient Cache Update (room for P buffered tokens)
   ste_partition      Eq. 5 (long/near split by r_s)
+  ste_long_2d, ste_evict_strata
+                     a variant of Eq. 5 not in the paper: the long-range
+                     subset is the T r_s history tokens farthest on the grid
   ste_scores_eq6     Eq. 6 as printed, fp64
   ste_scores_fp32    Eq. 6 ranking in the precision the decision is taken in
   ste_quotas         Sec. 4 STE (M/2 evicted from each subset)
@@ -114,6 +121,59 @@ def grouping_count_multi(Q, K, tau: float):
     return n_h, cum
 
 
+# Variant (not in the paper): distance on the image grid. Image token i sits
+# in row i // row_len, column i % row_len (end-of-row tokens included); the
+# distance of two image tokens is the squared Euclidean distance of their
+# cells, an integer.
+RASTER, GRID2D = 0, 1
+
+
+def grid_d2(i: int, j: int, row_len: int) -> int:
+    """Squared grid distance of image tokens i and j."""
+    dr = i // row_len - j // row_len
+    dc = i % row_len - j % row_len
+    return dr * dr + dc * dc
+
+
+def count_order_2d(n_tokens: int, n_cond: int, row_len: int) -> np.ndarray:
+    """Order in which the 2D variant of Step 2 counts the tokens of a cache in
+    position order (0 .. n_tokens-1, the first n_cond conditioning): image
+    tokens by grid distance from the newest image token, nearest first, equal
+    distances newer first; then the conditioning tokens, newest first (they
+    have no cell and come last, as in the raster count)."""
+    ref = n_tokens - 1 - n_cond
+    img = sorted(range(n_cond, n_tokens),
+                 key=lambda p: (grid_d2(p - n_cond, ref, row_len), -p))
+    return np.array(img + list(range(n_cond - 1, -1, -1)), dtype=np.int64)
+
+
+def _count_along(pbar, order, tau: float):
+    cum = np.cumsum(pbar[order])
+    hit = np.nonzero(cum >= tau)[0]
+    n_h = int(hit[0]) + 1 if hit.size else int(cum.size)
+    return n_h, cum
+
+
+def grouping_count_2d(q, K, tau: float, n_cond: int, row_len: int):
+    """Step 2 with the count running outward on the grid (count_order_2d)
+    instead of backward in raster order. K holds the cache in position
+    order. Returns (n_h, cum)."""
+    p = attention_weights(q, K)
+    return _count_along(p, count_order_2d(K.shape[0], n_cond, row_len), tau)
+
+
+def grouping_count_multi_2d(Q, K, tau: float, n_cond: int, row_len: int):
+    """grouping_count_multi's averaged attention counted in count_order_2d
+    (outward from the current, newest, token)."""
+    P, n = Q.shape[0], K.shape[0]
+    pbar = np.zeros(n, dtype=np.float64)
+    for p in range(P):
+        m = n - (P - 1 - p)
+        pbar[:m] += attention_weights(Q[p], K[:m])
+    pbar /= P
+    return _count_along(pbar, count_order_2d(n, n_cond, row_len), tau)
+
+
 def classify(n_h: int, w_loc: int) -> int:
     """Local head iff fewer than w_loc tokens carry tau of the attention."""
     return LOCAL if n_h < w_loc else GLOBAL
@@ -187,6 +247,19 @@ def ste_partition(T: int, r_s: float) -> int:
     return int(math.floor(float(T) * float(r_s)))
 
 
+def ste_long_2d(hist, n_long: int, n_cond: int, row_len: int, t_ref: int) -> np.ndarray:
+    """2D variant of Eq. 5 (not in the paper): the long-range subset is the
+    n_long history tokens (positions `hist`) farthest on the grid from image
+    token t_ref (the newest), equal distances older first. Boolean mask over
+    hist."""
+    hist = np.asarray(hist)
+    key = sorted(range(hist.size),
+                 key=lambda j: (-grid_d2(int(hist[j]) - n_cond, t_ref, row_len), int(hist[j])))
+    mask = np.zeros(hist.size, dtype=bool)
+    mask[key[:n_long]] = True
+    return mask
+
+
 def ste_scores_eq6(Q_past, Ck) -> np.ndarray:
     """Eq. 6 as printed: (1/P) 1^T (Q_past Ck^T / sqrt(d)), fp64."""
     Q = np.asarray(Q_past, dtype=np.float64)
@@ -245,6 +318,24 @@ def ste_evict(scores, positions, n_long: int, M: int) -> np.ndarray:
     return evict
 
 
+def ste_evict_strata(scores, positions, is_long, M: int) -> np.ndarray:
+    """ste_evict with the long-range subset given as a mask over the history
+    tokens (any membership): the quotas of ste_quotas, each subset's lowest
+    scores evicted, equal scores older first."""
+    scores = np.asarray(scores)
+    positions = np.asarray(positions)
+    is_long = np.asarray(is_long, dtype=bool)
+    n_long = int(is_long.sum())
+    m_long, m_near = ste_quotas(M, n_long, scores.size - n_long)
+    evict = np.zeros(scores.size, dtype=bool)
+    for members, m in ((np.flatnonzero(is_long), m_long), (np.flatnonzero(~is_long), m_near)):
+        if m == 0:
+            continue
+        order = np.lexsort((positions[members], scores[members]))
+        evict[members[order[:m]]] = True
+    return evict
+
+
 # ----------------------------------------------------------------------------
 # Eqs. 2-4: head-aware cache update
 # ----------------------------------------------------------------------------
@@ -259,16 +350,19 @@ class HeadParams:
     global_budget: int
     tau: float
     r_s: float
+    row_len: int = 0
+    distance: int = RASTER   # GRID2D: the grid-distance variants of Step 2 and Eq. 5
 
     @property
     def hist_budget(self) -> int:
         return self.global_budget - self.recent_w
 
     @classmethod
-    def of(cls, w) -> "HeadParams":
+    def of(cls, w, distance: int = RASTER) -> "HeadParams":
         return cls(n_cond=w.n_cond, n_image=w.n_image, recent_w=w.recent_w,
                    local_w=w.w_loc, period=w.period, group_at=w.group_at,
-                   global_budget=global_budget(w.rho, w.n_image), tau=w.tau, r_s=w.r_s)
+                   global_budget=global_budget(w.rho, w.n_image), tau=w.tau, r_s=w.r_s,
+                   row_len=w.row_len, distance=distance)
 
 
 @dataclass
@@ -278,6 +372,7 @@ class UpdateRecord:
     n_long: int
     evicted: np.ndarray    # evicted positions (sorted)
     pos: np.ndarray        # retained positions after the update
+    long_pos: np.ndarray | None = None   # positions of the long-range subset
 
 
 def cache_update(pos: np.ndarray, label: int, hp: HeadParams, q, k, t_last: int,
@@ -294,6 +389,10 @@ def cache_update(pos: np.ndarray, label: int, hp: HeadParams, q, k, t_last: int,
     hist, recent = img[: img.size - n_recent], img[img.size - n_recent:]
     T = int(hist.size)
     n_long = ste_partition(T, hp.r_s)
+    if hp.distance == GRID2D:
+        is_long = ste_long_2d(hist, n_long, C, hp.row_len, t_last)
+    else:
+        is_long = np.arange(T) < n_long
     if label == LOCAL:
         evicted, kept = hist, hist[:0]
     elif T > hp.hist_budget:
@@ -302,12 +401,16 @@ def cache_update(pos: np.ndarray, label: int, hp: HeadParams, q, k, t_last: int,
         Q_past = q[t_last - P + 1: t_last + 1]
         Ck = k[hist]
         s = ste_scores_fp32(Q_past, Ck) if scores == "fp32" else ste_scores_eq6(Q_past, Ck)
-        ev = ste_evict(s, hist, n_long, M)
+        if hp.distance == GRID2D:
+            ev = ste_evict_strata(s, hist, is_long, M)
+        else:
+            ev = ste_evict(s, hist, n_long, M)
         evicted, kept = hist[ev], hist[~ev]
     else:
         evicted, kept = hist[:0], hist
     new_pos = np.concatenate([cond, kept, recent])
-    return UpdateRecord(t_last=t_last, T=T, n_long=n_long, evicted=evicted, pos=new_pos)
+    return UpdateRecord(t_last=t_last, T=T, n_long=n_long, evicted=evicted, pos=new_pos,
+                        long_pos=hist[is_long])
 
 
 @dataclass
@@ -354,7 +457,10 @@ def run_head(hp: HeadParams, q, k, v, *, label: int | None = None, record=(),
         if t in record_pos:
             tr.pos_at[t] = pos.copy()
         if t == E - 1:                        # Step 2: head grouping
-            n_h, cum = grouping_count(q[t], k[pos], hp.tau)
+            if hp.distance == GRID2D:
+                n_h, cum = grouping_count_2d(q[t], k[pos], hp.tau, C, hp.row_len)
+            else:
+                n_h, cum = grouping_count(q[t], k[pos], hp.tau)
             tr.n_h = n_h
             tr.label_computed = classify(n_h, hp.local_w)
             tr.margin = label_margin(cum, hp.tau, hp.local_w)

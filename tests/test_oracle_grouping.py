@@ -120,3 +120,57 @@ def test_multi_query_older_queries_do_not_see_newer_keys():
     n_h, cum = O.grouping_count_multi(Q, K, 0.9)
     assert abs(cum[0] - 0.5) < 1e-12 and abs(cum[-2] - 0.5) < 1e-12
     assert n_h == n            # tau needs the oldest key too: global for any w_loc <= n
+
+
+# Grid-distance variant (not in the paper): the count runs outward from the
+# current token by squared distance on the image grid.
+
+def test_grid_distance_hand_values():
+    assert O.grid_d2(6, 6, 4) == 0
+    assert O.grid_d2(6, 5, 4) == 1 and O.grid_d2(6, 2, 4) == 1     # left, above
+    assert O.grid_d2(6, 0, 4) == 5                                 # one up, two left
+    assert O.grid_d2(0, 15, 4) == 18                               # opposite corners of 4x4
+
+
+def test_count_order_2d_hand_worked():
+    # row_len 4, two conditioning tokens, image tokens 0..6; the newest (6)
+    # sits at (1, 2). Squared distances: 5 and 2 -> 1 (newer first: 5, 2),
+    # 3 and 1 -> 2 (3, 1), 4 -> 4, 0 -> 5; then conditioning 1, 0.
+    # Image token i has position i + 2.
+    order = O.count_order_2d(9, 2, 4)
+    assert order.tolist() == [8, 7, 4, 5, 3, 6, 2, 1, 0]
+
+
+def test_grid_count_sees_the_token_above_as_adjacent():
+    # row_len 5, one conditioning token, image tokens 0..7: the newest (7)
+    # at (1, 2); all attention on image token 2, directly above it. Raster:
+    # the count reaches it after 6 tokens (7, 6, 5, 4, 3, 2): global for
+    # w_loc = 4. Grid: 7, then the distance-1 tokens 6 (left) and 2 (above):
+    # 3 tokens, local.
+    D, C, row, n = 8, 1, 5, 9
+    K = np.zeros((n, D))
+    K[C + 2, 0] = 60 * math.sqrt(D)
+    q = np.zeros(D); q[0] = 1.0
+    n_r, _ = O.grouping_count(q, K, 0.9)
+    n_g, _ = O.grouping_count_2d(q, K, 0.9, C, row)
+    assert n_r == 6 and n_g == 3
+    assert O.classify(n_r, 4) == O.GLOBAL and O.classify(n_g, 4) == O.LOCAL
+
+
+def test_grid_count_uniform_equals_raster():
+    rng = np.random.default_rng(4)
+    for n, C, row in ((31, 3, 7), (101, 1, 24)):   # tau * n not an integer
+        K = rng.normal(size=(n, 16))
+        a = O.grouping_count(np.zeros(16), K, 0.9)
+        b = O.grouping_count_2d(np.zeros(16), K, 0.9, C, row)
+        assert a[0] == b[0] == math.ceil(0.9 * n - 1e-12)
+        assert np.allclose(a[1], b[1], rtol=0, atol=1e-13)
+
+
+def test_grid_count_multi_with_one_query():
+    rng = np.random.default_rng(5)
+    K = rng.normal(size=(40, 16))
+    q = rng.normal(size=16) * 3
+    a = O.grouping_count_2d(q, K, 0.9, 4, 6)
+    b = O.grouping_count_multi_2d(q[None, :], K, 0.9, 4, 6)
+    assert a[0] == b[0] and np.array_equal(a[1], b[1])

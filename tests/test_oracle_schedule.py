@@ -56,7 +56,21 @@ def check_invariants(hp, tr, label):
                     pre = np.concatenate([prev_img, np.arange(prev_img.max() + 1, C + n_img_total)])
                 hist = pre[: pre.size - min(w, pre.size)]
                 assert hist.size == rec.T
-                in_long = np.isin(rec.evicted, hist[: rec.n_long]).sum()
+                if hp.distance == O.GRID2D:
+                    # the n_long farthest from the newest image token on the
+                    # grid: nothing outside the subset is farther, and among
+                    # equally far tokens the older are inside
+                    d2 = {int(x): O.grid_d2(int(x) - C, rec.t_last, hp.row_len) for x in hist}
+                    lp = set(rec.long_pos.tolist())
+                    assert len(lp) == rec.n_long and lp <= set(hist.tolist())
+                    for a in lp:
+                        for b in set(hist.tolist()) - lp:
+                            assert (d2[a], -a) > (d2[b], -b)
+                    long_set = rec.long_pos
+                else:
+                    long_set = hist[: rec.n_long]
+                    assert np.array_equal(rec.long_pos, long_set)
+                in_long = np.isin(rec.evicted, long_set).sum()
                 m_long = min(M // 2, rec.n_long)
                 m_long = max(m_long, M - (rec.T - rec.n_long))
                 assert in_long == m_long
@@ -98,3 +112,33 @@ def test_label_injection_overrides_grouping():
     tr = O.run_head(hp, hi.q, hi.k, hi.v, label=O.GLOBAL)
     assert tr.label_computed == O.LOCAL and tr.label == O.GLOBAL
     assert tr.final_pos.size == w.n_cond + hp.global_budget + tr.nbuf
+
+
+@pytest.mark.parametrize("name", ["tiny", "janus_pro_7b", "lumina768"])
+def test_retention_invariants_grid_distance(name):
+    """The grid-distance variant (not in the paper) keeps every budget and
+    always-kept class; its long-range subset is the farthest on the grid."""
+    w = configs.ALL[name].with_(n_layers=1)
+    hp = O.HeadParams.of(w, distance=O.GRID2D)
+    pe, cq = gen.pe_table(w), gen.q_coef(w)
+    heads = range(w.n_heads) if name == "tiny" else (0, 3, 7, 12)
+    for h in heads:
+        hi = gen.HeadInputs(w, 0, 0, h, pe, cq)
+        tr = O.run_head(hp, hi.q, hi.k, hi.v, label=O.GLOBAL if h % 2 else None)
+        check_invariants(hp, tr, tr.label)
+        budget = hp.global_budget if tr.label == O.GLOBAL else w.recent_w
+        assert tr.final_pos.size == w.n_cond + budget + tr.nbuf
+
+
+@pytest.mark.parametrize("r_s", [0.0, 1.0])
+def test_grid_distance_with_one_stratum_is_raster(r_s):
+    """With a single stratum the partition cannot matter: with the same
+    labels the grid-distance variant retains exactly what Eq. 5 retains."""
+    w = configs.ALL["janus_pro_7b"].with_(n_layers=1, r_s=r_s)
+    pe, cq = gen.pe_table(w), gen.q_coef(w)
+    for h in (1, 4):
+        hi = gen.HeadInputs(w, 0, 0, h, pe, cq)
+        a = O.run_head(O.HeadParams.of(w), hi.q, hi.k, hi.v, label=O.GLOBAL)
+        b = O.run_head(O.HeadParams.of(w, distance=O.GRID2D), hi.q, hi.k, hi.v, label=O.GLOBAL)
+        assert np.array_equal(a.final_pos, b.final_pos)
+        assert [u.evicted.tolist() for u in a.updates] == [u.evicted.tolist() for u in b.updates]

@@ -124,3 +124,51 @@ def test_fp32_decision_ranks_like_eq6():
         np.testing.assert_allclose(s32 / (P * math.sqrt(w.head_dim)), s64,
                                    rtol=0, atol=1e-5 * np.abs(s64).max())
     assert mismatches <= 1
+
+
+# Grid-distance variant of Eq. 5 (not in the paper).
+
+def test_long_subset_2d_hand_worked():
+    # row_len 4, C = 2, newest image token 9 at (2, 1); history image
+    # tokens 0..5 (positions 2..7) at squared distances 5, 4, 5, 8, 2, 1.
+    # The 3 farthest: token 3 (8), then tokens 0 and 2 (5; older first).
+    hist = np.arange(2, 8)
+    mask = O.ste_long_2d(hist, 3, 2, 4, 9)
+    assert hist[mask].tolist() == [2, 4, 5]
+    # raster Eq. 5 would take the oldest three: positions 2, 3, 4
+
+
+def brute_force_evict_mask(scores, is_long, m_long, m_near):
+    lo = [i for i in range(len(scores)) if is_long[i]]
+    ne = [i for i in range(len(scores)) if not is_long[i]]
+    best, best_sum = None, None
+    for ev_l in itertools.combinations(lo, m_long):
+        for ev_n in itertools.combinations(ne, m_near):
+            s = sum(scores[i] for i in ev_l + ev_n)
+            if best_sum is None or s < best_sum:
+                best, best_sum = set(ev_l + ev_n), s
+    return best
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_strata_mask_matches_brute_force(seed):
+    rng = np.random.default_rng(100 + seed)
+    T = int(rng.integers(4, 10))
+    is_long = rng.permutation(T) < O.ste_partition(T, 0.5)
+    M = int(rng.integers(1, T))
+    scores = rng.permutation(T * 3)[:T].astype(np.float32)
+    pos = np.arange(10, 10 + T)
+    m_long, m_near = O.ste_quotas(M, int(is_long.sum()), T - int(is_long.sum()))
+    ev = O.ste_evict_strata(scores, pos, is_long, M)
+    assert set(np.nonzero(ev)[0]) == brute_force_evict_mask(list(scores), is_long, m_long, m_near)
+
+
+def test_strata_mask_of_the_oldest_is_eq5():
+    rng = np.random.default_rng(7)
+    for T in (5, 17, 64):
+        scores = rng.normal(size=T).astype(np.float32)
+        pos = np.sort(rng.choice(1000, size=T, replace=False))
+        n_long = O.ste_partition(T, 0.5)
+        for M in (1, T // 3, T - 1):
+            assert np.array_equal(O.ste_evict_strata(scores, pos, np.arange(T) < n_long, M),
+                                  O.ste_evict(scores, pos, n_long, M))
