@@ -285,12 +285,14 @@ def run_ours(args):
                          f"on {workers} processes"}
 
     redistribute = args.budget == "redistribute"
+    grid2d = args.distance == "grid2d"
     cfg = H.make_config(n_layers=L, n_seqs=S, n_heads=Hh, head_dim=D, dtype=w.dtype,
                         n_cond=w.n_cond, n_image=w.n_image, row_len=w.row_len,
                         recent_w=w.recent_w, local_w=w.w_loc, period=P, group_at=w.group_at,
                         rho=w.rho, tau=w.tau, r_s=w.r_s,
                         budget_mode=H.HKV_BUDGET_REDISTRIBUTE if redistribute else
-                        H.HKV_BUDGET_PAPER)
+                        H.HKV_BUDGET_PAPER,
+                        distance_mode=H.HKV_DIST_GRID2D if grid2d else H.HKV_DIST_RASTER)
     eng = Engine(cfg, dev)
     synth = DeviceSynth(w, dev)
     generate(eng, synth, last_step=t0 - 1)      # dense phase, grouping, compression, decode
@@ -448,7 +450,9 @@ def run_ours(args):
             "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
             "config": {**bench_config(w, world),
                        **({"budget": "redistributed (aggregate-preserving), arena "
-                                     f"{eng.total_tokens} tokens"} if redistribute else {})},
+                                     f"{eng.total_tokens} tokens"} if redistribute else {}),
+                       **({"distance": "grid (identification and Eq. 5 strata by squared "
+                                       "distance on the image grid)"} if grid2d else {})},
             "global_head_fraction": float((labels == 1).mean()),
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak,
@@ -691,10 +695,10 @@ def run_labels(args):
     step, and at the paper's grouping token E - 1 and at that late token the
     heads of every layer are identified (hkv_identify_heads) with tau in
     {0.85, 0.9, 0.95}, and at tau = 0.9 also by the multi-query variant
-    (hkv_identify_heads_multi). Reports the share of global heads, the
-    agreement of the labels between the two points, between thresholds and
-    between the two identifications, and the device time of each
-    identification over all layers."""
+    (hkv_identify_heads_multi) and the grid-distance one. Reports the share
+    of global heads, the agreement of the labels between the two points,
+    between thresholds and between the identifications, and the device time
+    of each identification over all layers."""
     import torch
 
     from paper_2605_20600_gb300 import hkv as H
@@ -707,11 +711,11 @@ def run_labels(args):
     L, S, Hh, D, E, N = w.n_layers, w.n_seqs, w.n_heads, w.head_dim, w.group_at, w.n_image
     late = min(N, 4 * E)
     wl = w.with_(group_at=late)
-    def mk(tau):
+    def mk(tau, distance=H.HKV_DIST_RASTER):
         return H.make_config(n_layers=L, n_seqs=S, n_heads=Hh, head_dim=D, dtype=w.dtype,
                              n_cond=w.n_cond, n_image=N, row_len=w.row_len, recent_w=w.recent_w,
                              local_w=w.w_loc, period=w.period, group_at=late, rho=w.rho,
-                             tau=tau, r_s=w.r_s)
+                             tau=tau, r_s=w.r_s, distance_mode=distance)
 
     cfg = mk(w.tau)
     eng = Engine(cfg, dev)
@@ -734,18 +738,18 @@ def run_labels(args):
             for layer in range(L):
                 H.hkv_identify_heads(c, eng.dense.c, layer, q[layer], lab, nh, eng.stream())
             labels[(t, tau)] = lab.cpu().numpy()
-        c = mk(w.tau)
         lab = torch.empty(n, dtype=torch.uint8, device=dev)
         nh = torch.empty(n, dtype=torch.int32, device=dev)
-        for kind in ("single", "multi"):
+        for kind in ("single", "multi", "grid"):
+            c = mk(w.tau, H.HKV_DIST_GRID2D if kind == "grid" else H.HKV_DIST_RASTER)
             for rep in range(3):  # the last of three repetitions is timed
                 ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
                 ev[0].record()
                 for layer in range(L):
-                    if kind == "single":
-                        H.hkv_identify_heads(c, eng.dense.c, layer, q[layer], lab, nh, eng.stream())
-                    else:
+                    if kind == "multi":
                         H.hkv_identify_heads_multi(c, eng.dense.c, layer, lab, nh, eng.stream())
+                    else:
+                        H.hkv_identify_heads(c, eng.dense.c, layer, q[layer], lab, nh, eng.stream())
                 ev[1].record()
             torch.cuda.synchronize()
             labels[(t, kind)] = lab.cpu().numpy()
@@ -774,6 +778,13 @@ def run_labels(args):
                                  "multi_early": times[(E - 1, "multi")],
                                  "single_late": times[(late - 1, "single")],
                                  "multi_late": times[(late - 1, "multi")]}},
+            "grid_distance": {
+                "global_fraction": {"early": g(labels[(E - 1, "grid")]),
+                                    "late": g(labels[(late - 1, "grid")])},
+                "early_late_agreement": agree(labels[(E - 1, "grid")], labels[(late - 1, "grid")]),
+                "agreement_with_raster": {"early": agree(labels[(E - 1, "grid")], labels[(E - 1, "single")]),
+                                          "late": agree(labels[(late - 1, "grid")], labels[(late - 1, "single")])},
+                "us_per_layer": {"early": times[(E - 1, "grid")], "late": times[(late - 1, "grid")]}},
             "note": "synthetic inputs (per-head query scale drawn log-uniform); the paper's "
                     "grouping accuracy is against its models' own attention maps"}
     print(json.dumps(line), flush=True)
@@ -793,6 +804,10 @@ def main():
                     help="compare decode attention with the padding and per-group strategies")
     ap.add_argument("--budget", default="paper", choices=["paper", "redistribute"],
                     help="budget rule: the paper's, or local heads' unused tokens to global heads")
+    ap.add_argument("--distance", default="raster", choices=["raster", "grid2d"],
+                    help="token distance of identification and Eq. 5: the paper's raster order, "
+                         "or squared distance on the image grid (a variant; the CPU baseline "
+                         "stays the raster oracle)")
     ap.add_argument("--grouping", action="store_true",
                     help="time the grouping step with identification separate and fused")
     ap.add_argument("--labels", action="store_true",

@@ -99,6 +99,8 @@ typedef struct {
   int32_t recent_w, local_w, period, group_at;
   int32_t global_budget;
   int32_t budget_mode;
+  int32_t distance_mode; /* HKV_DIST_RASTER or HKV_DIST_GRID2D */
+  int32_t reserved;      /* must be 0 */
   double tau, r_s;
 } hkv_config;
 
@@ -112,6 +114,21 @@ enum {
    * keeps H * B_g image tokens, as if every head kept B_g. A group without
    * global heads keeps the paper's budgets. */
   HKV_BUDGET_REDISTRIBUTE = 1
+};
+
+/* token distance of head identification and of Eq. 5 (hkv_config.distance_mode) */
+enum {
+  /* the paper's: Step 2 counts backward from the newest token in raster
+   * order, Eq. 5's long-range subset is the T r_s oldest history tokens */
+  HKV_DIST_RASTER = 0,
+  /* not in the paper: image token i sits in grid cell (i / row_len,
+   * i % row_len) and distances are squared Euclidean distances of cells.
+   * Step 2 counts the image tokens outward from the newest, nearest first
+   * (equal distances newer first), then the conditioning tokens newest
+   * first; Eq. 5's long-range subset is the floor(T r_s) history tokens
+   * farthest from the newest image token (equal distances older first).
+   * hkv_decode_step_identify does not take it (HKV_ERR_INVALID_ARG). */
+  HKV_DIST_GRID2D = 1
 };
 
 /*

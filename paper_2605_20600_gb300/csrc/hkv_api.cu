@@ -125,6 +125,8 @@ MethodArgs method_args(const hkv_config *cfg) {
   m.P = cfg->period;
   m.r_s = cfg->r_s;
   m.tau = (float)cfg->tau;
+  m.grid2d = cfg->distance_mode == HKV_DIST_GRID2D ? 1 : 0;
+  m.row_len = cfg->row_len;
   return m;
 }
 
@@ -254,6 +256,14 @@ hkv_status hkv_validate_config(const hkv_config *c) {
     return HKV_ERR_INVALID_ARG;
   if (c->budget_mode != HKV_BUDGET_PAPER && c->budget_mode != HKV_BUDGET_REDISTRIBUTE)
     return HKV_ERR_INVALID_ARG;
+  if ((c->distance_mode != HKV_DIST_RASTER && c->distance_mode != HKV_DIST_GRID2D) ||
+      c->reserved != 0)
+    return HKV_ERR_INVALID_ARG;
+  if (c->distance_mode == HKV_DIST_GRID2D) {  // squared grid distances fit 31 bits
+    const long long rows = (c->n_image + c->row_len - 1) / c->row_len;
+    if ((rows - 1) * (rows - 1) + (long long)(c->row_len - 1) * (c->row_len - 1) >= (1ll << 31))
+      return HKV_ERR_SHAPE;
+  }
   // a capacity (C + budget + P) stays an int32
   if ((long long)c->n_cond + (long long)c->n_heads * c->global_budget + c->period > 0x7fffffffLL)
     return HKV_ERR_SHAPE;
@@ -365,6 +375,8 @@ hkv_status hkv_decode_step_identify(const hkv_config *cfg, const hkv_cache *cach
                                     uint8_t *label_out, void *workspace, size_t ws_bytes,
                                     int flags, hkv_stream_t stream) {
   if (!label_out) return HKV_ERR_INVALID_ARG;
+  // the fused count is the raster one (the newest rows of the segment)
+  if (cfg && cfg->distance_mode != HKV_DIST_RASTER) return HKV_ERR_INVALID_ARG;
   return decode_step("decode_step_identify", cfg, cache, layer, q, k, v, out, label_out,
                      workspace, ws_bytes, flags, stream);
 }
@@ -396,8 +408,10 @@ hkv_status hkv_identify_heads(const hkv_config *cfg, const hkv_cache *cache, int
   DeviceState *st;
   HKV_TRY(device_state(&st));
   const int max_len = cfg->n_cond + cfg->group_at;
-  HKV_TRY(update_ready(st, cfg->head_dim, cfg->dtype,
-                       update_smem_bytes(max_segment(cfg), cfg->head_dim, cfg->period, cfg->dtype)));
+  const size_t upd = update_smem_bytes(max_segment(cfg), cfg->head_dim, cfg->period, cfg->dtype);
+  const size_t need = identify_smem_bytes(max_len, cfg->period,
+                                          cfg->distance_mode == HKV_DIST_GRID2D, false);
+  HKV_TRY(update_ready(st, cfg->head_dim, cfg->dtype, upd > need ? upd : need));
   const int hpl = heads_per_layer(cfg);
   return cuda_status(launch_identify(cache_args(cache), method_args(cfg), layer * hpl, hpl, q,
                                      label_out, nh_out, cfg->head_dim, cfg->dtype, max_len,
@@ -415,7 +429,8 @@ hkv_status hkv_identify_heads_multi(const hkv_config *cfg, const hkv_cache *cach
   HKV_TRY(device_state(&st));
   const int max_len = cfg->n_cond + cfg->group_at;
   const size_t upd = update_smem_bytes(max_segment(cfg), cfg->head_dim, cfg->period, cfg->dtype);
-  const size_t need = identify_multi_smem_bytes(max_len, cfg->period);
+  const size_t need = identify_smem_bytes(max_len, cfg->period,
+                                          cfg->distance_mode == HKV_DIST_GRID2D, true);
   HKV_TRY(update_ready(st, cfg->head_dim, cfg->dtype, upd > need ? upd : need));
   const int hpl = heads_per_layer(cfg);
   return cuda_status(launch_identify_multi(cache_args(cache), method_args(cfg), layer * hpl, hpl,

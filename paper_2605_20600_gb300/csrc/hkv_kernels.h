@@ -102,6 +102,8 @@ struct MethodArgs {
   int C, w, w_loc, P;  // a global head's history budget comes from its capacity
   double r_s;
   float tau;
+  int grid2d;   // grid-distance count of Step 2 and long-range subset of Eq. 5
+  int row_len;  // image tokens per grid row
 };
 
 constexpr int kCacheThreads = 256;
@@ -126,10 +128,11 @@ cudaError_t launch_init_dense(const CacheArgs &c, int nheads_total, int seg_toke
 cudaError_t launch_identify(const CacheArgs &c, const MethodArgs &m, int layer_base, int nheads,
                             const void *q, uint8_t *label_out, int32_t *nh_out, int D, int dtype,
                             int max_len, cudaStream_t s);
-// multi-query Step 2 over the ring's newest min(P, ntok) queries (the
-// kernel needs identify_multi_smem_bytes(max_len, P) of shared memory, at
-// most what update_prepare enabled)
-size_t identify_multi_smem_bytes(int max_len, int P);
+// shared memory of the identification kernels (single query, or multi:
+// the ring's newest min(P, ntok) queries) for dense segments of up to
+// max_len tokens; at most what update_prepare enabled
+size_t identify_smem_bytes(int max_len, int P, bool grid2d, bool multi);
+// multi-query Step 2 over the ring's newest min(P, ntok) queries
 cudaError_t launch_identify_multi(const CacheArgs &c, const MethodArgs &m, int layer_base,
                                   int nheads, uint8_t *label_out, int32_t *nh_out, int D,
                                   int dtype, int max_len, cudaStream_t s);

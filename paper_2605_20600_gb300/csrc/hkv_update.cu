@@ -220,9 +220,23 @@ __device__ int select_evictions(const SegRef &sg, int label, const MethodArgs &m
   else if (NH > hist_budget) M = NH - hist_budget;
 
   if (label == HKV_GLOBAL && M > 0) {
-    // Eq. 5: the floor(NH r_s) oldest history tokens are long-range
+    // Eq. 5: the floor(NH r_s) oldest history tokens are long-range (or,
+    // in the grid-distance variant, the farthest from the newest image
+    // token, equal distances older first)
     const int n_long = (int)floor((double)NH * m.r_s);
-    if (n_long > 0 && n_long < NH) {
+    if (n_long > 0 && n_long < NH && m.grid2d) {
+      const int ref = ntok - 1;
+      for (int r = tid; r < sg.len; r += NT) {
+        const int i = u.ps[r] - C;
+        const long long dr = i / m.row_len - ref / m.row_len, dc = i % m.row_len - ref % m.row_len;
+        const unsigned long long far = 0x7FFFFFFFull - (unsigned long long)(dr * dr + dc * dc);
+        u.keys[r] = (far << 32) | (uint32_t)u.ps[r];
+      }
+      radix_select2(u.keys, u.aux, sg.len, n_long, 0, 56, u.hist, sh);
+      const unsigned long long k_long = sh.prefix[0];
+      for (int r = tid; r < sg.len; r += NT)
+        if (u.aux[r] == 0) u.aux[r] = u.keys[r] <= k_long ? 0 : 1;
+    } else if (n_long > 0 && n_long < NH) {
       for (int r = tid; r < sg.len; r += NT) u.keys[r] = (unsigned long long)(uint32_t)u.ps[r];
       const int maxp = C + ntok;  // positions are below it: start at its top byte
       const int top = maxp < (1 << 8) ? 0 : maxp < (1 << 16) ? 8 : maxp < (1 << 24) ? 16 : 24;
@@ -635,9 +649,50 @@ __global__ void init_dense_kernel(const CacheArgs c, int n, int seg) {
   if (blockIdx.x == 0 && threadIdx.x == 0) *c.err = 0u;
 }
 
+// Shared memory of the identification kernels beyond their weights: in the
+// grid-distance variant, the order keys ([max_len] 64-bit, 8-byte aligned
+// after `floats` floats) and the count order ([max_len] int).
+__host__ __device__ constexpr size_t id_order_offset(size_t floats) {
+  return (floats * 4 + 7) / 8 * 8;
+}
+__host__ __device__ constexpr size_t id_smem(size_t floats, int max_len, bool grid2d) {
+  return grid2d ? id_order_offset(floats) + (size_t)max_len * 12 : floats * 4;
+}
+
+// The count order of the grid-distance variant of Step 2: perm[j] = the row
+// of the j-th token counted. Image tokens by squared grid distance from image
+// token ref, nearest first, equal distances newer first; then the
+// conditioning tokens, newest first. Keys are unique (positions are); each
+// row's rank is the number of smaller keys (len^2 / NT comparisons per
+// thread, once per head and generation). Block-uniform.
+__device__ void grid_count_order(const int32_t *pos, int len, int C, int row_len, int ref,
+                                 unsigned long long *keys, int *perm) {
+  for (int r = threadIdx.x; r < len; r += blockDim.x) {
+    const int p = pos[r];
+    const unsigned long long newer = 0xFFFFFFFFull - (uint32_t)p;
+    unsigned long long key = (1ull << 63) | newer;  // conditioning: after every image token
+    if (p >= C) {
+      const int i = p - C;
+      const long long dr = i / row_len - ref / row_len, dc = i % row_len - ref % row_len;
+      key = ((unsigned long long)(dr * dr + dc * dc) << 32) | newer;
+    }
+    keys[r] = key;
+    perm[r] = r;  // a valid row for every slot even if positions repeat
+  }
+  __syncthreads();
+  for (int r = threadIdx.x; r < len; r += blockDim.x) {
+    const unsigned long long k = keys[r];
+    int rank = 0;
+    for (int j = 0; j < len; ++j) rank += keys[j] < k ? 1 : 0;
+    perm[rank] = r;
+  }
+  __syncthreads();
+}
+
 // Step 2: attention of the current query over the key cache, accumulated
-// backward from the newest token until tau; local iff fewer than w_loc
-// tokens were needed. The dense cache holds its tokens in position order.
+// backward from the newest token until tau (or outward on the grid in the
+// grid-distance variant); local iff fewer than w_loc tokens were needed.
+// The dense cache holds its tokens in position order.
 template <int D, typename T>
 __global__ void __launch_bounds__(NT)
     identify_kernel(const CacheArgs c, const MethodArgs m, int layer_base, const void *q,
@@ -724,10 +779,17 @@ __global__ void __launch_bounds__(NT)
   }
   __syncthreads();
   const float thr = s_bcast;
-  float running = 0.f;  // backward cumulative mass from the newest token
+  int *perm = nullptr;
+  if (m.grid2d) {
+    unsigned char *base = reinterpret_cast<unsigned char *>(e) + id_order_offset(max_len);
+    perm = reinterpret_cast<int *>(base + (size_t)max_len * 8);
+    grid_count_order(c.pos + off, len, m.C, m.row_len, c.ntok[i] - 1,
+                     reinterpret_cast<unsigned long long *>(base), perm);
+  }
+  float running = 0.f;  // cumulative mass from the newest token
   for (int base = 0; base < len; base += NT) {
-    const int jb = base + tid;  // jb-th newest token (0 = current)
-    const float x = jb < len ? e[len - 1 - jb] : 0.f;
+    const int jb = base + tid;  // jb-th token counted (0 = current)
+    const float x = jb < len ? e[perm ? perm[jb] : len - 1 - jb] : 0.f;
     float tot;
     const float cum = running + block_excl_scan<float>(x, fscan, &tot) + x;
     if (jb < len && cum >= thr) atomicMin(&s_nh, jb + 1);
@@ -900,10 +962,18 @@ __global__ void __launch_bounds__(NT)
   const float thr = tot[0] * m.tau;
   if (tid == 0) s_nh = len;
   __syncthreads();
-  float running = 0.f;  // backward cumulative mass from the newest token
+  int *perm = nullptr;
+  if (m.grid2d) {
+    unsigned char *base =
+        reinterpret_cast<unsigned char *>(e) + id_order_offset((size_t)(QB + 1) * max_len);
+    perm = reinterpret_cast<int *>(base + (size_t)max_len * 8);
+    grid_count_order(c.pos + off, len, m.C, m.row_len, ntok - 1,
+                     reinterpret_cast<unsigned long long *>(base), perm);
+  }
+  float running = 0.f;  // cumulative mass from the newest token
   for (int base = 0; base < len; base += NT) {
-    const int jb = base + tid;  // jb-th newest token (0 = current)
-    const float x = jb < len ? pbar[len - 1 - jb] : 0.f;
+    const int jb = base + tid;  // jb-th token counted (0 = current)
+    const float x = jb < len ? pbar[perm ? perm[jb] : len - 1 - jb] : 0.f;
     float t;
     const float cum = running + block_excl_scan<float>(x, fscan, &t) + x;
     if (jb < len && cum >= thr) atomicMin(&s_nh, jb + 1);
@@ -1122,7 +1192,7 @@ cudaError_t launch_identify(const CacheArgs &c, const MethodArgs &m, int layer_b
                             const void *q, uint8_t *label_out, int32_t *nh_out, int D, int dtype,
                             int max_len, cudaStream_t s) {
   const float qscale = (float)(1.4426950408889634 / sqrt((double)D));
-  const size_t smem = (size_t)max_len * 4;
+  const size_t smem = identify_smem_bytes(max_len, m.P, m.grid2d != 0, false);
   HKV_DISPATCH(D, dtype,
                return pdl_launch(identify_kernel<kD, kT>, nheads, NT, smem, s, c, m, layer_base,
                                  q, label_out, nh_out, qscale, max_len));
@@ -1133,7 +1203,7 @@ cudaError_t launch_identify_multi(const CacheArgs &c, const MethodArgs &m, int l
                                   int nheads, uint8_t *label_out, int32_t *nh_out, int D,
                                   int dtype, int max_len, cudaStream_t s) {
   const float qscale = (float)(1.4426950408889634 / sqrt((double)D));
-  const size_t smem = identify_multi_smem_bytes(max_len, m.P);
+  const size_t smem = identify_smem_bytes(max_len, m.P, m.grid2d != 0, true);
   if (id_qb(m.P) == 8) {
     HKV_DISPATCH(D, dtype,
                  return pdl_launch(identify_multi_kernel<kD, kT, 8>, nheads, NT, smem, s, c, m,
@@ -1146,8 +1216,9 @@ cudaError_t launch_identify_multi(const CacheArgs &c, const MethodArgs &m, int l
   return cudaErrorInvalidValue;
 }
 
-size_t identify_multi_smem_bytes(int max_len, int P) {
-  return (size_t)(id_qb(P) + 1) * 4 * max_len;
+size_t identify_smem_bytes(int max_len, int P, bool grid2d, bool multi) {
+  const size_t floats = multi ? (size_t)(id_qb(P) + 1) * max_len : (size_t)max_len;
+  return id_smem(floats, max_len, grid2d);
 }
 
 cudaError_t launch_budgets(const uint8_t *label, int32_t *budget, int32_t *cap, int64_t *off,

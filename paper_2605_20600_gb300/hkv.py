@@ -31,6 +31,7 @@ HKV_FP32, HKV_BF16 = 0, 1
 HKV_STEP_PREFETCH = 1
 HKV_LOCAL, HKV_GLOBAL, HKV_DENSE = 0, 1, 255
 HKV_BUDGET_PAPER, HKV_BUDGET_REDISTRIBUTE = 0, 1
+HKV_DIST_RASTER, HKV_DIST_GRID2D = 0, 1
 
 
 class hkv_config(Structure):
@@ -38,7 +39,8 @@ class hkv_config(Structure):
         ("n_layers", c_int32), ("n_seqs", c_int32), ("n_heads", c_int32), ("head_dim", c_int32),
         ("dtype", c_int32), ("n_cond", c_int32), ("n_image", c_int32), ("row_len", c_int32),
         ("recent_w", c_int32), ("local_w", c_int32), ("period", c_int32), ("group_at", c_int32),
-        ("global_budget", c_int32), ("budget_mode", c_int32), ("tau", c_double), ("r_s", c_double),
+        ("global_budget", c_int32), ("budget_mode", c_int32), ("distance_mode", c_int32),
+        ("reserved", c_int32), ("tau", c_double), ("r_s", c_double),
     ]
 
 
@@ -123,7 +125,8 @@ def hkv_status_str(status: int) -> str:
 
 def make_config(*, n_layers, n_seqs, n_heads, head_dim, dtype, n_cond, n_image, row_len,
                 recent_w, local_w, period, group_at, rho=None, global_budget=None,
-                tau=0.9, r_s=0.5, budget_mode=HKV_BUDGET_PAPER) -> hkv_config:
+                tau=0.9, r_s=0.5, budget_mode=HKV_BUDGET_PAPER,
+                distance_mode=HKV_DIST_RASTER) -> hkv_config:
     """Builds an hkv_config; the global budget is floor(rho * N) (Sec. 5.1)
     unless given explicitly."""
     if global_budget is None:
@@ -131,7 +134,8 @@ def make_config(*, n_layers, n_seqs, n_heads, head_dim, dtype, n_cond, n_image, 
     return hkv_config(n_layers, n_seqs, n_heads, head_dim,
                       HKV_BF16 if dtype in ("bf16", HKV_BF16) else HKV_FP32,
                       n_cond, n_image, row_len, recent_w, local_w, period, group_at,
-                      int(global_budget), int(budget_mode), float(tau), float(r_s))
+                      int(global_budget), int(budget_mode), int(distance_mode), 0, float(tau),
+                      float(r_s))
 
 
 def hkv_validate_config(cfg: hkv_config) -> None:

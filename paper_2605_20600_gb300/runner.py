@@ -27,10 +27,11 @@ def generate(engine: Engine, provider, *, last_step: int | None = None, on_step=
     decode step (fused path only; no n_h), "separate" runs
     hkv_identify_heads after it (labels and n_h), "multi" runs
     hkv_identify_heads_multi after it (the recent queries' averaged
-    attention; labels and n_h). Default: fused when the path is fused.
+    attention; labels and n_h). Default: fused when the path is fused and
+    the distances are the raster ones.
     """
-    if identify is None:
-        identify = "fused" if fused else "separate"
+    if identify is None:   # the fused count is the raster one
+        identify = "fused" if fused and engine.cfg.distance_mode == 0 else "separate"
     if identify not in ("fused", "separate", "multi") or (identify == "fused" and not fused):
         raise ValueError(f"identify={identify!r} with fused={fused}")
     cfg = engine.cfg

@@ -12,12 +12,12 @@ from oracle import headkv as O
 from synth import configs, gen
 
 
-def cfg_of(H, w: configs.Workload, budget_mode=0):
+def cfg_of(H, w: configs.Workload, budget_mode=0, distance_mode=0):
     return H.make_config(n_layers=w.n_layers, n_seqs=w.n_seqs, n_heads=w.n_heads,
                          head_dim=w.head_dim, dtype=w.dtype, n_cond=w.n_cond, n_image=w.n_image,
                          row_len=w.row_len, recent_w=w.recent_w, local_w=w.w_loc,
                          period=w.period, group_at=w.group_at, rho=w.rho, tau=w.tau, r_s=w.r_s,
-                         budget_mode=budget_mode)
+                         budget_mode=budget_mode, distance_mode=distance_mode)
 
 
 def flat(w, s, l, h):
@@ -25,7 +25,7 @@ def flat(w, s, l, h):
 
 
 def run_gpu(w, *, out_steps=(), pos_steps=(), pos_heads=(), last_step=None, fused=True,
-            out_heads=None, identify="separate", budget_mode=0):
+            out_heads=None, identify="separate", budget_mode=0, distance_mode=0):
     """One generation on the GPU. Returns outputs {t: [L,S,H,D] fp32, or
     {(s, l, h): [D]} for out_heads}, positions {t: {flat head: sorted
     positions}}, labels, n_h (None when the identification is fused into
@@ -36,7 +36,7 @@ def run_gpu(w, *, out_steps=(), pos_steps=(), pos_heads=(), last_step=None, fuse
     from paper_2605_20600_gb300.runner import generate
     from synth.gpu import DeviceSynth
 
-    eng = Engine(cfg_of(H, w, budget_mode), "cuda")
+    eng = Engine(cfg_of(H, w, budget_mode, distance_mode), "cuda")
     out_steps, pos_steps = set(out_steps), set(pos_steps)
     outs, poss = {}, {}
 
@@ -66,24 +66,25 @@ def run_gpu(w, *, out_steps=(), pos_steps=(), pos_heads=(), last_step=None, fuse
 
 
 def _oracle_job(args):
-    w, s, l, h, label, record, record_pos, budget = args
+    w, s, l, h, label, record, record_pos, budget, distance = args
     pe, cq = gen.pe_table(w), gen.q_coef(w)
     hi = gen.HeadInputs(w, s, l, h, pe, cq)
-    hp = O.HeadParams.of(w)
+    hp = O.HeadParams.of(w, distance)
     if budget is not None and label == O.GLOBAL:   # a per-head budget (redistributed)
         hp = dataclasses.replace(hp, global_budget=budget)
     tr = O.run_head(hp, hi.q, hi.k, hi.v, label=label, record=record, record_pos=record_pos)
     return (s, l, h), tr
 
 
-def oracle_heads(w, heads, labels=None, record=(), record_pos=(), budgets=None):
+def oracle_heads(w, heads, labels=None, record=(), record_pos=(), budgets=None, distance=0):
     """Oracle traces of the given (s, l, h) heads; labels (flat array) are
     injected when given, and so are per-head image-token budgets (flat
     array, used for global heads). Runs in a spawn pool (safe after CUDA
     init)."""
     jobs = [(w, s, l, h, None if labels is None else int(labels[flat(w, s, l, h)]),
              tuple(record), tuple(record_pos),
-             None if budgets is None else int(budgets[flat(w, s, l, h)])) for (s, l, h) in heads]
+             None if budgets is None else int(budgets[flat(w, s, l, h)]), distance)
+            for (s, l, h) in heads]
     if len(jobs) <= 2:
         return dict(map(_oracle_job, jobs))
     n = min(len(jobs), os.cpu_count() or 1, 16)
@@ -93,8 +94,9 @@ def oracle_heads(w, heads, labels=None, record=(), record_pos=(), budgets=None):
 
 def label_job(args):
     """Oracle grouping for heads of one (s, l): (label, n_h, margin) per head;
-    multi: from the newest min(P, E) queries (grouping_count_multi)."""
-    w, s, l, heads, multi = args
+    multi: from the newest min(P, E) queries (grouping_count_multi);
+    distance: O.GRID2D counts outward on the grid."""
+    w, s, l, heads, multi, distance = args
     pe, cq = gen.pe_table(w), gen.q_coef(w)
     hp = O.HeadParams.of(w)
     res = []
@@ -102,17 +104,21 @@ def label_job(args):
         hi = gen.HeadInputs(w, s, l, h, pe, cq)
         t = w.group_at - 1
         K = hi.k[: w.n_cond + t + 1]
-        if multi:
-            Q = hi.q[max(0, t + 1 - w.period): t + 1]
+        Q = hi.q[max(0, t + 1 - w.period): t + 1]
+        if multi and distance == O.GRID2D:
+            n_h, cum = O.grouping_count_multi_2d(Q, K, w.tau, w.n_cond, w.row_len)
+        elif multi:
             n_h, cum = O.grouping_count_multi(Q, K, w.tau)
+        elif distance == O.GRID2D:
+            n_h, cum = O.grouping_count_2d(hi.q[t], K, w.tau, w.n_cond, w.row_len)
         else:
             n_h, cum = O.grouping_count(hi.q[t], K, w.tau)
         res.append((O.classify(n_h, w.w_loc), n_h, O.label_margin(cum, w.tau, w.w_loc)))
     return (s, l), res
 
 
-def oracle_labels(w, layers, seqs, multi=False):
-    jobs = [(w, s, l, tuple(range(w.n_heads)), multi) for l in layers for s in seqs]
+def oracle_labels(w, layers, seqs, multi=False, distance=0):
+    jobs = [(w, s, l, tuple(range(w.n_heads)), multi, distance) for l in layers for s in seqs]
     n = min(len(jobs), os.cpu_count() or 1, 16)
     with mp.get_context("spawn").Pool(n) as pool:
         return dict(pool.map(label_job, jobs, chunksize=1))

@@ -55,7 +55,7 @@ def test_every_declared_symbol_is_exported(H):
 
 
 def test_struct_sizes(H):
-    assert ctypes.sizeof(H.hkv_config) == 14 * 4 + 2 * 8
+    assert ctypes.sizeof(H.hkv_config) == 16 * 4 + 2 * 8
     assert ctypes.sizeof(H.hkv_cache) == 11 * 8 + 8
 
 
@@ -68,7 +68,9 @@ def test_status_strings(H):
 @pytest.mark.parametrize("change,code", [
     (dict(head_dim=96), 2), (dict(dtype=5), 1), (dict(period=32), 2), (dict(global_budget=8), 2),
     (dict(global_budget=65), 2), (dict(group_at=65), 2), (dict(n_seqs=0), 2), (dict(tau=0.0), 1),
-    (dict(r_s=1.5), 1), (dict(budget_mode=2), 1),
+    (dict(r_s=1.5), 1), (dict(budget_mode=2), 1), (dict(distance_mode=2), 1), (dict(reserved=1), 1),
+    # squared grid distances of a 50000 x 1 grid do not fit 31 bits
+    (dict(distance_mode=1, row_len=1, n_image=50000), 2),
 ])
 def test_validate_config_rejects(H, change, code):
     cfg = tiny_cfg(H)
@@ -139,6 +141,11 @@ def test_null_and_misaligned_arguments(H):
                                         16, 1 << 30, 0, None) == 1
     assert lib.hkv_decode_step_identify(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, 16, 16, 16,
                                         16, 8, 0, None) == 3
+    grid = tiny_cfg(H)
+    grid.distance_mode = 1
+    H.hkv_validate_config(grid)
+    assert lib.hkv_decode_step_identify(ctypes.byref(grid), ctypes.byref(c), 0, 16, 16, 16, 16, 16,
+                                        16, 1 << 30, 0, None) == 1
     nopos = fake_cache(H, pos=None)
     assert lib.hkv_export_state(ctypes.byref(cfg), ctypes.byref(nopos), 0, None, None, None, None,
                                 16, 8, ctypes.byref(cnt), None) == 1

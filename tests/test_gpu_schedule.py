@@ -109,20 +109,23 @@ def test_hand_worked_grid_fused_identification():
         assert int(labels[h]) == hd["expected"]["label"], hd["name"]
 
 
-@pytest.mark.parametrize("fused,identify", [(True, "separate"), (False, "separate"),
-                                            (True, "fused"), (True, "multi")])
-def test_tiny_every_step_every_head(fused, identify):
+@pytest.mark.parametrize("fused,identify,distance", [
+    (True, "separate", O.RASTER), (False, "separate", O.RASTER), (True, "fused", O.RASTER),
+    (True, "multi", O.RASTER),
+    # the grid-distance variants of Step 2 and Eq. 5
+    (True, "separate", O.GRID2D), (False, "separate", O.GRID2D)])
+def test_tiny_every_step_every_head(fused, identify, distance):
     w = configs.TINY
     N = w.n_image
     heads = [(0, 0, h) for h in range(w.n_heads)]
     outs, poss, labels, nh, eng = run_gpu(w, out_steps=range(N), pos_steps=range(N),
                                           pos_heads=[flat(w, *x) for x in heads], fused=fused,
-                                          identify=identify)
-    lab = oracle_labels(w, [0], [0], multi=identify == "multi")
+                                          identify=identify, distance_mode=distance)
+    lab = oracle_labels(w, [0], [0], multi=identify == "multi", distance=distance)
     ties = check_labels(w, labels, nh, lab, "tiny")
     assert not ties
     assert labels.tolist() == [0, 0, 0, 0, 1, 1, 1, 1]
-    tr = oracle_heads(w, heads, labels, record=range(N), record_pos=range(N))
+    tr = oracle_heads(w, heads, labels, record=range(N), record_pos=range(N), distance=distance)
     worst = 0.0
     for (s, l, h) in heads:
         t_r = tr[(s, l, h)]
@@ -177,6 +180,33 @@ def test_model_shapes_two_layers_two_seqs(name, rho, fused, identify):
         # retained budget after the last update
         budget = O.global_budget(w.rho, w.n_image) if labels[i] == 1 else w.recent_w
         assert poss[w.n_image - 1][i].size == w.n_cond + budget + t_r.nbuf
+    assert worst <= TOL[w.dtype], worst
+
+
+@pytest.mark.parametrize("name,rho", [("lumina768", "1/4"), ("llamagen_xl", "1/6"),
+                                      ("janus_pro_7b", "1/8")])
+def test_grid_distance_two_layers_two_seqs(name, rho):
+    """The grid-distance variants (not in the paper): head types counted
+    outward on the image grid and Eq. 5's long-range subset the farthest on
+    it; labels, n_h, positions and outputs against the oracle run the same
+    way."""
+    from fractions import Fraction
+    w = configs.ALL[name].with_(n_layers=2, n_seqs=2, rho=Fraction(rho))
+    steps = sampled_steps(w, np.random.default_rng(43))
+    heads = [(s, l, h) for l in range(w.n_layers) for s in range(w.n_seqs) for h in range(w.n_heads)]
+    outs, poss, labels, nh, eng = run_gpu(w, out_steps=steps, pos_steps=steps,
+                                          pos_heads=[flat(w, *x) for x in heads],
+                                          distance_mode=O.GRID2D)
+    lab = oracle_labels(w, range(w.n_layers), range(w.n_seqs), distance=O.GRID2D)
+    ties = check_labels(w, labels, nh, lab, f"{name} grid")
+    assert len(ties) <= 2, ties
+    tr = oracle_heads(w, heads, labels, record=steps, record_pos=steps, distance=O.GRID2D)
+    worst = 0.0
+    for (s, l, h) in heads:
+        t_r, i = tr[(s, l, h)], flat(w, s, l, h)
+        for t in steps:
+            assert np.array_equal(poss[t][i], t_r.pos_at[t]), (name, s, l, h, t)
+            worst = max(worst, float(np.abs(outs[t][l, s, h] - t_r.outputs[t]).max()))
     assert worst <= TOL[w.dtype], worst
 
 
