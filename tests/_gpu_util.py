@@ -25,11 +25,13 @@ def flat(w, s, l, h):
 
 
 def run_gpu(w, *, out_steps=(), pos_steps=(), pos_heads=(), last_step=None, fused=True,
-            out_heads=None, identify="separate", budget_mode=0, distance_mode=0):
+            out_heads=None, identify="separate", budget_mode=0, distance_mode=0,
+            force_labels=None):
     """One generation on the GPU. Returns outputs {t: [L,S,H,D] fp32, or
     {(s, l, h): [D]} for out_heads}, positions {t: {flat head: sorted
     positions}}, labels, n_h (None when the identification is fused into
-    the grouping step, which gives no n_h) and the engine."""
+    the grouping step, which gives no n_h) and the engine. force_labels (a
+    flat array) replaces the labels after grouping, before compression."""
     import torch
     from paper_2605_20600_gb300 import hkv as H
     from paper_2605_20600_gb300.engine import Engine
@@ -57,8 +59,12 @@ def run_gpu(w, *, out_steps=(), pos_steps=(), pos_heads=(), last_step=None, fuse
             poss[t] = {i: np.sort(allpos[int(off[i]): int(off[i]) + int(ln[i])].cpu().numpy())
                        for i in pos_heads}
 
+    def before_compress(e):
+        if force_labels is not None:
+            e.labels.copy_(torch.as_tensor(np.asarray(force_labels, dtype=np.uint8), device="cuda"))
+
     generate(eng, DeviceSynth(w, "cuda"), on_step=on_step, last_step=last_step, fused=fused,
-             identify=identify)
+             identify=identify, before_compress=before_compress)
     torch.cuda.synchronize()
     eng.check()
     nh = eng.n_h.cpu().numpy() if identify in ("separate", "multi") else None
