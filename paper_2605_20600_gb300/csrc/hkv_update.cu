@@ -649,6 +649,18 @@ __global__ void init_dense_kernel(const CacheArgs c, int n, int seg) {
   if (blockIdx.x == 0 && threadIdx.x == 0) *c.err = 0u;
 }
 
+// Row steps of the identification kernels' logit loops whose key loads are
+// issued before the first is used (one step at a time costs a memory round
+// trip per step). Measured on a GB300 (one call per layer): dense segments
+// of 628 tokens or more go faster with 8 (single query; 26 -> 14 us per
+// layer at 628) or 4 (multi-query: -19 % at 628, -35 % at 2128 tokens) than
+// with one; segments of 101-164 tokens go best with 2, where more loads in
+// flight cost registers and resident CTAs.
+constexpr int kIdLongSegment = 512;
+__host__ __device__ constexpr int id_rows_in_flight(int max_len, bool multi) {
+  return max_len >= kIdLongSegment ? (multi ? 4 : 8) : 2;
+}
+
 // Shared memory of the identification kernels beyond their weights: in the
 // grid-distance variant, the order keys ([max_len] 64-bit, 8-byte aligned
 // after `floats` floats) and the count order ([max_len] int).
@@ -693,7 +705,7 @@ __device__ void grid_count_order(const int32_t *pos, int len, int C, int row_len
 // backward from the newest token until tau (or outward on the grid in the
 // grid-distance variant); local iff fewer than w_loc tokens were needed.
 // The dense cache holds its tokens in position order.
-template <int D, typename T>
+template <int D, typename T, int U>
 __global__ void __launch_bounds__(NT)
     identify_kernel(const CacheArgs c, const MethodArgs m, int layer_base, const void *q,
                     uint8_t *label_out, int32_t *nh_out, float qscale, int max_len) {
@@ -733,18 +745,27 @@ __global__ void __launch_bounds__(NT)
 #pragma unroll
   for (int x = 0; x < EPL; ++x) qf[x] *= qscale;
   const unsigned char *K = static_cast<const unsigned char *>(c.K) + off * RB;
-  for (int r0 = warp * RPW; r0 < len; r0 += NW * RPW) {  // logits (log2 units)
-    const int r = r0 + grp;
-    float dot = 0.f;
-    if (r < len) {
-      float kf[EPL];
-      Elem<T>::unpack(*reinterpret_cast<const uint4 *>(K + (size_t)r * RB + col * 16), kf);
+  // logits (log2 units); U row steps load before any is used
+  for (int r0 = warp * RPW; r0 < len; r0 += U * NW * RPW) {
+    uint4 kr[U];
 #pragma unroll
-      for (int x = 0; x < EPL; ++x) dot = fmaf(qf[x], kf[x], dot);
+    for (int u = 0; u < U; ++u) {
+      const int r = r0 + u * NW * RPW + grp;
+      kr[u] = r < len ? *reinterpret_cast<const uint4 *>(K + (size_t)r * RB + col * 16)
+                      : make_uint4(0u, 0u, 0u, 0u);
     }
 #pragma unroll
-    for (int o = LPR / 2; o >= 1; o >>= 1) dot += __shfl_xor_sync(0xFFFFFFFFu, dot, o);
-    if (r < len && col == 0) e[r] = dot;
+    for (int u = 0; u < U; ++u) {
+      const int r = r0 + u * NW * RPW + grp;
+      float kf[EPL];
+      Elem<T>::unpack(kr[u], kf);
+      float dot = 0.f;
+#pragma unroll
+      for (int x = 0; x < EPL; ++x) dot = fmaf(qf[x], kf[x], dot);
+#pragma unroll
+      for (int o = LPR / 2; o >= 1; o >>= 1) dot += __shfl_xor_sync(0xFFFFFFFFu, dot, o);
+      if (r < len && col == 0) e[r] = dot;
+    }
   }
   __syncthreads();
   float mx = -INFINITY;
@@ -835,7 +856,10 @@ __device__ __forceinline__ void block_all(float (&v)[N], float *red, float *bc) 
 // 8 is 17 % faster on 65-query rings over 628 keys, 4 is 26-33 % faster on
 // 24-query rings over 101-164 keys, where the fewer registers of 4 give
 // more CTAs per SM)
-constexpr int kIdQB8From = 48;
+#ifndef HKV_ID_QB8_FROM
+#define HKV_ID_QB8_FROM 48
+#endif
+constexpr int kIdQB8From = HKV_ID_QB8_FROM;
 __host__ __device__ constexpr int id_qb(int P) { return P >= kIdQB8From ? 8 : 4; }
 
 // Multi-query variant of Step 2 (not in the paper): the newest Pe = min(P,
@@ -845,7 +869,7 @@ __host__ __device__ constexpr int id_qb(int P) { return P >= kIdQB8From ? 8 : 4;
 // accumulated backward from the newest token until tau, as in
 // identify_kernel. One CTA per head; each pass over the keys serves QB
 // queries (every key row loaded once per pass, dotted with all of them).
-template <int D, typename T, int QB>
+template <int D, typename T, int QB, int U>
 __global__ void __launch_bounds__(NT)
     identify_multi_kernel(const CacheArgs c, const MethodArgs m, int layer_base,
                           uint8_t *label_out, int32_t *nh_out, float qscale, int max_len) {
@@ -901,24 +925,33 @@ __global__ void __launch_bounds__(NT)
       for (int x = 0; x < EPL; ++x) qf[b][x] = p < Pe ? qf[b][x] * qscale : 0.f;
     }
     const int mmax = len - max(0, Pe - 1 - (p0 + QB - 1));  // keys of the pass's newest query
-    for (int r0 = warp * RPW; r0 < mmax; r0 += NW * RPW) {  // logits (log2 units)
-      const int r = r0 + grp;
-      float dot[QB];
+    // logits (log2 units); U row steps load before any is used
+    for (int r0 = warp * RPW; r0 < mmax; r0 += U * NW * RPW) {
+      uint4 kr[U];
 #pragma unroll
-      for (int b = 0; b < QB; ++b) dot[b] = 0.f;
-      if (r < mmax) {
-        float kf[EPL];
-        Elem<T>::unpack(*reinterpret_cast<const uint4 *>(K + (size_t)r * RB + col * 16), kf);
-#pragma unroll
-        for (int b = 0; b < QB; ++b)
-#pragma unroll
-          for (int x = 0; x < EPL; ++x) dot[b] = fmaf(qf[b][x], kf[x], dot[b]);
+      for (int u = 0; u < U; ++u) {
+        const int r = r0 + u * NW * RPW + grp;
+        kr[u] = r < mmax ? *reinterpret_cast<const uint4 *>(K + (size_t)r * RB + col * 16)
+                         : make_uint4(0u, 0u, 0u, 0u);
       }
 #pragma unroll
-      for (int b = 0; b < QB; ++b) {
+      for (int u = 0; u < U; ++u) {
+        const int r = r0 + u * NW * RPW + grp;
+        float kf[EPL];
+        Elem<T>::unpack(kr[u], kf);
+        float dot[QB];
 #pragma unroll
-        for (int o = LPR / 2; o >= 1; o >>= 1) dot[b] += __shfl_xor_sync(0xFFFFFFFFu, dot[b], o);
-        if (col == 0 && r < mq[b]) e[b * max_len + r] = dot[b];
+        for (int b = 0; b < QB; ++b) {
+          dot[b] = 0.f;
+#pragma unroll
+          for (int x = 0; x < EPL; ++x) dot[b] = fmaf(qf[b][x], kf[x], dot[b]);
+        }
+#pragma unroll
+        for (int b = 0; b < QB; ++b) {
+#pragma unroll
+          for (int o = LPR / 2; o >= 1; o >>= 1) dot[b] += __shfl_xor_sync(0xFFFFFFFFu, dot[b], o);
+          if (col == 0 && r < mq[b]) e[b * max_len + r] = dot[b];
+        }
       }
     }
     __syncthreads();
@@ -1051,15 +1084,15 @@ cudaError_t prepare_t(size_t smem) {
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(repack_kernel<D, T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(identify_kernel<D, T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(identify_multi_kernel<D, T, 4>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(identify_multi_kernel<D, T, 8>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  const void *ident[] = {(const void *)identify_kernel<D, T, 2>,
+                         (const void *)identify_kernel<D, T, 8>,
+                         (const void *)identify_multi_kernel<D, T, 4, 2>,
+                         (const void *)identify_multi_kernel<D, T, 4, 4>,
+                         (const void *)identify_multi_kernel<D, T, 8, 2>,
+                         (const void *)identify_multi_kernel<D, T, 8, 4>};
+  for (const void *f : ident)
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   // all of an SM's L1 as shared memory, so that every head of a layer (one
   // CTA each) is resident at once
   if (e == cudaSuccess)
@@ -1193,8 +1226,13 @@ cudaError_t launch_identify(const CacheArgs &c, const MethodArgs &m, int layer_b
                             int max_len, cudaStream_t s) {
   const float qscale = (float)(1.4426950408889634 / sqrt((double)D));
   const size_t smem = identify_smem_bytes(max_len, m.P, m.grid2d != 0, false);
+  if (id_rows_in_flight(max_len, false) == 8) {
+    HKV_DISPATCH(D, dtype,
+                 return pdl_launch(identify_kernel<kD, kT, 8>, nheads, NT, smem, s, c, m,
+                                   layer_base, q, label_out, nh_out, qscale, max_len));
+  }
   HKV_DISPATCH(D, dtype,
-               return pdl_launch(identify_kernel<kD, kT>, nheads, NT, smem, s, c, m, layer_base,
+               return pdl_launch(identify_kernel<kD, kT, 2>, nheads, NT, smem, s, c, m, layer_base,
                                  q, label_out, nh_out, qscale, max_len));
   return cudaErrorInvalidValue;
 }
@@ -1204,15 +1242,16 @@ cudaError_t launch_identify_multi(const CacheArgs &c, const MethodArgs &m, int l
                                   int dtype, int max_len, cudaStream_t s) {
   const float qscale = (float)(1.4426950408889634 / sqrt((double)D));
   const size_t smem = identify_smem_bytes(max_len, m.P, m.grid2d != 0, true);
-  if (id_qb(m.P) == 8) {
-    HKV_DISPATCH(D, dtype,
-                 return pdl_launch(identify_multi_kernel<kD, kT, 8>, nheads, NT, smem, s, c, m,
-                                   layer_base, label_out, nh_out, qscale, max_len));
-  } else {
-    HKV_DISPATCH(D, dtype,
-                 return pdl_launch(identify_multi_kernel<kD, kT, 4>, nheads, NT, smem, s, c, m,
-                                   layer_base, label_out, nh_out, qscale, max_len));
-  }
+  const bool q8 = id_qb(m.P) == 8, u4 = id_rows_in_flight(max_len, true) == 4;
+#define HKV_ID_MULTI(QB_, U_)                                                                  \
+  HKV_DISPATCH(D, dtype,                                                                       \
+               return pdl_launch(identify_multi_kernel<kD, kT, QB_, U_>, nheads, NT, smem, s, c, \
+                                 m, layer_base, label_out, nh_out, qscale, max_len))
+  if (q8 && u4) HKV_ID_MULTI(8, 4);
+  if (q8) HKV_ID_MULTI(8, 2);
+  if (u4) HKV_ID_MULTI(4, 4);
+  HKV_ID_MULTI(4, 2);
+#undef HKV_ID_MULTI
   return cudaErrorInvalidValue;
 }
 
