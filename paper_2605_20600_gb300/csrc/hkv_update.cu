@@ -916,13 +916,15 @@ __global__ void __launch_bounds__(NT)
     for (int b = 0; b < QB; ++b) {
       const int p = p0 + b;
       mq[b] = p < Pe ? len - (Pe - 1 - p) : 0;
+#pragma unroll
+      for (int x = 0; x < EPL; ++x) qf[b][x] = 0.f;
       if (p < Pe) {
         const int slot = (ntok - Pe + p) % m.P;
         Elem<T>::unpack(*reinterpret_cast<const uint4 *>(ring + (size_t)slot * RB + col * 16),
                         qf[b]);
-      }
 #pragma unroll
-      for (int x = 0; x < EPL; ++x) qf[b][x] = p < Pe ? qf[b][x] * qscale : 0.f;
+        for (int x = 0; x < EPL; ++x) qf[b][x] *= qscale;
+      }
     }
     const int mmax = len - max(0, Pe - 1 - (p0 + QB - 1));  // keys of the pass's newest query
     // logits (log2 units); U row steps load before any is used
