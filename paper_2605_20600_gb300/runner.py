@@ -34,6 +34,8 @@ def generate(engine: Engine, provider, *, last_step: int | None = None, on_step=
         identify = "fused" if fused and engine.cfg.distance_mode == 0 else "separate"
     if identify not in ("fused", "separate", "multi") or (identify == "fused" and not fused):
         raise ValueError(f"identify={identify!r} with fused={fused}")
+    if identify == "fused" and engine.cfg.distance_mode != 0:
+        raise ValueError("the fused identification counts in raster order only")
     cfg = engine.cfg
     L, S, H, D, C = cfg.n_layers, cfg.n_seqs, cfg.n_heads, cfg.head_dim, cfg.n_cond
     E = cfg.group_at

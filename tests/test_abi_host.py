@@ -191,3 +191,28 @@ def test_fault_injection_raises_through_binding(H, monkeypatch):
 def test_fault_injection_other_name_does_not_fire(H, monkeypatch):
     monkeypatch.setenv("HKV_FAULT_INJECT", "repack:6")
     H.hkv_validate_config(tiny_cfg(H))
+
+
+@pytest.mark.parametrize("fused,identify,distance,ok", [
+    (True, "fused", 0, True), (True, "separate", 1, True), (True, "multi", 1, True),
+    (False, "fused", 0, False), (True, "fused", 1, False), (True, "bogus", 0, False),
+    # the default: fused where the distances are raster, separate otherwise
+    (True, None, 0, True), (True, None, 1, True), (False, None, 1, True)])
+def test_runner_identification_choices(H, fused, identify, distance, ok):
+    """The runner refuses combinations the library cannot run before it
+    touches the device (a stand-in engine with a configuration only)."""
+    from paper_2605_20600_gb300.runner import generate
+
+    class Stop(Exception):
+        pass
+
+    class FakeEngine:
+        cfg = tiny_cfg(H, distance_mode=distance)
+
+        @property
+        def device(self):
+            raise Stop()   # the first device access: the checks have passed
+
+    with pytest.raises(Stop if ok else ValueError):
+        generate(FakeEngine(), None, fused=fused, identify=identify)
+
