@@ -64,3 +64,31 @@ def test_reference_arm_prints_on_rank_zero_only():
                         "--steps", "1", "--warmup", "0"], env=env, capture_output=True,
                        text=True, timeout=120)
     assert r.returncode == 0 and r.stdout.strip() == ""
+
+
+def test_profiled_traffic_follows_the_committed_capture(monkeypatch, tmp_path):
+    """The roofline's traffic comes from the committed ncu summary while the
+    attention source still has the sha256 recorded there, scaled by the
+    launch's algorithmic bytes; any other source or workload gives None."""
+    import hashlib
+    sys.path.insert(0, ROOT)
+    import bench
+    prof = os.path.join(ROOT, "profiles", "decode_step_lumina1024_rho4.md")
+    src = os.path.join(ROOT, "paper_2605_20600_gb300", "csrc", "hkv_attention.cu")
+    vals = dict(line.strip().partition(": ")[::2] for line in open(prof) if ": " in line)
+    same = hashlib.sha256(open(src, "rb").read()).hexdigest() == vals.get("source_sha256")
+    t = bench.profiled_traffic("lumina1024", 1e8)
+    if same:
+        exp = float(vals["attn_traffic_ratio"]) * 1e8 + float(vals["finish_traffic_bytes_per_launch"])
+        assert t == pytest.approx(exp)
+    else:
+        assert t is None
+    assert bench.profiled_traffic("llamagen_xl", 1e8) is None
+    # a copy of the tree whose attention source differs: no traffic
+    (tmp_path / "profiles").mkdir()
+    (tmp_path / "profiles" / "decode_step_lumina1024_rho4.md").write_text(open(prof).read())
+    d = tmp_path / "paper_2605_20600_gb300" / "csrc"
+    d.mkdir(parents=True)
+    (d / "hkv_attention.cu").write_text(open(src).read() + "\n// changed\n")
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.profiled_traffic("lumina1024", 1e8) is None
