@@ -205,7 +205,8 @@ hkv_status hkv_prefill(const hkv_config *cfg, const hkv_cache *cache, int layer,
  *     first: a local head keeps its conditioning and newest w tokens
  *     (Eq. 3); a global head whose history exceeds its budget (cap - C - P
  *     - w: B_g - w under the paper's budgets) evicts the excess
- *     by STE (Eqs. 4-6: long/near split by r_s, scores from the P buffered
+ *     by STE (Eqs. 4-6: long/near split by r_s, in raster order or on the
+ *     grid per cfg->distance_mode; scores from the P buffered
  *     queries, the lowest floor(M/2) / M - floor(M/2) of each subset
  *     evicted, older first on equal score); the segment shrinks in place by
  *     moving the surviving rows above the new length into the evicted rows
@@ -295,8 +296,9 @@ hkv_status hkv_decode_attention_noalloc(const hkv_config *cfg, const hkv_cache *
 /* Sec. 4, Step 2 for one layer of an HKV_DENSE cache (heads of any other
  * label set HKV_ERR_STATE in the error word): for each head, the
  * attention of q over the live keys is accumulated backward from the newest
- * token until tau is reached; n_h is the number of tokens needed and the
- * head is HKV_LOCAL iff n_h < w_loc. Writes label_out[i] and, if non-null,
+ * token (or outward on the grid, HKV_DIST_GRID2D) until tau is reached; n_h
+ * is the number of tokens needed and the head is HKV_LOCAL iff n_h < w_loc.
+ * Writes label_out[i] and, if non-null,
  * nh_out[i] for the layer's heads (i = flat head index; both arrays are
  * [L*S*H]). */
 hkv_status hkv_identify_heads(const hkv_config *cfg, const hkv_cache *cache, int layer,
@@ -310,7 +312,8 @@ hkv_status hkv_identify_heads(const hkv_config *cfg, const hkv_cache *cache, int
  * decode steps; the newest is the current token's) each attend over the keys
  * that existed at their own step: the p-th oldest (p = 0 .. Pe-1) over the
  * oldest len - (Pe - 1 - p) keys. Their softmax rows are averaged, the
- * average is accumulated backward from the newest token until tau is
+ * average is accumulated backward from the newest token (or outward on the
+ * grid, HKV_DIST_GRID2D) until tau is
  * reached, n_h is the number of tokens needed, and the head is HKV_LOCAL iff
  * n_h < w_loc. With period = 1 this is hkv_identify_heads. Call it after the
  * grouping token's decode step, like hkv_identify_heads. Writes
