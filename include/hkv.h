@@ -322,6 +322,10 @@ hkv_status hkv_identify_heads(const hkv_config *cfg, const hkv_cache *cache, int
  *  - a head with another label than HKV_DENSE, or with ntok = 0 (no query
  *    buffered yet): HKV_ERR_STATE in the error word, head not decided;
  *  - len above n_cond + group_at: HKV_ERR_CAPACITY in the error word;
+ *  - n_cond + group_at tokens that do not fit one block's shared memory
+ *    (36 bytes a token for a period of 48 or more, else 20; 12 more with
+ *    HKV_DIST_GRID2D; 227 KB in all): HKV_ERR_CAPACITY returned, nothing
+ *    launched;
  *  - label_out NULL or layer out of range: HKV_ERR_INVALID_ARG. */
 hkv_status hkv_identify_heads_multi(const hkv_config *cfg, const hkv_cache *cache, int layer,
                                     uint8_t *label_out, int32_t *nh_out, hkv_stream_t stream);
