@@ -216,3 +216,13 @@ def test_runner_identification_choices(H, fused, identify, distance, ok):
     with pytest.raises(Stop if ok else ValueError):
         generate(FakeEngine(), None, fused=fused, identify=identify)
 
+
+
+def test_missing_library_fails_loudly(H, monkeypatch, tmp_path):
+    """No CPU fallback: without libheadkv.so every call raises."""
+    monkeypatch.setattr(H, "_lib", None)
+    monkeypatch.setattr(H, "LIB_PATH", str(tmp_path / "libheadkv.so"))
+    with pytest.raises(RuntimeError, match="missing"):
+        H.hkv_validate_config(tiny_cfg(H))
+    with pytest.raises(RuntimeError, match="missing"):
+        H.hkv_check(fake_cache(H))
