@@ -226,3 +226,22 @@ def test_missing_library_fails_loudly(H, monkeypatch, tmp_path):
         H.hkv_validate_config(tiny_cfg(H))
     with pytest.raises(RuntimeError, match="missing"):
         H.hkv_check(fake_cache(H))
+
+
+@pytest.mark.parametrize("period,group_at", [(16, 32), (1, 20), (5, 5), (7, 40)])
+def test_engine_update_schedule_matches_the_oracle(H, period, group_at):
+    """The steps at which the engine runs the periodic update (R7) are the
+    steps at which the oracle's generation does."""
+    from oracle import headkv as O
+    from synth import configs, gen
+    from paper_2605_20600_gb300.engine import Engine
+    w = configs.TINY.with_(period=period, group_at=group_at)
+    hi = gen.HeadInputs(w, 0, 0, 5)
+    tr = O.run_head(O.HeadParams.of(w), hi.q, hi.k, hi.v)
+    oracle_steps = [u.t_last + 1 for u in tr.updates[1:]]     # [0] is the grouping update
+
+    class Cfg:
+        pass
+    fake = Cfg()
+    fake.cfg = tiny_cfg(H, period=period, group_at=group_at, n_image=w.n_image)
+    assert [t for t in range(w.n_image) if Engine.update_due(fake, t)] == oracle_steps
