@@ -179,12 +179,29 @@ const char *hkv_status_str(hkv_status s);
  * only. */
 hkv_status hkv_validate_config(const hkv_config *cfg);
 
+/* Sec. 5.1: the image tokens a global head keeps, B_g = floor(rho * N),
+ * for rho = rho_num / rho_den (0 < rho <= 1, rho_den < 2^31) and N = n_image
+ * image tokens, in exact integer arithmetic. Writes *budget_out (host).
+ * Bad arguments -> HKV_ERR_INVALID_ARG. Host only. */
+hkv_status hkv_global_budget(int64_t rho_num, int64_t rho_den, int32_t n_image,
+                             int32_t *budget_out);
+
+/* Whether the decode step of image token t starts with the periodic update
+ * (Sec. 4, Efficient Cache Update): *due_out = 1 iff t > E and (t - E) is a
+ * multiple of P (E = group_at, P = period), else 0. The grouping step of
+ * token E - 1 runs the first update itself (hkv_repack); every P tokens
+ * after it the buffer is full, and the update runs after that step's
+ * attention, i.e. before the next step (hkv_evict, or inside
+ * hkv_append_evict). Host only. */
+hkv_status hkv_update_due(const hkv_config *cfg, int32_t t, int32_t *due_out);
+
 /* Bytes of device workspace hkv_decode_attention and hkv_decode_step need
  * for this config (split-K partial results, records of the heads split
- * between CTAs, and a small control block the two kernels of a call share).
- * The workspace must be zero-filled before its first use; every call leaves
- * it ready for the next one (after a call that reported an error, zero it
- * again). Concurrent calls must not share a workspace. Host only. */
+ * between CTAs, a small control block, ready flags of the partial results
+ * and two barrier words per layer). The workspace must be zero-filled before
+ * its first use; every call leaves it ready for the next one (after a call
+ * that reported an error, zero it again). Concurrent calls must not share a
+ * workspace. Host only. */
 size_t hkv_workspace_size(const hkv_config *cfg);
 
 /* Sets up the uncompressed cache of Step 1 (cache prefilling): every head
@@ -232,8 +249,12 @@ hkv_status hkv_evict(const hkv_config *cfg, const hkv_cache *cache, int layer, h
 
 /* One decode step of one layer: the append of the new token (Sec. 3, KV
  * Cache) fused with the attention of Eq. 1 over the cache including that
- * token, in two kernels chained on `stream` (attention over the cache, then
- * a finishing kernel that combines heads split across CTAs and appends). out[s][h][:] = softmax(q k^T / sqrt(d)) V over the
+ * token. One kernel launch when every CTA's share of the layer spans at
+ * most 128 heads (bounded from the config: the heads of a layer times the
+ * tiles of the longest segment it allows, over the grid), else two chained
+ * kernels (attention, then a finishing kernel that combines heads split
+ * across CTAs and advances the counters); hkv_decode_step_launches tells
+ * which. out[s][h][:] = softmax(q k^T / sqrt(d)) V over the
  * head's len live tokens and the new one (whose K/V are read straight from
  * k and v), fp32; then k, v join the arena at row len, q joins the Q_past
  * ring, and len, ntok (and nbuf for compressed heads) advance by one.
@@ -245,6 +266,11 @@ hkv_status hkv_evict(const hkv_config *cfg, const hkv_cache *cache, int layer, h
 hkv_status hkv_decode_step(const hkv_config *cfg, const hkv_cache *cache, int layer,
                            const void *q, const void *k, const void *v, float *out,
                            void *workspace, size_t ws_bytes, int flags, hkv_stream_t stream);
+
+/* Kernel launches one hkv_decode_step call of this config makes on the
+ * current device: 1 or 2 (see hkv_decode_step); 0 for an invalid config or
+ * a failed device query. Host only. */
+int hkv_decode_step_launches(const hkv_config *cfg);
 
 /* hkv_decode_step fused with the head-type identification of Sec. 4,
  * Step 2, for the grouping step (image token E - 1) on the uncompressed

@@ -23,7 +23,7 @@ ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
          "-I", os.path.join(ROOT, "include"), "-I", CSRC]
 
-SOURCES = ["hkv_api.cu", "hkv_attention.cu", "hkv_update.cu", "hkv_noalloc.cu"]
+SOURCES = ["hkv_api.cu", "hkv_attention.cu", "hkv_step.cu", "hkv_update.cu", "hkv_noalloc.cu"]
 
 
 def nvcc() -> str:

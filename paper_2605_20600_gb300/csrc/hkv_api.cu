@@ -8,6 +8,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <atomic>
 #include <mutex>
 #include <vector>
 
@@ -21,11 +22,15 @@ using namespace hkv;
 constexpr int kMaxDevices = 64;
 constexpr size_t kMaxSmem = 227 * 1024;
 
+// Per-device launch setup, filled on first use. Every field is written at
+// most once (under g_mu) and read lock-free: atomics with acquire/release
+// ordering, so a thread that sees a value also sees what was set up before
+// it was published.
 struct DeviceState {
-  bool init = false;
-  int sms = 0;
-  int attn_ctas[2][2] = {{0, 0}, {0, 0}};   // [dtype][D == 128]
-  size_t update_smem[2][2] = {{0, 0}, {0, 0}};
+  std::atomic<int> sms{0};
+  std::atomic<int> attn_ctas[2][2] = {};  // [dtype][D == 128]
+  std::atomic<int> step_ctas[2][2] = {};
+  std::atomic<size_t> update_smem[2][2] = {};
 };
 
 DeviceState g_dev[kMaxDevices];
@@ -52,40 +57,45 @@ hkv_status device_state(DeviceState **out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return HKV_ERR_CUDA;
   DeviceState &st = g_dev[dev];
-  if (!st.init) {
+  if (st.sms.load(std::memory_order_acquire) == 0) {
     std::lock_guard<std::mutex> lk(g_mu);
-    if (!st.init) {
-      if (cudaDeviceGetAttribute(&st.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    if (st.sms.load(std::memory_order_relaxed) == 0) {
+      int n = 0;
+      if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
         return HKV_ERR_CUDA;
-      st.init = true;
+      st.sms.store(n, std::memory_order_release);
     }
   }
   *out = &st;
   return HKV_OK;
 }
 
+// CTAs per SM of the decode kernels (both designs share the grid)
 hkv_status attention_ctas(DeviceState *st, int D, int dtype, int *ctas) {
-  int &c = st->attn_ctas[dt_index(dtype)][d_index(D)];
-  if (c == 0) {
+  std::atomic<int> &c = st->attn_ctas[dt_index(dtype)][d_index(D)];
+  int v = c.load(std::memory_order_acquire);
+  if (v == 0) {
     std::lock_guard<std::mutex> lk(g_mu);
-    if (c == 0) {
+    v = c.load(std::memory_order_relaxed);
+    if (v == 0) {
       int n = 0;
       if (attention_prepare(D, dtype, &n) != cudaSuccess || n <= 0) return HKV_ERR_CUDA;
-      c = n;
+      v = n;
+      c.store(v, std::memory_order_release);
     }
   }
-  *ctas = c;
+  *ctas = v;
   return HKV_OK;
 }
 
 hkv_status update_ready(DeviceState *st, int D, int dtype, size_t smem) {
-  size_t &have = st->update_smem[dt_index(dtype)][d_index(D)];
+  std::atomic<size_t> &have = st->update_smem[dt_index(dtype)][d_index(D)];
   if (smem > kMaxSmem) return HKV_ERR_CAPACITY;
-  if (have < smem) {
+  if (have.load(std::memory_order_acquire) < smem) {
     std::lock_guard<std::mutex> lk(g_mu);
-    if (have < smem) {
+    if (have.load(std::memory_order_relaxed) < smem) {
       if (update_prepare(D, dtype, smem) != cudaSuccess) return HKV_ERR_CUDA;
-      have = smem;
+      have.store(smem, std::memory_order_release);
     }
   }
   return HKV_OK;
@@ -151,20 +161,30 @@ int max_segment(const hkv_config *c) {
 
 size_t align256(size_t b) { return (b + 255) & ~(size_t)255; }
 
-// split-K partials: kAttnInlinePieces slots per CTA boundary, one overflow
-// slot per CTA
-size_t part_bytes(const hkv_config *c) {
-  return align256((size_t)kAttnMaxGrid * kAttnInlinePieces * attn_part_floats(c->head_dim) *
-                  sizeof(float));
-}
-size_t over_bytes(const hkv_config *c) {
-  return align256((size_t)kAttnMaxGrid * attn_part_floats(c->head_dim) * sizeof(float));
-}
-
-// where the head split at each CTA boundary is
-size_t rec_bytes() { return align256((size_t)kAttnMaxGrid * sizeof(int4)); }
-
 constexpr size_t kCtlBytes = 256;  // AttnCtl, padded
+
+// Workspace of the decode kernels, in this order: split-K partials
+// (kAttnInlinePieces slots per CTA boundary, one overflow slot per CTA), the
+// record of the head split at each CTA boundary, the control block the
+// two-kernel design's attention kernel leaves for its finishing kernel, the
+// epoch-tagged partial results of the one-launch step (two slots of D + 2
+// 8-byte pairs per CTA) and its per-layer barrier words.
+struct WsLayout {
+  size_t part, over, rec, ctl, pslot, bar, total;
+};
+
+WsLayout ws_layout(const hkv_config *c) {
+  WsLayout w;
+  const size_t pf = attn_part_floats(c->head_dim) * sizeof(float);
+  w.part = 0;
+  w.over = w.part + align256((size_t)kAttnMaxGrid * kAttnInlinePieces * pf);
+  w.rec = w.over + align256((size_t)kAttnMaxGrid * pf);
+  w.ctl = w.rec + align256((size_t)kAttnMaxGrid * sizeof(int4));
+  w.pslot = w.ctl + kCtlBytes;
+  w.bar = w.pslot + align256((size_t)kAttnMaxGrid * 2 * (c->head_dim + 2) * 8);
+  w.total = w.bar + align256((size_t)c->n_layers * 2 * sizeof(uint32_t));
+  return w;
+}
 
 // Fills the attention launch arguments for one layer; the workspace holds
 // the split-K partials (per CTA boundary, and overflow slots per CTA), which
@@ -182,10 +202,14 @@ AttnArgs attn_args(const hkv_config *cfg, const hkv_cache *cache, int layer, con
   a.q = q;
   a.out = out;
   unsigned char *ws = static_cast<unsigned char *>(workspace);
-  a.part = reinterpret_cast<float *>(ws);
-  a.over = reinterpret_cast<float *>(ws + part_bytes(cfg));
-  a.rec = reinterpret_cast<int4 *>(ws + part_bytes(cfg) + over_bytes(cfg));
-  a.ctl = reinterpret_cast<AttnCtl *>(ws + part_bytes(cfg) + over_bytes(cfg) + rec_bytes());
+  const WsLayout w = ws_layout(cfg);
+  a.part = reinterpret_cast<float *>(ws + w.part);
+  a.over = reinterpret_cast<float *>(ws + w.over);
+  a.rec = reinterpret_cast<int4 *>(ws + w.rec);
+  a.ctl = reinterpret_cast<AttnCtl *>(ws + w.ctl);
+  a.pslot = reinterpret_cast<unsigned long long *>(ws + w.pslot);
+  a.bar = reinterpret_cast<uint32_t *>(ws + w.bar) + (size_t)layer * 2;
+  a.n_layers = cfg->n_layers;
   a.err = cache->err;
   a.pos = cache->pos;
   a.nbuf = cache->nbuf;
@@ -201,6 +225,37 @@ AttnArgs attn_args(const hkv_config *cfg, const hkv_cache *cache, int layer, con
   return a;
 }
 
+// CTAs per SM of the one-launch step: kStepActivePerSm, if the kernel can
+// have that many resident (its own setup, once per device and shape)
+hkv_status step_ctas(DeviceState *st, int D, int dtype, int *ctas) {
+  std::atomic<int> &c = st->step_ctas[dt_index(dtype)][d_index(D)];
+  int v = c.load(std::memory_order_acquire);
+  if (v == 0) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    v = c.load(std::memory_order_relaxed);
+    if (v == 0) {
+      int m = 0;
+      if (step_prepare(D, dtype, &m) != cudaSuccess || m <= 0) return HKV_ERR_CUDA;
+      v = m < kStepActivePerSm ? m : kStepActivePerSm;
+      c.store(v, std::memory_order_release);
+    }
+  }
+  *ctas = v;
+  return HKV_OK;
+}
+
+hkv_status step_grid(const hkv_config *cfg, int *grid) {
+  DeviceState *st;
+  hkv_status s = device_state(&st);
+  if (s != HKV_OK) return s;
+  int ctas = 0;
+  s = step_ctas(st, cfg->head_dim, cfg->dtype, &ctas);
+  if (s != HKV_OK) return s;
+  const int g = st->sms.load(std::memory_order_acquire) * ctas;
+  *grid = g > kAttnMaxGrid ? kAttnMaxGrid : g;
+  return HKV_OK;
+}
+
 // attention CTAs: every SM filled
 hkv_status attn_grid(const hkv_config *cfg, int *grid) {
   DeviceState *st;
@@ -209,9 +264,24 @@ hkv_status attn_grid(const hkv_config *cfg, int *grid) {
   int ctas = 0;
   s = attention_ctas(st, cfg->head_dim, cfg->dtype, &ctas);
   if (s != HKV_OK) return s;
-  const int g = st->sms * ctas;
+  const int g = st->sms.load(std::memory_order_acquire) * ctas;
   *grid = g > kAttnMaxGrid ? kAttnMaxGrid : g;
   return HKV_OK;
+}
+
+// Whether hkv_decode_step runs as one launch (hkv_step.cu): every CTA's range
+// must fit the kernel's head table. A range of c tiles holds at most c + 1
+// heads (a head has at least one tile in a step, its new token), and c is at
+// most the layer's tile count over the grid, bounded by every head at the
+// longest segment the config allows. HKV_STEP_TWO_KERNELS in the
+// environment selects the two-kernel design regardless (tests of both).
+bool one_launch_step(const hkv_config *cfg, int grid) {
+  if (getenv("HKV_STEP_TWO_KERNELS")) return false;
+  const long long tt = step_tile_rows(cfg->head_dim, cfg->dtype);
+  const long long tiles = (long long)heads_per_layer(cfg) * ((max_segment(cfg) + tt - 1) / tt);
+  long long chunk = (tiles + grid - 1) / grid;
+  if (chunk < 2) chunk = 2;
+  return chunk + 1 <= kStepTable;
 }
 
 #define HKV_TRY(x)                 \
@@ -270,9 +340,33 @@ hkv_status hkv_validate_config(const hkv_config *c) {
   return HKV_OK;
 }
 
+hkv_status hkv_global_budget(int64_t rho_num, int64_t rho_den, int32_t n_image,
+                             int32_t *budget_out) {
+  HKV_TRY(injected("global_budget"));
+  if (!budget_out) return HKV_ERR_INVALID_ARG;
+  if (rho_num <= 0 || rho_den <= 0 || rho_num > rho_den || rho_den > 0x7fffffffLL ||
+      n_image <= 0)
+    return HKV_ERR_INVALID_ARG;
+  // Sec. 5.1: rho * N image tokens, rounded down; exact (num * N < 2^62)
+  *budget_out = (int32_t)(rho_num * (int64_t)n_image / rho_den);
+  return HKV_OK;
+}
+
+hkv_status hkv_update_due(const hkv_config *cfg, int32_t t, int32_t *due_out) {
+  HKV_TRY(injected("update_due"));
+  HKV_TRY(hkv_validate_config(cfg));
+  if (!due_out || t < 0) return HKV_ERR_INVALID_ARG;
+  // Sec. 4, Efficient Cache Update: the grouping step (image token E - 1)
+  // runs the first update; after it the buffer fills every P tokens, and the
+  // update that empties it runs before the step of the token after the P-th
+  const int E = cfg->group_at, P = cfg->period;
+  *due_out = t > E && (t - E) % P == 0 ? 1 : 0;
+  return HKV_OK;
+}
+
 size_t hkv_workspace_size(const hkv_config *c) {
   if (!c || hkv_validate_config(c) != HKV_OK) return 0;
-  return part_bytes(c) + over_bytes(c) + rec_bytes() + kCtlBytes;
+  return ws_layout(c).total;
 }
 
 hkv_status hkv_init_dense(const hkv_config *cfg, const hkv_cache *cache, hkv_stream_t stream) {
@@ -357,6 +451,12 @@ hkv_status decode_step(const char *name, const hkv_config *cfg, const hkv_cache 
   a.label_out = label_out;
   a.w_loc = cfg->local_w;
   a.tau = (float)cfg->tau;
+  if (!label_out) {
+    int sgrid = 0;
+    HKV_TRY(step_grid(cfg, &sgrid));
+    if (one_launch_step(cfg, sgrid))
+      return cuda_status(launch_step(a, cfg->head_dim, cfg->dtype, sgrid, (cudaStream_t)stream));
+  }
   return cuda_status(launch_attention(a, cfg->head_dim, cfg->dtype, grid, true,
                                       label_out != nullptr, (cudaStream_t)stream));
 }
@@ -368,6 +468,13 @@ hkv_status hkv_decode_step(const hkv_config *cfg, const hkv_cache *cache, int la
                            void *workspace, size_t ws_bytes, int flags, hkv_stream_t stream) {
   return decode_step("decode_step", cfg, cache, layer, q, k, v, out, nullptr, workspace, ws_bytes,
                      flags, stream);
+}
+
+int hkv_decode_step_launches(const hkv_config *cfg) {
+  if (hkv_validate_config(cfg) != HKV_OK) return 0;
+  int grid = 0;
+  if (step_grid(cfg, &grid) != HKV_OK) return 0;
+  return one_launch_step(cfg, grid) ? 1 : 2;
 }
 
 hkv_status hkv_decode_step_identify(const hkv_config *cfg, const hkv_cache *cache, int layer,

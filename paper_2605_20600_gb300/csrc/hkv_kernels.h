@@ -57,6 +57,13 @@ struct AttnArgs {
   uint8_t *label_out;         // [L*S*H]
   int w_loc;
   float tau;
+  // one-launch step (hkv_step.cu): the layer's barrier word pair {arrivals,
+  // generation}, zero between launches; the partial results of split heads
+  // as (value, launch epoch) pairs, two slots per CTA (the piece at the end
+  // of its range, the piece at its start), [grid][2][D + 2]
+  uint32_t *bar;
+  unsigned long long *pslot;
+  int n_layers;
 };
 
 // decode attention CTAs: one producer warp (TMA), consumer warps, one
@@ -77,7 +84,26 @@ __host__ __device__ constexpr int attn_part_floats(int D) { return D + 4; }
 // pieces of a split head kept per CTA boundary (loaded with its record)
 constexpr int kAttnInlinePieces = 4;
 
+// one-launch decode step: heads of a CTA's range it keeps in shared memory
+#ifndef HKV_STEP_TABLE
+#define HKV_STEP_TABLE 128
+#endif
+constexpr int kStepTable = HKV_STEP_TABLE;
+
 size_t attention_smem_bytes(int D, int dtype);
+// rows of K (and of V) per pipeline stage of the one-launch step
+int step_tile_rows(int D, int dtype);
+// CTAs per SM of the one-launch step's grid, and the shared memory and
+// occupancy setup of its kernel (resident CTAs per SM)
+#ifndef HKV_STEP_ACTIVE_PER_SM
+#define HKV_STEP_ACTIVE_PER_SM 2
+#endif
+constexpr int kStepActivePerSm = HKV_STEP_ACTIVE_PER_SM;
+cudaError_t step_prepare(int D, int dtype, int *ctas_per_sm);
+// the fused decode step of one layer in one launch (append + attention,
+// merges of split heads and counters in the same kernel); `grid` CTAs, at
+// most kAttnMaxGrid, a CTA's range spanning at most kStepTable heads
+cudaError_t launch_step(const AttnArgs &a, int D, int dtype, int grid, cudaStream_t s);
 cudaError_t attention_prepare(int D, int dtype, int *ctas_per_sm);
 // launches the attention kernel on `grid` CTAs (at most kAttnMaxGrid) and the
 // finishing kernel behind it; identify (fused only): also the Step 2 label of

@@ -1,0 +1,931 @@
+// One decode step of one layer in a single launch: attention of every head's
+// new query over the head's retained tokens and the step's new token (Eq. 1),
+// fused with the append of that token to the cache (Sec. 3, KV Cache).
+//
+// The split-K layout is the one of the two-kernel design in hkv_attention.cu
+// (the layer's heads rounded up to whole tiles and concatenated; gridDim.x
+// equal contiguous ranges, one per CTA; a warp-specialised TMA pipeline with
+// a producer warp, consumer warps and an epilogue warp), but the work that
+// the finishing kernel did there happens inside this launch:
+//
+//  * tile order: a CTA streams the piece of the head that began in an
+//    earlier range first, then the start of the head that continues into a
+//    later range, then the heads wholly inside its range. Every piece of a
+//    split head is then done early in its CTA, except the piece of a CTA
+//    whose whole range lies inside the head (a "middle" CTA);
+//  * merges: a split head is combined by its first middle CTA (whose whole
+//    range lies inside the head), else by the CTA holding its last row. The
+//    other pieces write their partial result to the workspace as 64-bit
+//    (value, launch epoch) pairs, which are single-copy atomic, so no fence
+//    or flag is needed: the combining CTA's merge warp reads the pieces until
+//    every pair carries this launch's epoch, while its consumers stream.
+//    Pieces are combined in index order and the CTA's own piece last, so the
+//    result does not depend on timing;
+//  * appends and counters: the merge warp copies the new token of every head
+//    whose last row is in the CTA's range into the cache as soon as the
+//    step's inputs are visible (nothing in the launch reads those rows).
+//    Every CTA reads the layer's lengths in its prologue and arrives on a
+//    per-layer barrier word when it is done reading them; the merge warp
+//    advances len, ntok and nbuf of its heads once the whole grid has
+//    arrived. The next launch of the same layer starts after this one
+//    completes, so the barrier word is free again by then;
+//  * programmatic dependent launch: with the prefetch flag the prologue and
+//    the first tiles of old K/V rows go ahead of the wait for the previous
+//    kernel; the step's inputs (q, the new k and v) are read after it;
+//  * every wait is bounded (HKV_ERR_TIMEOUT in the error word).
+//
+// The lengths of every head whose range a CTA touches are kept in a table in
+// shared memory (kStepTable heads); the host takes this path only when no
+// range can hold more heads than that.
+#include <math.h>
+#include <stdlib.h>
+
+#include "hkv_attn_common.cuh"
+#include "hkv_device.cuh"
+#include "hkv_kernels.h"
+
+namespace hkv {
+namespace {
+
+#ifdef HKV_ATTN_TRACE
+__device__ unsigned long long *g_step_trace = nullptr;  // [layer][kAttnMaxGrid][32]
+#define STEP_TRACE_AT(slot) \
+  g_step_trace[((size_t)(p.layer_base / p.nheads) * kAttnMaxGrid + blockIdx.x) * 32 + (slot)]
+#define STEP_TRACE(slot)                                    \
+  do {                                                      \
+    if (g_step_trace) STEP_TRACE_AT(slot) = globaltimer(); \
+  } while (0)
+#define STEP_TRACE_SET(slot, v)                 \
+  do {                                          \
+    if (g_step_trace) STEP_TRACE_AT(slot) = (v); \
+  } while (0)
+#else
+#define STEP_TRACE(slot) \
+  do {                   \
+  } while (0)
+#define STEP_TRACE_SET(slot, v) \
+  do {                          \
+    (void)(v);                  \
+  } while (0)
+#endif
+
+// Tuning knobs (compile time) of the one-launch step, per head dimension:
+// consumer warps, bytes of K per stage, stages, tiles loaded before the wait;
+// CTAs per SM in the grid (kStepActivePerSm) and CTAs per SM the kernel is
+// built to be resident with (kStepResidentPerSm: with one more than the
+// grid uses, the next layer's CTAs can start while this layer streams).
+#ifndef HKV_STEP_CW_D128
+#define HKV_STEP_CW_D128 HKV_ATTN_CW_D128
+#endif
+#ifndef HKV_STEP_TILE_BYTES_D128
+#define HKV_STEP_TILE_BYTES_D128 HKV_ATTN_TILE_BYTES_D128
+#endif
+#ifndef HKV_STEP_STAGES_D128
+#define HKV_STEP_STAGES_D128 3
+#endif
+#ifndef HKV_STEP_PRE_D128
+#define HKV_STEP_PRE_D128 2
+#endif
+#ifndef HKV_STEP_CW_D64
+#define HKV_STEP_CW_D64 HKV_ATTN_CW_D64
+#endif
+#ifndef HKV_STEP_TILE_BYTES_D64
+#define HKV_STEP_TILE_BYTES_D64 HKV_ATTN_TILE_BYTES_D64
+#endif
+#ifndef HKV_STEP_STAGES_D64
+#define HKV_STEP_STAGES_D64 HKV_ATTN_STAGES_D64
+#endif
+#ifndef HKV_STEP_PRE_D64
+#define HKV_STEP_PRE_D64 HKV_ATTN_PRE_TILES
+#endif
+#ifndef HKV_STEP_RESIDENT_PER_SM
+#define HKV_STEP_RESIDENT_PER_SM 2
+#endif
+// heads of a thread's prologue slice kept in registers (more: reloaded)
+#ifndef HKV_STEP_SLICE_REGS
+#define HKV_STEP_SLICE_REGS 8
+#endif
+
+template <int D, typename T>
+using StepShape =
+    TileShape<D, T, D == 64 ? HKV_STEP_CW_D64 : HKV_STEP_CW_D128,
+              D == 64 ? HKV_STEP_TILE_BYTES_D64 : HKV_STEP_TILE_BYTES_D128,
+              D == 64 ? HKV_STEP_STAGES_D64 : HKV_STEP_STAGES_D128,
+              D == 64 ? HKV_STEP_PRE_D64 : HKV_STEP_PRE_D128>;
+
+struct StepTable {
+  int h0, n;                      // heads h0 .. h0 + n - 1
+  long long start[kStepTable];    // first index (slot space) of head h0 + j
+  long long off[kStepTable];      // arena offset
+  int vlen[kStepTable];           // len + 1 (the new token)
+  int nbuf[kStepTable];
+  int ntok[kStepTable];           // written by the append (epilogue warp)
+  unsigned char label[kStepTable];
+};
+
+constexpr int kFirst = 1, kLast = 2, kDone = 4;
+
+struct TileMeta {  // producer -> consumers, one per stage
+  int h, n, flags;
+  long long hs, he;  // the head's rows in the index space
+};
+
+struct SegMeta {  // consumers -> epilogue; h < 0: no more segments
+  int h;
+  long long hs, he;
+};
+
+// Tiles of a slot-aligned sub-range [g, b) of the index space, head by head,
+// over the table (j: table index of the current head).
+template <int TT>
+struct StepIter {
+  int j, hl;
+  long long hs, g, b;
+  __device__ __forceinline__ bool done() const { return g >= b; }
+  __device__ __forceinline__ long long tile_end() const {
+    long long e = g + TT;
+    if (e > hs + hl) e = hs + hl;
+    if (e > b) e = b;
+    return e;
+  }
+  __device__ __forceinline__ void advance(const StepTable &t) {
+    g += TT;
+    if (g >= b) return;
+    while (g >= hs + slot_len<TT>(hl) && j + 1 < t.n) {
+      ++j;
+      hs = t.start[j];
+      hl = t.vlen[j];
+    }
+  }
+};
+
+__device__ __forceinline__ uint32_t ld_acquire(const uint32_t *p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release(uint32_t *p, uint32_t v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// A float and the epoch of the launch that wrote it, as one 64-bit word:
+// single-copy atomic, so a reader that sees the epoch sees the value.
+__device__ __forceinline__ void st_pair(unsigned long long *p, float v, uint32_t ep) {
+  const unsigned long long w = ((unsigned long long)ep << 32) | __float_as_uint(v);
+  asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(p), "l"(w) : "memory");
+}
+__device__ __forceinline__ bool ld_pair(const unsigned long long *p, uint32_t ep, float &v) {
+  unsigned long long w;
+  asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(w) : "l"(p) : "memory");
+  v = __uint_as_float((uint32_t)w);
+  return (uint32_t)(w >> 32) == ep;
+}
+
+// threads: a producer warp, the consumer warps, the epilogue warp and the
+// merge warp
+template <int D, typename T>
+__host__ __device__ constexpr int step_threads() {
+  return StepShape<D, T>::kThreads + 32;
+}
+
+template <int D, typename T>
+__global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM)
+    step_kernel(const AttnArgs p) {
+  using S = StepShape<D, T>;
+  constexpr int kCW = S::kCW, kThr = step_threads<D, T>();
+  constexpr int LPR = S::kLPR, EPL = S::kEPL, RPW = S::kRPW, TT = S::kTT;
+  constexpr int RB = S::kRB, NS = S::kNS;
+  constexpr int NST = kCW * RPW;  // row-group states per segment
+  constexpr int CPL = D / 32;     // output channels per epilogue lane
+  static_assert(NST <= 32, "a lane of the epilogue per state");
+  using V = Vec<CPL>;
+
+  extern __shared__ __align__(128) unsigned char stages[];
+  __shared__ uint64_t full[NS], empty[NS];
+  __shared__ uint64_t epi_full[2], epi_free[2];  // two hand-over buffers
+  __shared__ __align__(16) float red_acc[2][NST][D];
+  __shared__ float red_m[2][NST], red_l[2][NST];
+  __shared__ TileMeta meta[NS];
+  __shared__ SegMeta seg[2];
+  __shared__ StepTable tab;
+  __shared__ long long scan_scratch[33];
+  __shared__ long long s_s0, s_mg_k0;
+  __shared__ int s_h0, s_h1, s_bad;
+  __shared__ int s_mg_h, s_mg_j, s_mg_np;  // the split head this CTA combines
+  __shared__ uint32_t s_ep;                // the launch's epoch
+  __shared__ uint64_t ep_bar, own_bar;     // merge warp -> epilogue, and back
+  __shared__ __align__(16) float own_acc[D];
+  __shared__ float own_ml[2];
+  __shared__ volatile int s_abort;
+
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int nheads = p.nheads;
+  const int G = gridDim.x;
+  const int bx = blockIdx.x;
+
+  if (tid == 0) {
+    STEP_TRACE(0);
+#ifdef HKV_ATTN_TRACE
+    if (g_step_trace) {
+      unsigned smid;
+      asm volatile("mov.u32 %0, %%smid;" : "=r"(smid));
+      STEP_TRACE_AT(16) = smid;
+    }
+#endif
+    for (int s = 0; s < NS; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], kCW);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&epi_full[s], kCW);
+      mbar_init(&epi_free[s], 1);
+    }
+    mbar_init(&ep_bar, 32);
+    mbar_init(&own_bar, 1);
+    fence_barrier_init();
+    s_abort = 0;
+    s_bad = 0;
+    s_h0 = 0;
+    s_h1 = -1;
+    s_s0 = 0;
+    s_mg_h = -1;
+  }
+  if (!p.prefetch) pdl_wait();
+
+  // ---- prologue: the layer's lengths, one round of loads -------------------
+  // Every thread takes a contiguous slice of the layer's heads and checks
+  // them (all loads of a head issued before any check); a block scan gives
+  // each slice its first index. Every CTA checks every head, so all CTAs take
+  // the same decision.
+  const int per = (nheads + kThr - 1) / kThr;
+  const int h_lo = tid * per < nheads ? tid * per : nheads;
+  const int h_hi = h_lo + per < nheads ? h_lo + per : nheads;
+  long long mine = 0;
+  int bad = 0;
+  auto check = [&](int l, long long o, int cp, int lab, int nb) {
+    if (l < 0 || o < 0 || o + cp > p.arena_tokens) bad = HKV_ERR_BOUNDS;
+    else if (l + 1 > cp) bad = bad ? bad : HKV_ERR_CAPACITY;
+    else if (lab != HKV_DENSE && nb >= p.period)
+      bad = bad ? bad : HKV_ERR_STATE;  // the periodic update is due first
+    mine += slot_len<TT>(l + 1);
+  };
+  // A slice of up to KR heads stays in registers for the whole prologue (one
+  // round of loads); a longer one is read again where needed.
+  constexpr int KR = HKV_STEP_SLICE_REGS;
+  const bool in_regs = per <= KR;
+  int rl[KR], rnb[KR];
+  long long ro[KR];
+  unsigned char rlb[KR];
+  if (in_regs) {
+    int rcp[KR];
+#pragma unroll
+    for (int u = 0; u < KR; ++u) {  // every load issued before any use
+      const int h = h_lo + u;
+      rl[u] = rnb[u] = rcp[u] = 0;
+      ro[u] = 0;
+      rlb[u] = 0;
+      if (h < h_hi) {
+        rl[u] = p.len[h];
+        ro[u] = p.off[h];
+        rcp[u] = p.cap[h];
+        rlb[u] = p.label[p.layer_base + h];
+        rnb[u] = p.nbuf[p.layer_base + h];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < KR; ++u)
+      if (h_lo + u < h_hi) check(rl[u], ro[u], rcp[u], rlb[u], rnb[u]);
+  } else {
+#pragma unroll 4
+    for (int h = h_lo; h < h_hi; ++h)
+      check(p.len[h], p.off[h], p.cap[h], p.label[p.layer_base + h], p.nbuf[p.layer_base + h]);
+  }
+  long long total;
+  const long long slice_start = block_excl_scan<long long>(mine, scan_scratch, &total);
+  if (tid == 0) STEP_TRACE(10);
+  if (bad) atomicMax(&s_bad, bad);
+  __syncthreads();
+  if (s_bad) {  // no CTA reads further or arrives: the step is not taken
+    pdl_wait();
+    if (bx == 0 && tid == 0) set_err(p.err, (uint32_t)s_bad);
+    return;
+  }
+  long long chunk = slot_len<TT>((total + G - 1) / G);
+  if (chunk < S::kMinChunk) chunk = S::kMinChunk;
+  const long long a = (long long)bx * chunk;
+  const long long b = a + chunk < total ? a + chunk : total;
+  bool active = a < total;
+  if (active && mine > 0) {  // the heads holding the range's first and last index
+    const bool has_a = slice_start <= a && a < slice_start + mine;
+    const bool has_b = slice_start <= b - 1 && b - 1 < slice_start + mine;
+    if (has_a || has_b) {
+      long long st = slice_start;
+      auto visit = [&](int h, int l) {
+        const long long L = slot_len<TT>(l + 1);
+        if (has_a && a >= st && a < st + L) {
+          s_h0 = h;
+          s_s0 = st;
+        }
+        if (has_b && b - 1 >= st && b - 1 < st + L) s_h1 = h;
+        st += L;
+      };
+      if (in_regs) {
+#pragma unroll
+        for (int u = 0; u < KR; ++u)
+          if (h_lo + u < h_hi) visit(h_lo + u, rl[u]);
+      } else {
+        for (int h = h_lo; h < h_hi; ++h) visit(h, p.len[h]);
+      }
+    }
+  }
+  __syncthreads();
+  if (tid == 0) STEP_TRACE(11);
+  int n = active ? s_h1 - s_h0 + 1 : 0;
+  if (n > kStepTable) {  // excluded by the host; reported, range skipped
+    if (tid == 0) set_err(p.err, HKV_ERR_CAPACITY);
+    n = 0;
+    active = false;
+  }
+  const int h0 = s_h0;
+  // the table: every thread fills the entries of its slice
+  if (active && h_lo <= h0 + n - 1 && h_hi > h0) {
+    long long st = slice_start;
+    auto fill = [&](int h, int l, long long o, int nb, int lab) {
+      if (h >= h0 && h < h0 + n) {
+        const int j = h - h0;
+        tab.start[j] = st;
+        tab.off[j] = o;
+        tab.vlen[j] = l + 1;
+        tab.nbuf[j] = nb;
+        tab.label[j] = (unsigned char)lab;
+      }
+      st += slot_len<TT>(l + 1);
+    };
+    if (in_regs) {
+#pragma unroll
+      for (int u = 0; u < KR; ++u)
+        if (h_lo + u < h_hi) fill(h_lo + u, rl[u], ro[u], rnb[u], rlb[u]);
+    } else {
+      for (int h = h_lo; h < h_hi; ++h)
+        fill(h, p.len[h], p.off[h], p.nbuf[p.layer_base + h], p.label[p.layer_base + h]);
+    }
+  }
+  if (tid == 0) {
+    tab.h0 = h0;
+    tab.n = n;
+  }
+  __syncthreads();
+  // From here on nothing reads the layer's counters in global memory: the
+  // epilogue warp arrives on the layer's barrier word below.
+  if (tid == 0) STEP_TRACE(1);
+
+  // ---- the range's sub-ranges, in streaming order --------------------------
+  // S: the piece of the head that began before a; E: the start of the head
+  // that continues past b; M: the heads in between.
+  long long sub_g[3], sub_b[3];
+  int sub_j[3], nsub = 0;
+  if (active) {
+    const long long hs0 = tab.start[0];
+    const long long se0 = hs0 + slot_len<TT>(tab.vlen[0]);
+    const long long hs1 = tab.start[n - 1];
+    const long long he1 = hs1 + tab.vlen[n - 1];
+    const bool has_s = hs0 < a;
+    const bool has_e = he1 > b && (n > 1 || !has_s);
+    const long long s_end = se0 < b ? se0 : b;
+    const long long e_beg = hs1 > a ? hs1 : a;
+    if (has_s) {
+      sub_g[nsub] = a, sub_b[nsub] = s_end, sub_j[nsub] = 0;
+      ++nsub;
+    }
+    if (has_e) {
+      sub_g[nsub] = e_beg, sub_b[nsub] = b, sub_j[nsub] = n - 1;
+      ++nsub;
+    }
+    const long long m_lo = has_s ? s_end : a, m_hi = has_e ? e_beg : b;
+    if (m_lo < m_hi) {
+      sub_g[nsub] = m_lo, sub_b[nsub] = m_hi, sub_j[nsub] = has_s ? 1 : 0;
+      ++nsub;
+    }
+  }
+
+  // ---- producer state (warp 0, lane 0) ------------------------------------
+  const bool producer = tid == 0;
+  StepIter<TT> pit;
+  int sr = 0;  // current sub-range
+  auto start_sub = [&](int r) {
+    pit.j = sub_j[r];
+    pit.hs = tab.start[pit.j];
+    pit.hl = tab.vlen[pit.j];
+    pit.g = sub_g[r];
+    pit.b = sub_b[r];
+  };
+  pit.g = pit.b = 0;
+  pit.j = 0;
+  pit.hs = 0;
+  pit.hl = 0;
+  if (nsub > 0) start_sub(0);
+  auto more = [&]() {  // moves to the next sub-range when one is exhausted
+    while (pit.done() && sr + 1 < nsub) start_sub(++sr);
+    return !pit.done();
+  };
+  int issued = 0;
+  const uint64_t stream_pol = producer ? l2_evict_first_policy() : 0;
+  struct Pending {
+    int h, slot_new;
+    bool first, has_new;
+  };
+  auto issue_old = [&](Pending &pd) {  // describe, expect and copy the arena rows
+    const int stage = issued % NS;
+    const long long ge = pit.tile_end();
+    const long long he = pit.hs + pit.hl;
+    const int r0 = (int)(pit.g - pit.hs), r1 = (int)(ge - pit.hs);
+    const int real = pit.hl - 1;  // rows in the arena
+    const int n_old = (r1 < real ? r1 : real) - r0;
+    unsigned char *dk = stages + stage * S::kStageBytes;
+    const int h = h0 + pit.j;
+    pd.h = h;
+    pd.slot_new = real - r0;
+    pd.first = pit.g == pit.hs || pit.g == sub_g[sr];
+    pd.has_new = r1 == pit.hl;
+    TileMeta &mt = meta[stage];
+    mt.h = h;
+    mt.n = (int)(ge - pit.g);
+    mt.flags = (pd.first ? kFirst : 0) | (ge == (pit.b < he ? pit.b : he) ? kLast : 0);
+    mt.hs = pit.hs;
+    mt.he = he;
+    if (n_old > 0) {
+      const uint32_t bytes = (uint32_t)n_old * RB;
+      const long long row = tab.off[pit.j] + r0;
+      mbar_expect_tx(&full[stage], 2 * bytes);
+      bulk_g2s_hint(dk, static_cast<const unsigned char *>(p.K) + row * RB, bytes, &full[stage],
+                    stream_pol);
+      bulk_g2s_hint(dk + TT * RB, static_cast<const unsigned char *>(p.V) + row * RB, bytes,
+                    &full[stage], stream_pol);
+    }
+    pit.advance(tab);
+    ++issued;
+  };
+  auto issue_extra = [&](const Pending &pd, int stage) {  // the step's inputs, then arrive
+    unsigned char *dk = stages + stage * S::kStageBytes;
+    unsigned char *dv = dk + TT * RB;
+    mbar_arrive_expect_tx(&full[stage], (pd.has_new ? 2 * RB : 0) + (pd.first ? RB : 0));
+    if (pd.has_new) {
+      bulk_g2s(dk + pd.slot_new * RB,
+               static_cast<const unsigned char *>(p.k_new) + (size_t)pd.h * RB, RB, &full[stage]);
+      bulk_g2s(dv + pd.slot_new * RB,
+               static_cast<const unsigned char *>(p.v_new) + (size_t)pd.h * RB, RB, &full[stage]);
+    }
+    if (pd.first)
+      bulk_g2s(dv + TT * RB, static_cast<const unsigned char *>(p.q) + (size_t)pd.h * RB, RB,
+               &full[stage]);
+  };
+  Pending pre[NS];
+  int n_pre = 0;
+  if (producer)
+    for (; n_pre < (p.prefetch ? S::kPre : NS) && more(); ++n_pre) issue_old(pre[n_pre]);
+
+  if (p.prefetch) pdl_wait();  // the step's inputs are visible from here on
+  if (tid == 0) STEP_TRACE(2);
+  pdl_launch_dependents();
+
+  if (warp == 0) {
+    // ---- producer ----------------------------------------------------------
+    if (producer) {
+      int armed = 0;  // stages whose producer arrival is done (issued order)
+#pragma unroll
+      for (int j = 0; j < NS; ++j)
+        if (j < n_pre) issue_extra(pre[j], j);
+      armed = n_pre;
+      while (more()) {
+        const int stage = issued % NS;
+        if (s_abort ||
+            (issued >= NS && !mbar_wait(&empty[stage], (uint32_t)(issued / NS - 1) & 1u))) {
+          s_abort = 1;
+          set_err(p.err, HKV_ERR_TIMEOUT);
+          break;
+        }
+        Pending pd;
+        issue_old(pd);
+        issue_extra(pd, stage);
+        armed = issued;
+      }
+      if (!s_abort) {  // no more tiles: a closing record for the consumers
+        const int stage = issued % NS;
+        if (issued >= NS && !mbar_wait(&empty[stage], (uint32_t)(issued / NS - 1) & 1u)) {
+          s_abort = 1;
+          set_err(p.err, HKV_ERR_TIMEOUT);
+        } else {
+          meta[stage].flags = kDone;
+          mbar_arrive(&full[stage]);
+        }
+      }
+      if (s_abort) {
+        // No bulk copy may land in shared memory after the CTA exits: wait
+        // (bounded) for every armed stage that may still be in flight. A
+        // stage reused after an empty-barrier wait is complete already.
+        const int first = armed - NS > 0 ? armed - NS : 0;
+        for (int t = first; t < armed; ++t) mbar_wait(&full[t % NS], (uint32_t)(t / NS) & 1u);
+      }
+    }
+  } else if (warp <= kCW) {
+    // ---- consumers ---------------------------------------------------------
+    const int ctid = tid - 32, cw = warp - 1;
+    const int grp = lane / LPR, col = lane % LPR;
+    using M = LaneMath<T>;
+    static_assert(M::kEPL == EPL, "lane mapping");
+    typename M::Q q;
+    float2 acc[EPL / 2];
+    float m = -INFINITY, l = 0.f;
+    int nseg = 0;
+#pragma unroll
+    for (int e = 0; e < EPL / 2; ++e) acc[e] = make_float2(0.f, 0.f);
+    int n_tiles = 0;
+    // hands one segment's state (or the closing record) to the epilogue
+    auto hand_over = [&](const SegMeta *sm) {
+      const int bb = nseg & 1;
+      if (nseg >= 2 && !s_abort &&
+          !mbar_wait(&epi_free[bb], (uint32_t)((nseg >> 1) - 1) & 1u)) {
+        s_abort = 1;
+        set_err(p.err, HKV_ERR_TIMEOUT);
+      }
+      if (sm) {
+        const int si = cw * RPW + grp;
+        float2 *dst = reinterpret_cast<float2 *>(&red_acc[bb][si][col * EPL]);
+#pragma unroll
+        for (int e = 0; e < EPL / 2; ++e) dst[e] = acc[e];
+        if (col == 0) {
+          red_m[bb][si] = m;
+          red_l[bb][si] = l;
+        }
+        if (cw == 0 && lane == 0) seg[bb] = *sm;
+      } else if (cw == 0 && lane == 0) {
+        seg[bb].h = -1;
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&epi_full[bb]);
+      ++nseg;
+    };
+    for (int tile = 0;; ++tile) {
+      const int stage = tile % NS;
+      if (!s_abort && !mbar_wait(&full[stage], (uint32_t)(tile / NS) & 1u)) {
+        s_abort = 1;
+        set_err(p.err, HKV_ERR_TIMEOUT);
+      }
+      if (s_abort) break;
+      const int flags = meta[stage].flags;
+      if (flags & kDone) break;
+      if (tile == 0 && ctid == 0) STEP_TRACE(3);
+      ++n_tiles;
+      const int nr = meta[stage].n;
+      const unsigned char *Ks = stages + stage * S::kStageBytes;
+      const unsigned char *Vs = Ks + TT * RB;
+      if (flags & kFirst) {  // first tile of this head in this piece
+        M::load_q(q, *reinterpret_cast<const uint4 *>(Vs + TT * RB + col * 16), p.qscale);
+#pragma unroll
+        for (int e = 0; e < EPL / 2; ++e) acc[e] = make_float2(0.f, 0.f);
+        m = -INFINITY;
+        l = 0.f;
+      }
+      float sc[S::kSteps];
+#pragma unroll
+      for (int st = 0; st < S::kSteps; ++st) {
+        const int r = st * (kCW * RPW) + cw * RPW + grp;
+        float dot = 0.f;
+        if (r < nr) dot = M::dot(q, *reinterpret_cast<const uint4 *>(Ks + r * RB + col * 16));
+#pragma unroll
+        for (int o = LPR / 2; o >= 1; o >>= 1) dot += __shfl_xor_sync(0xFFFFFFFFu, dot, o);
+        sc[st] = r < nr ? M::score(dot, p.qscale) : -INFINITY;
+      }
+      float mt = sc[0];
+#pragma unroll
+      for (int st = 1; st < S::kSteps; ++st) mt = fmaxf(mt, sc[st]);
+      const float mn = fmaxf(m, mt);
+      if (mn != -INFINITY) {
+        const float corr = exp2f(m - mn);
+        l *= corr;
+#pragma unroll
+        for (int e = 0; e < EPL / 2; ++e) acc[e] = __fmul2_rn(acc[e], make_float2(corr, corr));
+#pragma unroll
+        for (int st = 0; st < S::kSteps; ++st) {
+          const int r = st * (kCW * RPW) + cw * RPW + grp;
+          if (r < nr) {
+            const float pr = exp2f(sc[st] - mn);
+            l += pr;
+            M::add_v(acc, *reinterpret_cast<const uint4 *>(Vs + r * RB + col * 16), pr);
+          }
+        }
+        m = mn;
+      }
+      if (flags & kLast) {  // last tile of this head in this piece: hand it over
+        SegMeta sm;
+        sm.h = meta[stage].h;
+        sm.hs = meta[stage].hs;
+        sm.he = meta[stage].he;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[stage]);
+        hand_over(&sm);
+      } else {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[stage]);
+      }
+    }
+    if (ctid == 0) STEP_TRACE(4);
+    if (ctid == 0) STEP_TRACE_SET(17, n_tiles);
+    hand_over(nullptr);  // nothing more
+  } else if (warp == kCW + 1) {
+    // ---- epilogue: combine each segment's row-group states ----------------
+    if (!mbar_wait(&ep_bar, 0u)) {  // the launch's epoch (merge warp)
+      s_abort = 1;
+      set_err(p.err, HKV_ERR_TIMEOUT);
+    }
+    int k = 0;
+    for (;; ++k) {
+      const int bb = k & 1;
+      if (!s_abort && !mbar_wait(&epi_full[bb], (uint32_t)(k >> 1) & 1u)) {
+        s_abort = 1;
+        set_err(p.err, HKV_ERR_TIMEOUT);
+      }
+      if (s_abort) break;
+      const SegMeta sg = seg[bb];
+      if (sg.h < 0) break;
+      const int h = sg.h;
+      const long long hs = sg.hs, he = sg.he;
+      // lane s < NST weighs state s
+      const float ms = lane < NST ? red_m[bb][lane] : -INFINITY;
+      float mx = ms;
+#pragma unroll
+      for (int o = 16; o >= 1; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, o));
+      const float ws = ms == -INFINITY ? 0.f : exp2f(ms - mx);
+      float L = lane < NST ? red_l[bb][lane] * ws : 0.f;
+#pragma unroll
+      for (int o = 16; o >= 1; o >>= 1) L += __shfl_xor_sync(0xFFFFFFFFu, L, o);
+      float A[CPL];
+#pragma unroll
+      for (int c = 0; c < CPL; ++c) A[c] = 0.f;
+#pragma unroll
+      for (int si = 0; si < NST; ++si) {
+        const float sw = __shfl_sync(0xFFFFFFFFu, ws, si);
+        float r[CPL];
+        V::lds(&red_acc[bb][si][CPL * lane], r);
+#pragma unroll
+        for (int c = 0; c < CPL; ++c) A[c] = fmaf(r[c], sw, A[c]);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&epi_free[bb]);  // the consumers may reuse the buffer
+      if (hs >= a && he <= b) {  // the whole head is in this CTA's range
+#pragma unroll
+        for (int c = 0; c < CPL; ++c) A[c] /= L;
+        V::st(p.out + (size_t)h * D + CPL * lane, A);
+      } else if (h == s_mg_h) {  // this CTA combines the head: to the merge warp
+        V::st(&own_acc[CPL * lane], A);
+        if (lane == 0) {
+          own_ml[0] = mx;
+          own_ml[1] = L;
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&own_bar);
+      } else {  // a piece for the combining CTA: epoch-tagged, no fence needed
+        unsigned long long *ps = p.pslot + ((size_t)bx * 2 + (hs < a ? 1 : 0)) * (D + 2);
+#pragma unroll
+        for (int c = 0; c < CPL; ++c) st_pair(ps + CPL * lane + c, A[c], s_ep);
+        if (lane == 0) {
+          st_pair(ps + D, mx, s_ep);
+          st_pair(ps + D + 1, L, s_ep);
+        }
+      }
+    }
+    if (lane == 0) STEP_TRACE(5);
+    STEP_TRACE_SET(9, k);
+  } else {
+    // ---- merge warp: barrier, appends, counters, the combined split head ---
+    // Arrive on the layer's barrier word: this CTA is done reading counters.
+    // The last of the grid to arrive resets the count and bumps the
+    // generation, which the others watch.
+    uint32_t gen0 = 0;
+    int bar_done = 0;
+    if (lane == 0) {
+      gen0 = ld_acquire(p.bar + 1);
+      const uint32_t old = atomicAdd(p.bar, 1u);
+      if (old == (uint32_t)G - 1) {
+        p.bar[0] = 0;
+        st_release(p.bar + 1, gen0 + 1);
+        bar_done = 1;
+      }
+    }
+    gen0 = __shfl_sync(0xFFFFFFFFu, gen0, 0);
+    bar_done = __shfl_sync(0xFFFFFFFFu, bar_done, 0);
+    // the launch's epoch, unique per (layer, launch of that layer)
+    const uint32_t ep = (gen0 + 1u) * (uint32_t)p.n_layers + (uint32_t)(p.layer_base / nheads);
+    if (lane == 0) {
+      s_ep = ep;
+      // The split head this CTA combines, if any: the head of its range's
+      // first index when this CTA is that head's first middle CTA (its whole
+      // range inside the head) or, for a head in two pieces, holds its last
+      // row.
+      if (active && tab.start[0] < a) {
+        const long long hs0 = tab.start[0], he0 = hs0 + tab.vlen[0];
+        const long long k0 = hs0 / chunk, k1 = (he0 - 1) / chunk;
+        const long long np = k1 - k0 + 1;
+        if ((np >= 3 ? k0 + 1 : k1) == bx) {
+          s_mg_k0 = k0;
+          s_mg_np = (int)np;
+          s_mg_j = (int)(bx - k0);
+          s_mg_h = h0;
+        }
+      }
+    }
+    __syncwarp();
+    mbar_arrive(&ep_bar);  // all 32 lanes: the epilogue may read s_ep, s_mg_*
+    const uint64_t t0 = globaltimer();
+    auto timed_out = [&]() {
+      if (globaltimer() - t0 <= kWaitTimeoutNs) return false;
+      if (lane == 0) {
+        s_abort = 1;
+        set_err(p.err, HKV_ERR_TIMEOUT);
+      }
+      return true;
+    };
+
+    // Appends: the CTA holding a head's last row writes the new token (K/V
+    // row at index len, its position, q into the ring of the periodic
+    // update). Nothing in this launch reads them, so they go first, while
+    // the consumers stream. The inputs are visible (after the wait above).
+    if (active) {
+      for (int j0 = 0; j0 < n; j0 += 32) {  // ntok of 32 heads per round
+        const int j = j0 + lane;
+        if (j < n && tab.start[j] + tab.vlen[j] > a && tab.start[j] + tab.vlen[j] <= b)
+          tab.ntok[j] = p.ntok[p.layer_base + h0 + j];
+      }
+      __syncwarp();
+      constexpr int CH = RB / 16;                // 16-byte chunks of a row
+      constexpr int PER = (3 * CH + 31) / 32;    // chunks of the K, V, q rows per lane
+      for (int j = 0; j < n; ++j) {
+        const long long he = tab.start[j] + tab.vlen[j];
+        if (he <= a || he > b) continue;
+        const int h = h0 + j, i = p.layer_base + h;
+        const int ntj = tab.ntok[j];
+        const long long row = tab.off[j] + tab.vlen[j] - 1;
+        const unsigned char *src[3] = {static_cast<const unsigned char *>(p.k_new),
+                                       static_cast<const unsigned char *>(p.v_new),
+                                       static_cast<const unsigned char *>(p.q)};
+        unsigned char *dst[3] = {static_cast<unsigned char *>(p.K) + row * RB,
+                                 static_cast<unsigned char *>(p.V) + row * RB,
+                                 static_cast<unsigned char *>(p.qbuf) +
+                                     ((size_t)i * p.period + ntj % p.period) * RB};
+        uint4 x[PER];
+#pragma unroll
+        for (int u = 0; u < PER; ++u) {
+          const int c = lane + 32 * u;
+          if (c < 3 * CH)
+            x[u] = reinterpret_cast<const uint4 *>(src[c / CH] + (size_t)h * RB)[c % CH];
+        }
+#pragma unroll
+        for (int u = 0; u < PER; ++u) {
+          const int c = lane + 32 * u;
+          if (c < 3 * CH) reinterpret_cast<uint4 *>(dst[c / CH])[c % CH] = x[u];
+        }
+        if (lane == 0) p.pos[row] = p.n_cond + ntj;
+      }
+    }
+    STEP_TRACE_SET(8, globaltimer());
+
+    // counters of the heads this CTA appended, once every CTA has read them
+    while (!s_abort && !bar_done) {
+      if (lane == 0) bar_done = ld_acquire(p.bar + 1) != gen0;
+      bar_done = __shfl_sync(0xFFFFFFFFu, bar_done, 0);
+      if (!bar_done && timed_out()) break;
+    }
+    __syncwarp();
+    STEP_TRACE_SET(19, globaltimer());
+    if (!s_abort && active) {
+      for (int j = lane; j < n; j += 32) {
+        const long long hs = tab.start[j], he = hs + tab.vlen[j];
+        if (he > a && he <= b) {
+          const int h = h0 + j, i = p.layer_base + h;
+          p.len[h] = tab.vlen[j];
+          p.ntok[i] = tab.ntok[j] + 1;
+          if (tab.label[j] != HKV_DENSE) p.nbuf[i] = tab.nbuf[j] + 1;
+        }
+      }
+    }
+
+    // The split head this CTA combines: the other pieces, combined in index
+    // order once all of them carry this launch's epoch, then this CTA's own
+    // piece (from the epilogue), so the result does not depend on timing.
+    const int mh = s_mg_h;
+    if (mh >= 0 && !s_abort) {
+      const int np = s_mg_np, mj = s_mg_j;
+      const long long k0 = s_mg_k0;
+      float om = -INFINITY, ol = 0.f, oA[CPL];
+#pragma unroll
+      for (int c = 0; c < CPL; ++c) oA[c] = 0.f;
+      for (;;) {
+        bool ready = true;
+        om = -INFINITY;
+        ol = 0.f;
+#pragma unroll
+        for (int c = 0; c < CPL; ++c) oA[c] = 0.f;
+        for (int t = 0; t < np && ready; ++t) {
+          if (t == mj) continue;
+          // piece t: the end piece of CTA k0, the start piece of the others
+          const unsigned long long *ps = p.pslot + ((size_t)(k0 + t) * 2 + (t > 0 ? 1 : 0)) * (D + 2);
+          float At[CPL], mt, lt;
+          bool ok = true;
+#pragma unroll
+          for (int c = 0; c < CPL; ++c) ok &= ld_pair(ps + CPL * lane + c, s_ep, At[c]);
+          ok &= ld_pair(ps + D, s_ep, mt);
+          ok &= ld_pair(ps + D + 1, s_ep, lt);
+          ready = __all_sync(0xFFFFFFFFu, ok);
+          if (!ready) break;
+          const float mn = fmaxf(om, mt);
+          const float co = om == -INFINITY ? 0.f : exp2f(om - mn);
+          const float ct = mt == -INFINITY ? 0.f : exp2f(mt - mn);
+          ol = ol * co + lt * ct;
+#pragma unroll
+          for (int c = 0; c < CPL; ++c) oA[c] = fmaf(At[c], ct, oA[c] * co);
+          om = mn;
+        }
+        if (ready || timed_out()) break;
+      }
+      // this CTA's own piece
+      while (!s_abort && !mbar_try_wait(&own_bar, 0u))
+        if (timed_out()) break;
+      __syncwarp();
+      if (!s_abort) {
+        const float m1 = own_ml[0], l1 = own_ml[1];
+        float A1[CPL];
+        V::lds(&own_acc[CPL * lane], A1);
+        const float mx = fmaxf(m1, om);
+        const float w1 = m1 == -INFINITY ? 0.f : exp2f(m1 - mx);
+        const float w2 = om == -INFINITY ? 0.f : exp2f(om - mx);
+        const float Lt = l1 * w1 + ol * w2;
+        float A[CPL];
+#pragma unroll
+        for (int c = 0; c < CPL; ++c) A[c] = fmaf(A1[c], w1, oA[c] * w2) / Lt;
+        V::st(p.out + (size_t)mh * D + CPL * lane, A);
+      }
+      STEP_TRACE_SET(18, globaltimer());
+    }
+    if (lane == 0) STEP_TRACE(6);
+  }
+}
+
+template <int D, typename T>
+size_t step_smem() {
+  return (size_t)StepShape<D, T>::kNS * StepShape<D, T>::kStageBytes;
+}
+
+template <int D, typename T>
+cudaError_t step_prepare_t(int *ctas) {
+  const size_t smem = step_smem<D, T>();
+  cudaError_t e = cudaFuncSetAttribute(step_kernel<D, T>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas, step_kernel<D, T>,
+                                                       step_threads<D, T>(), smem);
+}
+
+template <int D, typename T>
+cudaError_t step_launch_t(const AttnArgs &a, int grid, cudaStream_t s) {
+  static const bool pdl = getenv("HKV_NO_PDL") == nullptr;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(step_threads<D, T>());
+  cfg.dynamicSmemBytes = step_smem<D, T>();
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, step_kernel<D, T>, a);
+}
+
+}  // namespace
+
+#ifdef HKV_ATTN_TRACE
+extern "C" int hkv_debug_set_step_trace(unsigned long long *buf) {
+  return cudaMemcpyToSymbol(g_step_trace, &buf, sizeof(buf)) == cudaSuccess ? 0 : 7;
+}
+#endif
+
+int step_tile_rows(int D, int dtype) {
+  if (dtype == HKV_BF16) return D == 64 ? StepShape<64, __nv_bfloat16>::kTT : StepShape<128, __nv_bfloat16>::kTT;
+  return D == 64 ? StepShape<64, float>::kTT : StepShape<128, float>::kTT;
+}
+
+cudaError_t step_prepare(int D, int dtype, int *ctas) {
+  if (dtype == HKV_BF16)
+    return D == 64 ? step_prepare_t<64, __nv_bfloat16>(ctas) : step_prepare_t<128, __nv_bfloat16>(ctas);
+  return D == 64 ? step_prepare_t<64, float>(ctas) : step_prepare_t<128, float>(ctas);
+}
+
+cudaError_t launch_step(const AttnArgs &a, int D, int dtype, int grid, cudaStream_t s) {
+  if (grid < 1 || grid > kAttnMaxGrid) return cudaErrorInvalidValue;
+  if (dtype == HKV_BF16)
+    return D == 64 ? step_launch_t<64, __nv_bfloat16>(a, grid, s)
+                   : step_launch_t<128, __nv_bfloat16>(a, grid, s);
+  return D == 64 ? step_launch_t<64, float>(a, grid, s) : step_launch_t<128, float>(a, grid, s);
+}
+
+}  // namespace hkv

@@ -95,11 +95,9 @@ class Engine:
                           flags, self.stream())
 
     def update_due(self, t: int) -> bool:
-        """Whether image token t's step starts with the periodic update: the
-        buffer filled P steps after grouping (image token E-1) and every P
-        steps since."""
-        E, P = self.cfg.group_at, self.cfg.period
-        return t > E and (t - E) % P == 0
+        """Whether image token t's step starts with the periodic update
+        (decided by the library, hkv_update_due)."""
+        return H.hkv_update_due(self.cfg, t)
 
     # Step 2
     def step_identify(self, layer: int, q, k, v, out) -> None:

@@ -9,7 +9,6 @@ import of a function fails loudly.
 from __future__ import annotations
 
 import ctypes
-import math
 import os
 from ctypes import POINTER, Structure, c_char_p, c_double, c_int, c_int32, c_int64, c_size_t, c_void_p
 from fractions import Fraction
@@ -76,6 +75,9 @@ _SIGNATURES = {
     "hkv_decode_step_identify": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p, c_void_p,
                                   c_void_p, c_void_p, c_void_p, c_void_p, c_size_t, c_int, c_void_p],
                                  c_int),
+    "hkv_decode_step_launches": ([POINTER(hkv_config)], c_int),
+    "hkv_global_budget": ([c_int64, c_int64, c_int32, POINTER(c_int32)], c_int),
+    "hkv_update_due": ([POINTER(hkv_config), c_int32, POINTER(c_int32)], c_int),
     "hkv_evict": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p], c_int),
     "hkv_identify_heads": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p, c_void_p, c_void_p,
                             c_void_p], c_int),
@@ -127,15 +129,30 @@ def make_config(*, n_layers, n_seqs, n_heads, head_dim, dtype, n_cond, n_image, 
                 recent_w, local_w, period, group_at, rho=None, global_budget=None,
                 tau=0.9, r_s=0.5, budget_mode=HKV_BUDGET_PAPER,
                 distance_mode=HKV_DIST_RASTER) -> hkv_config:
-    """Builds an hkv_config; the global budget is floor(rho * N) (Sec. 5.1)
-    unless given explicitly."""
+    """Builds an hkv_config; the global budget is the library's
+    hkv_global_budget(rho, N) unless given explicitly."""
     if global_budget is None:
-        global_budget = math.floor(Fraction(rho) * n_image)
+        global_budget = hkv_global_budget(rho, n_image)
     return hkv_config(n_layers, n_seqs, n_heads, head_dim,
                       HKV_BF16 if dtype in ("bf16", HKV_BF16) else HKV_FP32,
                       n_cond, n_image, row_len, recent_w, local_w, period, group_at,
                       int(global_budget), int(budget_mode), int(distance_mode), 0, float(tau),
                       float(r_s))
+
+
+def hkv_global_budget(rho, n_image: int) -> int:
+    """B_g for a budget ratio rho (a Fraction, or anything Fraction takes)."""
+    r = Fraction(rho)
+    out = c_int32(0)
+    _call("global_budget", r.numerator, r.denominator, n_image, ctypes.byref(out))
+    return int(out.value)
+
+
+def hkv_update_due(cfg: hkv_config, t: int) -> bool:
+    """Whether image token t's decode step starts with the periodic update."""
+    out = c_int32(0)
+    _call("update_due", ctypes.byref(cfg), t, ctypes.byref(out))
+    return bool(out.value)
 
 
 def hkv_validate_config(cfg: hkv_config) -> None:
@@ -167,6 +184,15 @@ def hkv_decode_step(cfg, cache, layer, q, k, v, out, workspace, ws_bytes, flags=
                     stream=0) -> None:
     _call("decode_step", ctypes.byref(cfg), ctypes.byref(cache), layer, _p(q), _p(k), _p(v), _p(out),
           _p(workspace), ws_bytes, flags, stream)
+
+
+def hkv_decode_step_launches(cfg) -> int:
+    """Kernel launches of one hkv_decode_step call (1 or 2) on the current
+    device; raises on an invalid config."""
+    n = int(lib().hkv_decode_step_launches(ctypes.byref(cfg)))
+    if n <= 0:
+        raise HkvError("decode_step_launches", HKV_ERR_INVALID_ARG)
+    return n
 
 
 def hkv_decode_step_identify(cfg, cache, layer, q, k, v, out, label_out, workspace, ws_bytes,

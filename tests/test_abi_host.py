@@ -47,7 +47,7 @@ def fake_cache(H, **kw):
 
 def test_every_declared_symbol_is_exported(H):
     names = declared_functions()
-    assert len(names) == 17
+    assert len(names) == 20
     for n in names:
         assert hasattr(H.lib(), n), n
     assert set(names) >= {"hkv_identify_heads", "hkv_allocate_budgets", "hkv_append_evict",
@@ -245,3 +245,37 @@ def test_engine_update_schedule_matches_the_oracle(H, period, group_at):
     fake = Cfg()
     fake.cfg = tiny_cfg(H, period=period, group_at=group_at, n_image=w.n_image)
     assert [t for t in range(w.n_image) if Engine.update_due(fake, t)] == oracle_steps
+
+
+def test_global_budget_is_the_oracle_rule(H):
+    """hkv_global_budget (Sec. 5.1, B_g = floor(rho N)) against the oracle's
+    global_budget: Table 3's B column and a sweep of ratios and grid sizes."""
+    from fractions import Fraction
+    from oracle import headkv as O
+    assert H.hkv_global_budget(Fraction(1, 4), 576) == 144
+    assert H.hkv_global_budget(Fraction(1, 6), 576) == 96
+    assert H.hkv_global_budget(Fraction(1, 8), 576) == 72
+    assert H.hkv_global_budget(Fraction(1, 8), 2352) == 294
+    for den in range(1, 13):
+        for num in range(1, den + 1):
+            for n in (1, 7, 256, 576, 2352, 4160, 9999):
+                r = Fraction(num, den)
+                assert H.hkv_global_budget(r, n) == O.global_budget(r, n), (r, n)
+    lib = H.lib()
+    out = ctypes.c_int32(0)
+    for args in [(0, 4, 100), (5, 4, 100), (1, 0, 100), (1, 4, 0), (-1, 4, 100), (1, 1 << 40, 10)]:
+        assert lib.hkv_global_budget(*args, ctypes.byref(out)) == 1, args
+    assert lib.hkv_global_budget(1, 4, 100, None) == 1
+
+
+def test_update_due_rejects_bad_arguments(H):
+    lib = H.lib()
+    out = ctypes.c_int32(0)
+    cfg = tiny_cfg(H)
+    assert lib.hkv_update_due(ctypes.byref(cfg), -1, ctypes.byref(out)) == 1
+    assert lib.hkv_update_due(ctypes.byref(cfg), 3, None) == 1
+    assert lib.hkv_update_due(ctypes.byref(tiny_cfg(H, head_dim=32)), 3, ctypes.byref(out)) == 2
+
+
+def test_decode_step_launches_answers_zero_for_a_bad_config(H):
+    assert H.lib().hkv_decode_step_launches(ctypes.byref(tiny_cfg(H, head_dim=32))) == 0

@@ -50,9 +50,14 @@ def run_case(lens, D, dtype, seed, n_layers=1, layer=0, repeat=2):
                                torch.cuda.current_stream().cuda_stream)
         outs.append(out.cpu().numpy())
     H.hkv_check(cb.c)
-    # the workspace ends with the kernels' 256-byte control block: the launch
-    # passed its checks (int32 at byte 0)
-    ctl = ws[-256:].view(torch.int32)
+    # the control block after the partial slots (4 per CTA boundary and one
+    # per CTA, D + 4 floats each) and the boundary records (16 bytes per CTA),
+    # 4096 CTAs at most, every region 256-byte aligned: the launch passed its
+    # checks (int32 at byte 0)
+    a256 = lambda b: (b + 255) // 256 * 256
+    pf = (D + 4) * 4
+    at = a256(4096 * 4 * pf) + a256(4096 * pf) + a256(4096 * 16)
+    ctl = ws[at:at + 256].view(torch.int32)
     assert int(ctl[0]) == 1
     Kx = cb.k.float().cpu().numpy().astype(np.float64)
     Vx = cb.v.float().cpu().numpy().astype(np.float64)
