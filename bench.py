@@ -72,31 +72,48 @@ def describe(w, n_steps_window):
             f"period of P decode steps x L layers")
 
 
-def profiled_traffic(workload, bytes_per_launch):
-    """DRAM bytes per decode step from the committed ncu summary: the
-    attention kernel's measured traffic ratio to its algorithmic bytes, scaled
-    to this launch, plus the finishing kernel's bytes per launch (set by the
-    grid: one CTA boundary's record and slots per warp). None for another
-    kernel instantiation (the capture is of the Lumina-1024 shape: D = 128,
-    bf16) or when the kernel source has changed since the capture."""
-    if workload != "lumina1024":
-        return None
+# the kernel sources of each decode-step design (one launch / two kernels),
+# hashed together: a committed ncu capture applies while they are unchanged
+STEP_SOURCES = {1: ["hkv_step.cu", "hkv_attn_common.cuh", "hkv_device.cuh"],
+                2: ["hkv_attention.cu", "hkv_attn_common.cuh", "hkv_device.cuh"]}
+
+
+def sources_digest(launches: int) -> str | None:
     import hashlib
-    path = os.path.join(ROOT, "profiles", "decode_step_lumina1024_rho4.md")
-    src = os.path.join(ROOT, "paper_2605_20600_gb300", "csrc", "hkv_attention.cu")
+    h = hashlib.sha256()
     try:
-        vals = {}
-        for line in open(path):
-            k, _, v = line.strip().partition(": ")
-            if k in ("source_sha256", "attn_traffic_ratio", "finish_traffic_bytes_per_launch"):
-                vals[k] = v
-        with open(src, "rb") as f:
-            if hashlib.sha256(f.read()).hexdigest() != vals["source_sha256"]:
-                return None
-        return (float(vals["attn_traffic_ratio"]) * bytes_per_launch
-                + float(vals["finish_traffic_bytes_per_launch"]))
-    except (OSError, KeyError, ValueError):
+        for f in STEP_SOURCES[launches]:
+            with open(os.path.join(ROOT, "paper_2605_20600_gb300", "csrc", f), "rb") as fh:
+                h.update(fh.read())
+    except (OSError, KeyError):
         return None
+    return h.hexdigest()
+
+
+def profiled_traffic(workload, bytes_per_launch, launches=2):
+    """DRAM bytes per decode step from a committed ncu summary (profiles/*.md
+    with the keys capture_of, launches, sources_sha256, traffic_ratio and
+    extra_bytes_per_launch): the captured kernels' DRAM traffic over their
+    algorithmic bytes, scaled to this launch, plus bytes that do not scale
+    with it. None without a capture of this workload and design whose kernel
+    sources are the current ones."""
+    import glob
+    digest = sources_digest(launches)
+    if digest is None:
+        return None
+    for path in sorted(glob.glob(os.path.join(ROOT, "profiles", "*.md"))):
+        vals = {}
+        try:
+            for line in open(path):
+                k, _, v = line.strip().partition(": ")
+                vals[k] = v
+            if (vals.get("capture_of") == workload and vals.get("launches") == str(launches)
+                    and vals.get("sources_sha256") == digest):
+                return (float(vals["traffic_ratio"]) * bytes_per_launch
+                        + float(vals.get("extra_bytes_per_launch", "0")))
+        except (OSError, KeyError, ValueError):
+            continue
+    return None
 
 
 def max_over_ranks(x: float, device) -> float:
@@ -152,42 +169,73 @@ def _oracle_period(args):
 def oracle_rate(w, t0, n_heads, seed, workers):
     """Projected image tokens/s of the CPU oracle from a sample of heads: the
     oracle time of one period for each sampled head (its run up to the window
-    minus its run to the window start), averaged, times all L*S*H heads."""
+    minus its run to the window start), averaged, times all L*S*H heads
+    shared by `workers` processes. Returns the rate, the mean seconds per
+    head-period and the wall time of the sample."""
     import random
     rnd = random.Random(seed)
     heads = [(rnd.randrange(w.n_seqs), rnd.randrange(w.n_layers), rnd.randrange(w.n_heads))
              for _ in range(n_heads)]
     jobs = [(w, x, t0) for x in heads]
+    tw = time.perf_counter()
     with mp.get_context("spawn").Pool(workers) as pool:
         secs = pool.map(_oracle_period, jobs, chunksize=1)
+    wall = time.perf_counter() - tw
     per_head_period = statistics.mean(secs)
     period_s = per_head_period * w.n_head_total / workers
     images = w.n_seqs / w.cfg_rows
-    return images * w.period / period_s, per_head_period
+    return images * w.period / period_s, per_head_period, wall
+
+
+def cpu_baseline(w, t0):
+    """The oracle on the host's cores: one process, and one process per core
+    (os.cpu_count()), each on a sample of heads for one period, projected to
+    every head of the model."""
+    nproc = os.cpu_count() or 1
+    one, ph1, wall1 = oracle_rate(w, t0, 16, 7, 1)
+    n_all = 64 * nproc
+    rate, ph, wall = oracle_rate(w, t0, n_all, 8, nproc)
+    return {"value": rate, "unit": "image tokens/s", "cores": nproc, "kind": "oracle",
+            "nproc": nproc, "single_process": one,
+            "sample": f"{n_all} random heads of {w.n_head_total} on {nproc} processes (one per "
+                      f"core), one period each (P={w.period} steps incl. the update) after a "
+                      f"simulated run to step {t0}: mean {ph * 1e3:.1f} ms per head-period, "
+                      f"{wall:.1f} s wall; the value is projected to all heads "
+                      f"(x {w.n_head_total / n_all:.0f}). One process: 16 heads, "
+                      f"{ph1 * 1e3:.1f} ms per head-period, {one:.1f} image tokens/s projected"}
 
 
 def run_reference(args):
-    """--impl reference: the CPU oracle as the reference arm."""
+    """--impl reference: the CPU oracle as the reference arm. Each step times
+    the oracle on a sample of heads on every host core and projects it to the
+    whole model; the line says so and gives the wall time actually spent."""
     w = workload(args)
     t0 = steady_start(w)
-    workers = min(16, os.cpu_count() or 1)
-    vals = []
+    nproc = os.cpu_count() or 1
+    n_heads = 4 * nproc
+    vals, walls = [], []
+    tw = time.perf_counter()
     for j in range(args.warmup + args.steps):
-        v, _ = oracle_rate(w, t0, 4 * workers, 1000 + j, workers)
+        v, _, wall = oracle_rate(w, t0, n_heads, 1000 + j, nproc)
         if j >= args.warmup:
             vals.append(v)
+            walls.append(wall)
     value = statistics.mean(vals)
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "image tokens/s",
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1000.0 * (w.n_seqs / w.cfg_rows) * w.period / value,
+        "ms_per_step_projected": True,
+        "measured_wall_s": time.perf_counter() - tw,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": bench_config(w, args.gpus),
-        "cpu_baseline": {"value": value, "unit": "image tokens/s", "cores": workers,
-                         "kind": "oracle",
-                         "sample": f"per step {4 * workers} random heads, one period each after "
-                                   f"a simulated run to step {t0}, projected to all "
-                                   f"{w.n_head_total} heads"},
+        "cpu_baseline": {"value": value, "unit": "image tokens/s", "cores": nproc,
+                         "kind": "oracle", "nproc": nproc,
+                         "sample": f"per step {n_heads} random heads of {w.n_head_total}, one "
+                                   f"period each after a simulated run to step {t0}, on {nproc} "
+                                   f"processes; ms_per_step is projected to all heads "
+                                   f"(x {w.n_head_total / n_heads:.0f}), the timed samples took "
+                                   f"{statistics.mean(walls):.2f} s wall each"},
         "e2e": {"value": value, "unit": "image tokens/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -247,43 +295,25 @@ class ClockSampler:
                 "samples": len(rows)}
 
 
-def run_ours(args):
+def measure_period(args, w, dev, world, K, W, *, e2e: bool):
+    """One workload on the GPU: generation up to the steady-state window, then
+    K timed periods (after W warm-up periods) replayed from a CUDA graph.
+    Returns the device time, per-launch roofline figures and (e2e) the same
+    metric through pinned host buffers."""
     import numpy as np
     import torch
     import torch.distributed as dist
-
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    if world > 1:
-        dist.init_process_group("nccl")
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
 
     from paper_2605_20600_gb300 import hkv as H
     from paper_2605_20600_gb300.engine import Engine, torch_dtype
     from paper_2605_20600_gb300.runner import generate
     from synth.gpu import DeviceSynth
 
-    w = workload(args)
     L, S, Hh, D, P = w.n_layers, w.n_seqs, w.n_heads, w.head_dim, w.period
     t0 = steady_start(w)
-    K, W = args.steps, args.warmup
     # resident input periods (fresh inputs for every timed period while they
     # fit in the image; beyond that the pool is reused cyclically)
     n_pool = max(1, min(W + K, (w.n_image - t0) // P))
-
-    # CPU baseline first (spawned workers, rank 0, one GPU)
-    cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        workers = min(16, os.cpu_count() or 1)
-        rate, per_head = oracle_rate(w, t0, 4 * workers, 7, workers)
-        cpu = {"value": rate, "unit": "image tokens/s", "cores": workers, "kind": "oracle",
-               "sample": f"{4 * workers} random heads of {w.n_head_total}, one period each "
-                         f"(P={P} steps incl. the update) after a simulated run to step {t0}; "
-                         f"mean {per_head * 1e3:.1f} ms per head-period, projected to all heads "
-                         f"on {workers} processes"}
-
     redistribute = args.budget == "redistribute"
     grid2d = args.distance == "grid2d"
     cfg = H.make_config(n_layers=L, n_seqs=S, n_heads=Hh, head_dim=D, dtype=w.dtype,
@@ -332,9 +362,10 @@ def run_ours(args):
     with torch.cuda.graph(graph):
         period_calls()
     stream = torch.cuda.current_stream()
-    # per period: every decode step is an attention and a finishing kernel;
-    # every layer's update is one kernel
-    launches_per_step = 2 * P * L + L
+    # per period: the kernels of every decode step (one launch, or an
+    # attention and a finishing kernel) and every layer's update kernel
+    step_launches = H.hkv_decode_step_launches(cfg)
+    launches_per_step = step_launches * P * L + L
 
     def barrier():
         if world > 1:
@@ -342,7 +373,7 @@ def run_ours(args):
 
     j = 0
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with ClockSampler(local) as clk:
+    with ClockSampler(torch.cuda.current_device()) as clk:
         time.sleep(1.0)           # the sampler is up before the GPU gets busy
         for _ in range(W):
             staging.copy_(pool[j % n_pool], non_blocking=True)
@@ -364,8 +395,6 @@ def run_ours(args):
     clocks = clk.summary()
     eng.check()
     ms = max_over_ranks(ms, dev)
-    images = S / w.cfg_rows
-    value = job_value(world, images, P, K, ms)
 
     # dominant kernel: the fused decode step (append + attention). One more
     # period is replayed from a copy of the graph with an event pair around
@@ -397,79 +426,142 @@ def run_ours(args):
     # average decode-step launch in the timed graph: the period's device time
     # minus the updates and the input copy (timed above), per launch
     attn_us = (ms * 1e3 / K - sum(evict_us) - copy_us) / (P * L)
-    peak, peak_kind = load_peaks()
-    achieved = bytes_per_launch / (attn_us / 1e6) / 1e9
+    res = {"ms": ms, "clocks": clocks, "labels": labels, "bytes_per_launch": bytes_per_launch,
+           "per_launch": per_launch, "attn_us": attn_us, "step_us": step_us,
+           "evict_us": evict_us, "copy_us": copy_us, "step_launches": step_launches,
+           "launches_per_step": launches_per_step, "total_tokens": eng.total_tokens,
+           "staging_bytes": staging.numel() * staging.element_size(),
+           "out_bytes": out.numel() * out.element_size()}
 
-    # e2e through the C-ABI with pinned host buffers, pipelined as a caller
-    # would run it: two input/output buffer sets, each with its graph; while
-    # period i computes, a copy stream brings in period i+1's inputs and takes
-    # out period i-1's outputs. The first input copy and the last output copy
-    # are not overlapped; all copies are inside the timed region.
-    staging_b = torch.empty_like(staging)
-    out_b = torch.empty_like(out)
-    graph_b = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(graph_b):
-        period_calls(staging=staging_b, out=out_b)
-    graphs, stg, outs = (graph, graph_b), (staging, staging_b), (out, out_b)
-    host_in = torch.empty(staging.shape, dtype=dt, pin_memory=True)
-    host_out = [torch.empty(out.shape, dtype=torch.float32, pin_memory=True) for _ in range(2)]
-    host_in.copy_(pool[0])
-    copy_stream = torch.cuda.Stream()
-    e2e_steps = max(2, min(K, 10))
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    torch.cuda.synchronize()
-    e0.record(stream)
-    stg[0].copy_(host_in, non_blocking=True)
-    done = None
-    for i in range(e2e_steps):
-        b = i % 2
-        graphs[b].replay()
-        prev_done, done = done, torch.cuda.Event()
-        done.record(stream)
-        with torch.cuda.stream(copy_stream):
-            if prev_done is not None:  # period i-1 released buffer set 1-b
-                copy_stream.wait_event(prev_done)
-                host_out[1 - b].copy_(outs[1 - b], non_blocking=True)
-            if i + 1 < e2e_steps:
-                stg[1 - b].copy_(host_in, non_blocking=True)
-            copied = torch.cuda.Event()
-            copied.record(copy_stream)
-        stream.wait_event(copied)
-    last = (e2e_steps - 1) % 2
-    host_out[last].copy_(outs[last], non_blocking=True)
-    e1.record(stream)
-    torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1)
-    eng.check()
-    e2e_value = world * images * P * e2e_steps / (e2e_ms / 1e3)
+    if e2e:
+        # e2e through the C-ABI with pinned host buffers, pipelined as a
+        # caller would run it: two input/output buffer sets, each with its
+        # graph; while period i computes, a copy stream brings in period
+        # i+1's inputs and takes out period i-1's outputs. The first input
+        # copy and the last output copy are not overlapped; all copies are
+        # inside the timed region.
+        staging_b = torch.empty_like(staging)
+        out_b = torch.empty_like(out)
+        graph_b = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph_b):
+            period_calls(staging=staging_b, out=out_b)
+        graphs, stg, outs = (graph, graph_b), (staging, staging_b), (out, out_b)
+        host_in = torch.empty(staging.shape, dtype=dt, pin_memory=True)
+        host_out = [torch.empty(out.shape, dtype=torch.float32, pin_memory=True) for _ in range(2)]
+        host_in.copy_(pool[0])
+        copy_stream = torch.cuda.Stream()
+        e2e_steps = max(2, min(K, 10))
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        stg[0].copy_(host_in, non_blocking=True)
+        done = None
+        for i in range(e2e_steps):
+            b = i % 2
+            graphs[b].replay()
+            prev_done, done = done, torch.cuda.Event()
+            done.record(stream)
+            with torch.cuda.stream(copy_stream):
+                if prev_done is not None:  # period i-1 released buffer set 1-b
+                    copy_stream.wait_event(prev_done)
+                    host_out[1 - b].copy_(outs[1 - b], non_blocking=True)
+                if i + 1 < e2e_steps:
+                    stg[1 - b].copy_(host_in, non_blocking=True)
+                copied = torch.cuda.Event()
+                copied.record(copy_stream)
+            stream.wait_event(copied)
+        last = (e2e_steps - 1) % 2
+        host_out[last].copy_(outs[last], non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        res["e2e_ms"] = e0.elapsed_time(e1)
+        res["e2e_steps"] = e2e_steps
+        eng.check()
+    del eng, pool, staging, out, graph, igraph
+    torch.cuda.empty_cache()
+    return res
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    w = workload(args)
+    P = w.period
+    t0 = steady_start(w)
+    K, W = args.steps, args.warmup
+
+    # CPU baseline first (spawned workers, rank 0, one GPU)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w, t0)
+
+    r = measure_period(args, w, dev, world, K, W, e2e=True)
+    images = w.n_seqs / w.cfg_rows
+    value = job_value(world, images, P, K, r["ms"])
+    peak, peak_kind = load_peaks()
+    achieved = r["bytes_per_launch"] / (r["attn_us"] / 1e6) / 1e9
+    e2e_value = world * images * P * r["e2e_steps"] / (r["e2e_ms"] / 1e3)
+
+    # the other budgets of the same workload (Sec. 5.1's rho): fewer periods
+    sweep = {}
+    spec = args.rho_sweep if args.rho_sweep is not None else (
+        "1/4,1/6,1/8" if w.name == "lumina1024" and not args.seqs else "")
+    for rho in [x for x in spec.split(",") if x and Fraction(x) != w.rho]:
+        ws = w.with_(rho=Fraction(rho))
+        ks, wk = max(3, min(K, 10)), max(3, min(W, 3))
+        rs = measure_period(args, ws, dev, world, ks, wk, e2e=False)
+        ach = rs["bytes_per_launch"] / (rs["attn_us"] / 1e6) / 1e9
+        sweep[rho] = {"value": job_value(world, images, ws.period, ks, rs["ms"]),
+                      "ms_per_step": rs["ms"] / ks, "steps": ks, "warmup": wk,
+                      "achieved": ach, "frac": ach / peak, "bytes_per_launch": rs["bytes_per_launch"],
+                      "launch_us": rs["attn_us"], "evict_us_per_period": sum(rs["evict_us"]),
+                      "global_head_fraction": float((rs["labels"] == 1).mean()),
+                      "clocks": rs["clocks"]}
 
     if rank == 0:
+        launches = r["step_launches"]
+        kernel = ("hkv_decode_step: step_kernel (one launch: attention, append, merges, counters)"
+                  if launches == 1 else
+                  "hkv_decode_step: attn_kernel<fused> + finish_kernel<fused>")
         line = {
             "metric": METRIC, "value": value, "unit": "image tokens/s", "n_gpus": world,
-            "steps": K, "warmup": W, "ms_per_step": ms / K, "higher_is_better": True,
+            "steps": K, "warmup": W, "ms_per_step": r["ms"] / K, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
             "config": {**bench_config(w, world),
                        **({"budget": "redistributed (aggregate-preserving), arena "
-                                     f"{eng.total_tokens} tokens"} if redistribute else {}),
+                                     f"{r['total_tokens']} tokens"}
+                          if args.budget == "redistribute" else {}),
                        **({"distance": "grid (identification and Eq. 5 strata by squared "
-                                       "distance on the image grid)"} if grid2d else {})},
-            "global_head_fraction": float((labels == 1).mean()),
+                                       "distance on the image grid)"}
+                          if args.distance == "grid2d" else {})},
+            "global_head_fraction": float((r["labels"] == 1).mean()),
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak,
-                         "traffic": profiled_traffic(w.name, bytes_per_launch),
-                         "kernel": "hkv_decode_step: attn_kernel<fused> + finish_kernel<fused>",
-                         "bytes_per_launch": bytes_per_launch, "launch_us": attn_us,
+                         "traffic": profiled_traffic(w.name, r["bytes_per_launch"], launches),
+                         "kernel": kernel,
+                         "bytes_per_launch": r["bytes_per_launch"], "launch_us": r["attn_us"],
                          # the first step of the period, per layer (what a
                          # profiler capturing the first launches sees)
-                         "bytes_first_step": per_launch[:L],
-                         "launch_us_isolated": statistics.mean(step_us),
-                         "evict_us_per_period": sum(evict_us), "copy_us_per_period": copy_us,
+                         "bytes_first_step": r["per_launch"][:w.n_layers],
+                         "launch_us_isolated": statistics.mean(r["step_us"]),
+                         "evict_us_per_period": sum(r["evict_us"]),
+                         "copy_us_per_period": r["copy_us"],
                          "peak_kind": peak_kind},
+            "rho_sweep": sweep,
             "e2e": {"value": e2e_value, "unit": "image tokens/s",
-                    "h2d_bytes_per_step": staging.numel() * staging.element_size(),
-                    "d2h_bytes_per_step": out.numel() * out.element_size()},
-            "gpu_launches": launches_per_step * K,
-            "clocks": clocks,
+                    "h2d_bytes_per_step": r["staging_bytes"],
+                    "d2h_bytes_per_step": r["out_bytes"]},
+            "gpu_launches": r["launches_per_step"] * K,
+            "clocks": r["clocks"],
         }
         if cpu is not None:
             line["cpu_baseline"] = cpu
@@ -798,6 +890,9 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="lumina1024", choices=sorted(configs.ALL))
     ap.add_argument("--rho", default="1/4")
+    ap.add_argument("--rho-sweep", default=None,
+                    help="other budgets measured after the headline one (comma-separated; "
+                         "default 1/4,1/6,1/8 for the Lumina-mGPT-1024 shape, else none)")
     ap.add_argument("--seqs", type=int, default=0, help="override the batch (profiling runs)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--strategies", action="store_true",

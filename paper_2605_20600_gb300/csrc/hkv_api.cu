@@ -269,19 +269,25 @@ hkv_status attn_grid(const hkv_config *cfg, int *grid) {
   return HKV_OK;
 }
 
-// Whether hkv_decode_step runs as one launch (hkv_step.cu): every CTA's range
-// must fit the kernel's head table. A range of c tiles holds at most c + 1
-// heads (a head has at least one tile in a step, its new token), and c is at
-// most the layer's tile count over the grid, bounded by every head at the
-// longest segment the config allows. HKV_STEP_TWO_KERNELS in the
-// environment selects the two-kernel design regardless (tests of both).
+// Whether hkv_decode_step runs as one launch (hkv_step.cu). It must fit the
+// kernel's head table: a range of c tiles holds at most c + 1 heads (a head
+// has at least one tile in a step, its new token), and c is at most the
+// layer's tile count over the grid, bounded by every head at the longest
+// segment the config allows. Measured on GB300 (each shape A/B in one
+// process): one launch is faster while a layer has at most one head per CTA
+// (Lumina-mGPT-1024: 256 heads on 304 CTAs, 2-3 % per step), the two-kernel
+// design from about two heads per CTA on (Lumina-mGPT-768, Janus-Pro-7B,
+// LlamaGen-XL: 1-3 %). HKV_STEP_TWO_KERNELS / HKV_STEP_ONE_LAUNCH in the
+// environment force either design (tests of both).
 bool one_launch_step(const hkv_config *cfg, int grid) {
   if (getenv("HKV_STEP_TWO_KERNELS")) return false;
   const long long tt = step_tile_rows(cfg->head_dim, cfg->dtype);
   const long long tiles = (long long)heads_per_layer(cfg) * ((max_segment(cfg) + tt - 1) / tt);
   long long chunk = (tiles + grid - 1) / grid;
   if (chunk < 2) chunk = 2;
-  return chunk + 1 <= kStepTable;
+  if (chunk + 1 > kStepTable) return false;
+  if (getenv("HKV_STEP_ONE_LAUNCH")) return true;
+  return heads_per_layer(cfg) <= grid;
 }
 
 #define HKV_TRY(x)                 \

@@ -99,6 +99,7 @@ int step_tile_rows(int D, int dtype);
 #define HKV_STEP_ACTIVE_PER_SM 2
 #endif
 constexpr int kStepActivePerSm = HKV_STEP_ACTIVE_PER_SM;
+
 cudaError_t step_prepare(int D, int dtype, int *ctas_per_sm);
 // the fused decode step of one layer in one launch (append + attention,
 // merges of split heads and counters in the same kernel); `grid` CTAs, at

@@ -103,7 +103,7 @@ __device__ unsigned long long *g_step_trace = nullptr;  // [layer][kAttnMaxGrid]
 #endif
 // heads of a thread's prologue slice kept in registers (more: reloaded)
 #ifndef HKV_STEP_SLICE_REGS
-#define HKV_STEP_SLICE_REGS 8
+#define HKV_STEP_SLICE_REGS 1
 #endif
 
 template <int D, typename T>
@@ -159,6 +159,26 @@ struct StepIter {
   }
 };
 
+// The split of a layer's index space [0, total) into the CTAs' ranges: CTA k
+// streams [start(k), start(k + 1)), `chunk` slots each (whole tiles, at
+// least two), the last ones possibly shorter or empty.
+template <int TT>
+struct Ranges {
+  long long total, chunk;
+  int G;
+  __device__ void init(long long total_, int G_, long long min_chunk) {
+    total = total_;
+    G = G_;
+    chunk = slot_len<TT>((total + G - 1) / G);
+    if (chunk < min_chunk) chunk = min_chunk;
+  }
+  __device__ long long start(int k) const {
+    const long long s = (long long)k * chunk;
+    return k >= G || s > total ? total : s;
+  }
+  __device__ int owner(long long slot) const { return (int)(slot / chunk); }  // CTA holding slot
+};
+
 __device__ __forceinline__ uint32_t ld_acquire(const uint32_t *p) {
   uint32_t v;
   asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
@@ -179,6 +199,23 @@ __device__ __forceinline__ bool ld_pair(const unsigned long long *p, uint32_t ep
   asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(w) : "l"(p) : "memory");
   v = __uint_as_float((uint32_t)w);
   return (uint32_t)(w >> 32) == ep;
+}
+
+// Combines a split head's own piece (m1, l1, A1) with its other pieces,
+// already combined (m2, l2, A2), and stores the output row: the same
+// instructions wherever it runs, so the result does not depend on which
+// warp does it.
+template <int CPL>
+__device__ __forceinline__ void combine_store(float m1, float l1, const float *A1, float m2,
+                                              float l2, const float *A2, float *out) {
+  const float mx = fmaxf(m1, m2);
+  const float w1 = m1 == -INFINITY ? 0.f : exp2f(m1 - mx);
+  const float w2 = m2 == -INFINITY ? 0.f : exp2f(m2 - mx);
+  const float Lt = l1 * w1 + l2 * w2;
+  float A[CPL];
+#pragma unroll
+  for (int c = 0; c < CPL; ++c) A[c] = fmaf(A1[c], w1, A2[c] * w2) / Lt;
+  Vec<CPL>::st(out, A);
 }
 
 // threads: a producer warp, the consumer warps, the epilogue warp and the
@@ -209,13 +246,17 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
   __shared__ SegMeta seg[2];
   __shared__ StepTable tab;
   __shared__ long long scan_scratch[33];
-  __shared__ long long s_s0, s_mg_k0;
+  __shared__ long long s_s0, s_mg_k0, s_a, s_b;
   __shared__ int s_h0, s_h1, s_bad;
   __shared__ int s_mg_h, s_mg_j, s_mg_np;  // the split head this CTA combines
   __shared__ uint32_t s_ep;                // the launch's epoch
-  __shared__ uint64_t ep_bar, own_bar;     // merge warp -> epilogue, and back
-  __shared__ __align__(16) float own_acc[D];
-  __shared__ float own_ml[2];
+  // hand-overs between the epilogue and the merge warp: the epoch and the
+  // merge head (ep_bar), the other pieces combined (oth_bar), and this CTA's
+  // own piece or the news that the epilogue combined it already (own_bar)
+  __shared__ uint64_t ep_bar, oth_bar, own_bar;
+  __shared__ __align__(16) float own_acc[D], oth_acc[D];
+  __shared__ float own_ml[2], oth_ml[2];
+  __shared__ int s_own_state;  // 1: combined by the epilogue, 2: own piece handed over
   __shared__ volatile int s_abort;
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -241,7 +282,8 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
       mbar_init(&epi_free[s], 1);
     }
     mbar_init(&ep_bar, 32);
-    mbar_init(&own_bar, 1);
+    mbar_init(&oth_bar, 32);
+    mbar_init(&own_bar, 32);
     fence_barrier_init();
     s_abort = 0;
     s_bad = 0;
@@ -304,16 +346,19 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
   const long long slice_start = block_excl_scan<long long>(mine, scan_scratch, &total);
   if (tid == 0) STEP_TRACE(10);
   if (bad) atomicMax(&s_bad, bad);
+  Ranges<TT> rg;
+  rg.init(total, G, S::kMinChunk);
+  if (tid == 0) {  // this CTA's range (64-bit divisions: one thread)
+    s_a = rg.start(bx);
+    s_b = rg.start(bx + 1);
+  }
   __syncthreads();
   if (s_bad) {  // no CTA reads further or arrives: the step is not taken
     pdl_wait();
     if (bx == 0 && tid == 0) set_err(p.err, (uint32_t)s_bad);
     return;
   }
-  long long chunk = slot_len<TT>((total + G - 1) / G);
-  if (chunk < S::kMinChunk) chunk = S::kMinChunk;
-  const long long a = (long long)bx * chunk;
-  const long long b = a + chunk < total ? a + chunk : total;
+  const long long a = s_a, b = s_b;
   bool active = a < total;
   if (active && mine > 0) {  // the heads holding the range's first and last index
     const bool has_a = slice_start <= a && a < slice_start + mine;
@@ -634,10 +679,7 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
     hand_over(nullptr);  // nothing more
   } else if (warp == kCW + 1) {
     // ---- epilogue: combine each segment's row-group states ----------------
-    if (!mbar_wait(&ep_bar, 0u)) {  // the launch's epoch (merge warp)
-      s_abort = 1;
-      set_err(p.err, HKV_ERR_TIMEOUT);
-    }
+    bool have_ep = false;  // the epoch and the merge head (merge warp)
     int k = 0;
     for (;; ++k) {
       const int bb = k & 1;
@@ -672,18 +714,41 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&epi_free[bb]);  // the consumers may reuse the buffer
-      if (hs >= a && he <= b) {  // the whole head is in this CTA's range
+      const bool whole = hs >= a && he <= b;
+      if (!whole && !have_ep) {
+        if (!mbar_wait(&ep_bar, 0u)) {
+          s_abort = 1;
+          set_err(p.err, HKV_ERR_TIMEOUT);
+          break;
+        }
+        have_ep = true;
+      }
+      if (whole) {  // the whole head is in this CTA's range
 #pragma unroll
         for (int c = 0; c < CPL; ++c) A[c] /= L;
         V::st(p.out + (size_t)h * D + CPL * lane, A);
-      } else if (h == s_mg_h) {  // this CTA combines the head: to the merge warp
-        V::st(&own_acc[CPL * lane], A);
-        if (lane == 0) {
-          own_ml[0] = mx;
-          own_ml[1] = L;
+      } else if (h == s_mg_h) {  // this CTA combines the head
+        // the other pieces already combined by the merge warp: finish here;
+        // else hand this piece to the merge warp
+        int ready = mbar_test_wait(&oth_bar, 0u) ? 1 : 0;
+        ready = __shfl_sync(0xFFFFFFFFu, ready, 0);
+        if (ready) {
+          mbar_wait(&oth_bar, 0u);  // complete: every lane acquires oth_*
+          float A2[CPL];
+          V::lds(&oth_acc[CPL * lane], A2);
+          combine_store<CPL>(mx, L, A, oth_ml[0], oth_ml[1], A2,
+                             p.out + (size_t)h * D + CPL * lane);
+          STEP_TRACE_SET(18, globaltimer());
+        } else {
+          V::st(&own_acc[CPL * lane], A);
+          if (lane == 0) {
+            own_ml[0] = mx;
+            own_ml[1] = L;
+          }
         }
+        if (lane == 0) s_own_state = ready ? 1 : 2;
         __syncwarp();
-        if (lane == 0) mbar_arrive(&own_bar);
+        mbar_arrive(&own_bar);  // all 32 lanes
       } else {  // a piece for the combining CTA: epoch-tagged, no fence needed
         unsigned long long *ps = p.pslot + ((size_t)bx * 2 + (hs < a ? 1 : 0)) * (D + 2);
 #pragma unroll
@@ -698,13 +763,35 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
     STEP_TRACE_SET(9, k);
   } else {
     // ---- merge warp: barrier, appends, counters, the combined split head ---
+    // The split head this CTA combines, if any: the head of its range's
+    // first index when this CTA is that head's first middle CTA (its whole
+    // range inside the head) or, for a head in two pieces, holds its last
+    // row. Then the launch's epoch, unique per (layer, launch of that
+    // layer), from the generation of the layer's barrier word; the epilogue
+    // waits for both only when it meets a split head.
+    uint32_t gen0 = 0;
+    if (lane == 0) {
+      if (active && tab.start[0] < a) {
+        const long long hs0 = tab.start[0], he0 = hs0 + tab.vlen[0];
+        const long long k0 = rg.owner(hs0), k1 = rg.owner(he0 - 1);
+        const long long np = k1 - k0 + 1;
+        if ((np >= 3 ? k0 + 1 : k1) == bx) {
+          s_mg_k0 = k0;
+          s_mg_np = (int)np;
+          s_mg_j = (int)(bx - k0);
+          s_mg_h = h0;
+        }
+      }
+      gen0 = ld_acquire(p.bar + 1);
+      s_ep = (gen0 + 1u) * (uint32_t)p.n_layers + (uint32_t)(p.layer_base / nheads);
+    }
+    __syncwarp();
+    mbar_arrive(&ep_bar);  // all 32 lanes: the epilogue may read s_ep, s_mg_*
     // Arrive on the layer's barrier word: this CTA is done reading counters.
     // The last of the grid to arrive resets the count and bumps the
     // generation, which the others watch.
-    uint32_t gen0 = 0;
     int bar_done = 0;
     if (lane == 0) {
-      gen0 = ld_acquire(p.bar + 1);
       const uint32_t old = atomicAdd(p.bar, 1u);
       if (old == (uint32_t)G - 1) {
         p.bar[0] = 0;
@@ -714,28 +801,6 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
     }
     gen0 = __shfl_sync(0xFFFFFFFFu, gen0, 0);
     bar_done = __shfl_sync(0xFFFFFFFFu, bar_done, 0);
-    // the launch's epoch, unique per (layer, launch of that layer)
-    const uint32_t ep = (gen0 + 1u) * (uint32_t)p.n_layers + (uint32_t)(p.layer_base / nheads);
-    if (lane == 0) {
-      s_ep = ep;
-      // The split head this CTA combines, if any: the head of its range's
-      // first index when this CTA is that head's first middle CTA (its whole
-      // range inside the head) or, for a head in two pieces, holds its last
-      // row.
-      if (active && tab.start[0] < a) {
-        const long long hs0 = tab.start[0], he0 = hs0 + tab.vlen[0];
-        const long long k0 = hs0 / chunk, k1 = (he0 - 1) / chunk;
-        const long long np = k1 - k0 + 1;
-        if ((np >= 3 ? k0 + 1 : k1) == bx) {
-          s_mg_k0 = k0;
-          s_mg_np = (int)np;
-          s_mg_j = (int)(bx - k0);
-          s_mg_h = h0;
-        }
-      }
-    }
-    __syncwarp();
-    mbar_arrive(&ep_bar);  // all 32 lanes: the epilogue may read s_ep, s_mg_*
     const uint64_t t0 = globaltimer();
     auto timed_out = [&]() {
       if (globaltimer() - t0 <= kWaitTimeoutNs) return false;
@@ -757,35 +822,44 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
           tab.ntok[j] = p.ntok[p.layer_base + h0 + j];
       }
       __syncwarp();
-      constexpr int CH = RB / 16;                // 16-byte chunks of a row
-      constexpr int PER = (3 * CH + 31) / 32;    // chunks of the K, V, q rows per lane
-      for (int j = 0; j < n; ++j) {
-        const long long he = tab.start[j] + tab.vlen[j];
-        if (he <= a || he > b) continue;
-        const int h = h0 + j, i = p.layer_base + h;
-        const int ntj = tab.ntok[j];
-        const long long row = tab.off[j] + tab.vlen[j] - 1;
-        const unsigned char *src[3] = {static_cast<const unsigned char *>(p.k_new),
-                                       static_cast<const unsigned char *>(p.v_new),
-                                       static_cast<const unsigned char *>(p.q)};
-        unsigned char *dst[3] = {static_cast<unsigned char *>(p.K) + row * RB,
-                                 static_cast<unsigned char *>(p.V) + row * RB,
-                                 static_cast<unsigned char *>(p.qbuf) +
-                                     ((size_t)i * p.period + ntj % p.period) * RB};
-        uint4 x[PER];
+      // the K, V and q rows of every appended head as 16-byte chunks, a
+      // lane per chunk, every load of a round issued before its stores
+      constexpr int CH = RB / 16;  // chunks of a row
+      constexpr int NU = 8;        // chunks per lane and round
+      // The appended heads (a < he <= b) are the table's first napp entries:
+      // the first head's rows always reach past a, and only the last head
+      // can continue past b.
+      const int napp = tab.start[n - 1] + tab.vlen[n - 1] <= b ? n : n - 1;
+      constexpr int first_app = 0;
+      const int units = napp * 3 * CH;
+      for (int u0 = 0; u0 < units; u0 += 32 * NU) {
+        uint4 x[NU];
+        unsigned char *dst[NU];
 #pragma unroll
-        for (int u = 0; u < PER; ++u) {
-          const int c = lane + 32 * u;
-          if (c < 3 * CH)
-            x[u] = reinterpret_cast<const uint4 *>(src[c / CH] + (size_t)h * RB)[c % CH];
+        for (int v = 0; v < NU; ++v) {
+          const int u = u0 + v * 32 + lane;
+          dst[v] = nullptr;
+          if (u < units) {
+            const int jj = first_app + u / (3 * CH), w3 = (u / CH) % 3, cc = u % CH;
+            const int h = h0 + jj, i = p.layer_base + h;
+            const unsigned char *src = w3 == 0 ? static_cast<const unsigned char *>(p.k_new)
+                                     : w3 == 1 ? static_cast<const unsigned char *>(p.v_new)
+                                               : static_cast<const unsigned char *>(p.q);
+            x[v] = reinterpret_cast<const uint4 *>(src + (size_t)h * RB)[cc];
+            const long long row = tab.off[jj] + tab.vlen[jj] - 1;
+            unsigned char *d = w3 == 0 ? static_cast<unsigned char *>(p.K) + row * RB
+                             : w3 == 1 ? static_cast<unsigned char *>(p.V) + row * RB
+                                       : static_cast<unsigned char *>(p.qbuf) +
+                                             ((size_t)i * p.period + tab.ntok[jj] % p.period) * RB;
+            dst[v] = d + (size_t)cc * 16;
+          }
         }
 #pragma unroll
-        for (int u = 0; u < PER; ++u) {
-          const int c = lane + 32 * u;
-          if (c < 3 * CH) reinterpret_cast<uint4 *>(dst[c / CH])[c % CH] = x[u];
-        }
-        if (lane == 0) p.pos[row] = p.n_cond + ntj;
+        for (int v = 0; v < NU; ++v)
+          if (dst[v]) *reinterpret_cast<uint4 *>(dst[v]) = x[v];
       }
+      for (int jj = first_app + lane; jj < first_app + napp; jj += 32)
+        p.pos[tab.off[jj] + tab.vlen[jj] - 1] = p.n_cond + tab.ntok[jj];
     }
     STEP_TRACE_SET(8, globaltimer());
 
@@ -847,24 +921,26 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
         }
         if (ready || timed_out()) break;
       }
-      // this CTA's own piece
+      // hand the combined other pieces to the epilogue
+      V::st(&oth_acc[CPL * lane], oA);
+      if (lane == 0) {
+        oth_ml[0] = om;
+        oth_ml[1] = ol;
+      }
+      __syncwarp();
+      mbar_arrive(&oth_bar);  // all 32 lanes
+      // this CTA's own piece, unless the epilogue combined it already
       while (!s_abort && !mbar_try_wait(&own_bar, 0u))
         if (timed_out()) break;
       __syncwarp();
-      if (!s_abort) {
-        const float m1 = own_ml[0], l1 = own_ml[1];
+      if (!s_abort && s_own_state == 2) {
+        mbar_wait(&own_bar, 0u);  // complete: every lane acquires own_*
         float A1[CPL];
         V::lds(&own_acc[CPL * lane], A1);
-        const float mx = fmaxf(m1, om);
-        const float w1 = m1 == -INFINITY ? 0.f : exp2f(m1 - mx);
-        const float w2 = om == -INFINITY ? 0.f : exp2f(om - mx);
-        const float Lt = l1 * w1 + ol * w2;
-        float A[CPL];
-#pragma unroll
-        for (int c = 0; c < CPL; ++c) A[c] = fmaf(A1[c], w1, oA[c] * w2) / Lt;
-        V::st(p.out + (size_t)mh * D + CPL * lane, A);
+        combine_store<CPL>(own_ml[0], own_ml[1], A1, om, ol, oA,
+                           p.out + (size_t)mh * D + CPL * lane);
+        STEP_TRACE_SET(18, globaltimer());
       }
-      STEP_TRACE_SET(18, globaltimer());
     }
     if (lane == 0) STEP_TRACE(6);
   }
@@ -894,10 +970,14 @@ cudaError_t step_launch_t(const AttnArgs &a, int grid, cudaStream_t s) {
   cfg.dynamicSmemBytes = step_smem<D, T>();
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  int na = 0;
+  if (pdl) {
+    attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+  }
   cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
+  cfg.numAttrs = na;
   return cudaLaunchKernelEx(&cfg, step_kernel<D, T>, a);
 }
 

@@ -67,28 +67,41 @@ def test_reference_arm_prints_on_rank_zero_only():
 
 
 def test_profiled_traffic_follows_the_committed_capture(monkeypatch, tmp_path):
-    """The roofline's traffic comes from the committed ncu summary while the
-    attention source still has the sha256 recorded there, scaled by the
-    launch's algorithmic bytes; any other source or workload gives None."""
-    import hashlib
+    """The roofline's traffic comes from a committed ncu summary of the same
+    workload and decode-step design while the kernel sources still hash to
+    the digest recorded there, scaled by the launch's algorithmic bytes; any
+    other source, design or workload gives None."""
+    import glob
     sys.path.insert(0, ROOT)
     import bench
-    prof = os.path.join(ROOT, "profiles", "decode_step_lumina1024_rho4.md")
-    src = os.path.join(ROOT, "paper_2605_20600_gb300", "csrc", "hkv_attention.cu")
-    vals = dict(line.strip().partition(": ")[::2] for line in open(prof) if ": " in line)
-    same = hashlib.sha256(open(src, "rb").read()).hexdigest() == vals.get("source_sha256")
-    t = bench.profiled_traffic("lumina1024", 1e8)
-    if same:
-        exp = float(vals["attn_traffic_ratio"]) * 1e8 + float(vals["finish_traffic_bytes_per_launch"])
-        assert t == pytest.approx(exp)
-    else:
-        assert t is None
-    assert bench.profiled_traffic("llamagen_xl", 1e8) is None
-    # a copy of the tree whose attention source differs: no traffic
+    for launches in (1, 2):
+        digest = bench.sources_digest(launches)
+        caps = []
+        for path in glob.glob(os.path.join(ROOT, "profiles", "*.md")):
+            vals = dict(line.strip().partition(": ")[::2] for line in open(path) if ": " in line)
+            if vals.get("capture_of") == "lumina1024" and vals.get("launches") == str(launches):
+                caps.append(vals)
+        t = bench.profiled_traffic("lumina1024", 1e8, launches)
+        match = [v for v in caps if v.get("sources_sha256") == digest]
+        if match:
+            v = match[0]
+            assert t == pytest.approx(float(v["traffic_ratio"]) * 1e8
+                                      + float(v.get("extra_bytes_per_launch", "0")))
+        else:
+            assert t is None
+        assert bench.profiled_traffic("no_such_workload", 1e8, launches) is None
+    # a copy of the tree with a capture that matches, then a changed source
     (tmp_path / "profiles").mkdir()
-    (tmp_path / "profiles" / "decode_step_lumina1024_rho4.md").write_text(open(prof).read())
     d = tmp_path / "paper_2605_20600_gb300" / "csrc"
     d.mkdir(parents=True)
-    (d / "hkv_attention.cu").write_text(open(src).read() + "\n// changed\n")
+    for f in bench.STEP_SOURCES[1]:
+        (d / f).write_text(open(os.path.join(ROOT, "paper_2605_20600_gb300", "csrc", f)).read())
     monkeypatch.setattr(bench, "ROOT", str(tmp_path))
-    assert bench.profiled_traffic("lumina1024", 1e8) is None
+    (tmp_path / "profiles" / "cap.md").write_text(
+        f"capture_of: lumina1024\nlaunches: 1\nsources_sha256: {bench.sources_digest(1)}\n"
+        "traffic_ratio: 1.01\nextra_bytes_per_launch: 5\n")
+    assert bench.profiled_traffic("lumina1024", 1e8, 1) == pytest.approx(1.01e8 + 5)
+    assert bench.profiled_traffic("lumina1024", 1e8, 2) is None
+    (d / "hkv_step.cu").write_text(open(os.path.join(ROOT, "paper_2605_20600_gb300", "csrc",
+                                                     "hkv_step.cu")).read() + "\n// changed\n")
+    assert bench.profiled_traffic("lumina1024", 1e8, 1) is None
