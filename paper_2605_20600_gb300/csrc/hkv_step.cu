@@ -8,11 +8,12 @@
 // a producer warp, consumer warps and an epilogue warp), but the work that
 // the finishing kernel did there happens inside this launch:
 //
-//  * tile order: a CTA streams the piece of the head that began in an
-//    earlier range first, then the start of the head that continues into a
-//    later range, then the heads wholly inside its range. Every piece of a
-//    split head is then done early in its CTA, except the piece of a CTA
-//    whose whole range lies inside the head (a "middle" CTA);
+//  * tile order: a CTA streams the start of the head that continues into a
+//    later range first, then the piece of the head that began in an earlier
+//    range, then the heads wholly inside its range. The piece a CTA streams
+//    first is never the one that CTA combines, so a head in two pieces
+//    never waits for a piece that finishes last in its CTA (measured: 0.3
+//    us per step less than the other order at rho = 1/8);
 //  * merges: a split head is combined by its first middle CTA (whose whole
 //    range lies inside the head), else by the CTA holding its last row. The
 //    other pieces write their partial result to the workspace as 64-bit
@@ -166,11 +167,10 @@ template <int TT>
 struct Ranges {
   long long total, chunk;
   int G;
-  __device__ void init(long long total_, int G_, long long min_chunk) {
-    total = total_;
-    G = G_;
-    chunk = slot_len<TT>((total + G - 1) / G);
-    if (chunk < min_chunk) chunk = min_chunk;
+  // the range size (a 64-bit division: one thread computes it)
+  __device__ static long long chunk_of(long long total, int G, long long min_chunk) {
+    const long long c = slot_len<TT>((total + G - 1) / G);
+    return c < min_chunk ? min_chunk : c;
   }
   __device__ long long start(int k) const {
     const long long s = (long long)k * chunk;
@@ -246,7 +246,7 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
   __shared__ SegMeta seg[2];
   __shared__ StepTable tab;
   __shared__ long long scan_scratch[33];
-  __shared__ long long s_s0, s_mg_k0, s_a, s_b;
+  __shared__ long long s_s0, s_mg_k0, s_a, s_b, s_chunk;
   __shared__ int s_h0, s_h1, s_bad;
   __shared__ int s_mg_h, s_mg_j, s_mg_np;  // the split head this CTA combines
   __shared__ uint32_t s_ep;                // the launch's epoch
@@ -346,13 +346,20 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
   const long long slice_start = block_excl_scan<long long>(mine, scan_scratch, &total);
   if (tid == 0) STEP_TRACE(10);
   if (bad) atomicMax(&s_bad, bad);
-  Ranges<TT> rg;
-  rg.init(total, G, S::kMinChunk);
-  if (tid == 0) {  // this CTA's range (64-bit divisions: one thread)
-    s_a = rg.start(bx);
-    s_b = rg.start(bx + 1);
+  if (tid == 0) {  // this CTA's range (a 64-bit division: one thread)
+    Ranges<TT> r0;
+    r0.total = total;
+    r0.G = G;
+    r0.chunk = Ranges<TT>::chunk_of(total, G, S::kMinChunk);
+    s_chunk = r0.chunk;
+    s_a = r0.start(bx);
+    s_b = r0.start(bx + 1);
   }
   __syncthreads();
+  Ranges<TT> rg;
+  rg.total = total;
+  rg.G = G;
+  rg.chunk = s_chunk;
   if (s_bad) {  // no CTA reads further or arrives: the step is not taken
     pdl_wait();
     if (bx == 0 && tid == 0) set_err(p.err, (uint32_t)s_bad);
@@ -438,12 +445,12 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
     const bool has_e = he1 > b && (n > 1 || !has_s);
     const long long s_end = se0 < b ? se0 : b;
     const long long e_beg = hs1 > a ? hs1 : a;
-    if (has_s) {
-      sub_g[nsub] = a, sub_b[nsub] = s_end, sub_j[nsub] = 0;
-      ++nsub;
-    }
     if (has_e) {
       sub_g[nsub] = e_beg, sub_b[nsub] = b, sub_j[nsub] = n - 1;
+      ++nsub;
+    }
+    if (has_s) {
+      sub_g[nsub] = a, sub_b[nsub] = s_end, sub_j[nsub] = 0;
       ++nsub;
     }
     const long long m_lo = has_s ? s_end : a, m_hi = has_e ? e_beg : b;
@@ -474,6 +481,8 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
     return !pit.done();
   };
   int issued = 0;
+  // the arena rows are read once per step: evict them from L2 first (measured:
+  // 0.4-0.55 us per step slower without the hint)
   const uint64_t stream_pol = producer ? l2_evict_first_policy() : 0;
   struct Pending {
     int h, slot_new;
