@@ -312,7 +312,8 @@ hkv_status hkv_decode_attention(const hkv_config *cfg, const hkv_cache *cache, i
  * hkv_decode_attention; it allocates nothing.
  *  - The first call on a device, with that device current, looks up the
  *    array's device address and prepares the kernel; make that first call
- *    before any stream capture.
+ *    before any stream capture. The address is kept for the rest of the
+ *    process: do not reset the device (cudaDeviceReset) after that call.
  *  - Every call uses the same array; calls that may overlap on the GPU
  *    (other streams, other host threads) race on it and must be serialised
  *    by the caller. */

@@ -187,6 +187,19 @@ def label_margin(cum: np.ndarray, tau: float, w_loc: int) -> float:
     return abs(mass - tau)
 
 
+def count_margin(cum: np.ndarray, tau: float, n_h: int) -> float:
+    """Distance of the count n_h from its own threshold: n_h is the minimum n
+    with cum[n-1] >= tau, so it changes if cum[n_h-1] falls below tau or
+    cum[n_h-2] reaches it. Returns min(cum[n_h-1] - tau, tau - cum[n_h-2]),
+    over the terms that exist (the mass of zero tokens is 0), as absolute
+    values."""
+    terms = []
+    if 1 <= n_h <= cum.size:
+        terms.append(abs(float(cum[n_h - 1]) - tau))
+    terms.append(abs(tau - (float(cum[n_h - 2]) if n_h >= 2 else 0.0)))
+    return min(terms)
+
+
 # ----------------------------------------------------------------------------
 # Sec. 5.1: budgets
 # ----------------------------------------------------------------------------

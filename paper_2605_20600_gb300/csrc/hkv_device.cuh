@@ -10,7 +10,11 @@
 
 namespace hkv {
 
-constexpr uint64_t kWaitTimeoutNs = 2000000000ull;  // 2 s for any device wait
+// the limit of any device wait (a test build may shorten it)
+#ifndef HKV_WAIT_TIMEOUT_NS
+#define HKV_WAIT_TIMEOUT_NS 2000000000ull
+#endif
+constexpr uint64_t kWaitTimeoutNs = HKV_WAIT_TIMEOUT_NS;  // 2 s by default
 
 // ---------------------------------------------------------------------------
 // elements: a 16-byte piece holds 4 fp32 or 8 bf16 values

@@ -13,6 +13,9 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <stdlib.h>
+#include <string.h>
+
 #include <mutex>
 
 #include "hkv.h"
@@ -26,7 +29,10 @@ using namespace hkv;
 // head is split at each CTA boundary, then the control block the attention
 // kernel leaves for the finishing kernel: 1.06 MiB in total. The kernels write all of it
 // before reading it, so nothing in it has to start at zero.
-constexpr size_t kPartBytes = 1u << 20;
+#ifndef HKV_NOALLOC_PART_BYTES
+#define HKV_NOALLOC_PART_BYTES (1u << 20)
+#endif
+constexpr size_t kPartBytes = HKV_NOALLOC_PART_BYTES;
 constexpr size_t kRecBytes = (size_t)kAttnMaxGrid * sizeof(int4);
 constexpr size_t kScratchBytes = kPartBytes + kRecBytes + 256;
 
@@ -45,6 +51,17 @@ NoAllocDevice g_devs[kMaxDevices];
 std::mutex g_mu;
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// HKV_FAULT_INJECT=decode_attention_noalloc:<code> makes the call return
+// <code> before touching the GPU, like every other entry point
+hkv_status injected() {
+  const char *s = getenv("HKV_FAULT_INJECT");
+  static const char name[] = "decode_attention_noalloc";
+  if (!s) return HKV_OK;
+  const size_t n = sizeof(name) - 1;
+  if (strncmp(s, name, n) == 0 && s[n] == ':') return (hkv_status)atoi(s + n + 1);
+  return HKV_OK;
+}
 
 // Per-device set-up, done by the first call on each device with that device
 // current: the host-side name g_scratch is only a stand-in for the array, so
@@ -77,6 +94,8 @@ hkv_status setup(int D, int dtype, NoAllocDevice **out) {
 extern "C" hkv_status hkv_decode_attention_noalloc(const hkv_config *cfg, const hkv_cache *cache,
                                                    int layer, const void *q, float *out,
                                                    hkv_stream_t stream) {
+  const hkv_status inj = injected();
+  if (inj != HKV_OK) return inj;
   const hkv_status vs = hkv_validate_config(cfg);
   if (vs != HKV_OK) return vs;
   if (!cache || !cache->k || !cache->v || !cache->off || !cache->len || !cache->err || !q ||

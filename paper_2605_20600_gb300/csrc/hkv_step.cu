@@ -899,6 +899,13 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
     if (mh >= 0 && !s_abort) {
       const int np = s_mg_np, mj = s_mg_j;
       const long long k0 = s_mg_k0;
+#ifdef HKV_STEP_TEST_STALL
+      // test builds only: wait for an epoch no launch writes, so that the
+      // bounded wait runs out (HKV_ERR_TIMEOUT) with no bulk copy involved
+      const uint32_t want = s_ep + 1u;
+#else
+      const uint32_t want = s_ep;
+#endif
       float om = -INFINITY, ol = 0.f, oA[CPL];
 #pragma unroll
       for (int c = 0; c < CPL; ++c) oA[c] = 0.f;
@@ -915,9 +922,9 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
           float At[CPL], mt, lt;
           bool ok = true;
 #pragma unroll
-          for (int c = 0; c < CPL; ++c) ok &= ld_pair(ps + CPL * lane + c, s_ep, At[c]);
-          ok &= ld_pair(ps + D, s_ep, mt);
-          ok &= ld_pair(ps + D + 1, s_ep, lt);
+          for (int c = 0; c < CPL; ++c) ok &= ld_pair(ps + CPL * lane + c, want, At[c]);
+          ok &= ld_pair(ps + D, want, mt);
+          ok &= ld_pair(ps + D + 1, want, lt);
           ready = __all_sync(0xFFFFFFFFu, ok);
           if (!ready) break;
           const float mn = fmaxf(om, mt);
@@ -930,14 +937,17 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
         }
         if (ready || timed_out()) break;
       }
-      // hand the combined other pieces to the epilogue
-      V::st(&oth_acc[CPL * lane], oA);
-      if (lane == 0) {
-        oth_ml[0] = om;
-        oth_ml[1] = ol;
+      // hand the combined other pieces to the epilogue (not after a wait
+      // that ran out: the head's output is then not written)
+      if (!s_abort) {
+        V::st(&oth_acc[CPL * lane], oA);
+        if (lane == 0) {
+          oth_ml[0] = om;
+          oth_ml[1] = ol;
+        }
+        __syncwarp();
+        mbar_arrive(&oth_bar);  // all 32 lanes
       }
-      __syncwarp();
-      mbar_arrive(&oth_bar);  // all 32 lanes
       // this CTA's own piece, unless the epilogue combined it already
       while (!s_abort && !mbar_try_wait(&own_bar, 0u))
         if (timed_out()) break;

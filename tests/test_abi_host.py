@@ -279,3 +279,29 @@ def test_update_due_rejects_bad_arguments(H):
 
 def test_decode_step_launches_answers_zero_for_a_bad_config(H):
     assert H.lib().hkv_decode_step_launches(ctypes.byref(tiny_cfg(H, head_dim=32))) == 0
+
+
+def test_noalloc_host_checks_answer_before_the_device(H, monkeypatch):
+    """hkv_decode_attention_noalloc validates its arguments on the host (no
+    CUDA call: this runs without a GPU) and honours fault injection."""
+    f = H.lib().hkv_decode_attention_noalloc
+    f.argtypes = [ctypes.POINTER(H.hkv_config), ctypes.POINTER(H.hkv_cache), ctypes.c_int,
+                  ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]
+    f.restype = ctypes.c_int
+    cfg = tiny_cfg(H)
+    c = fake_cache(H)
+    q = out = c.k  # aligned, never dereferenced by the checks
+    assert f(ctypes.byref(tiny_cfg(H, head_dim=32)), ctypes.byref(c), 0, q, out, None) == 2
+    assert f(ctypes.byref(cfg), None, 0, q, out, None) == 1
+    for field in ("k", "v", "off", "len", "err"):
+        assert f(ctypes.byref(cfg), ctypes.byref(fake_cache(H, **{field: None})), 0, q, out,
+                 None) == 1, field
+    assert f(ctypes.byref(cfg), ctypes.byref(c), 0, None, out, None) == 1
+    assert f(ctypes.byref(cfg), ctypes.byref(c), 0, q, None, None) == 1
+    assert f(ctypes.byref(cfg), ctypes.byref(c), 0, q + 8, out, None) == 8
+    assert f(ctypes.byref(cfg), ctypes.byref(c), 0, q, out + 4, None) == 8
+    assert f(ctypes.byref(cfg), ctypes.byref(fake_cache(H, k=c.k + 8)), 0, q, out, None) == 8
+    assert f(ctypes.byref(cfg), ctypes.byref(c), 2, q, out, None) == 1   # n_layers = 2
+    assert f(ctypes.byref(cfg), ctypes.byref(c), -1, q, out, None) == 1
+    monkeypatch.setenv("HKV_FAULT_INJECT", "decode_attention_noalloc:6")
+    assert f(ctypes.byref(cfg), ctypes.byref(c), 0, q, out, None) == 6

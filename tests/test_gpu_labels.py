@@ -46,7 +46,7 @@ def test_multi_query_labels(name):
     ties = check_labels(w, labels, nh, lab, f"{name} multi")
     assert len(ties) <= 2, ties
     # every margin is far from tau here, so n_h was compared for every head
-    assert min(m for res in lab.values() for (_, _, m) in res) > 1e-3
+    assert min(m for res in lab.values() for (_, _, m, _) in res) > 1e-3
 
 
 @pytest.mark.parametrize("name", ["llamagen_xl", "lumina768"])

@@ -174,3 +174,21 @@ def test_grid_count_multi_with_one_query():
     a = O.grouping_count_2d(q, K, 0.9, 4, 6)
     b = O.grouping_count_multi_2d(q[None, :], K, 0.9, 4, 6)
     assert a[0] == b[0] and np.array_equal(a[1], b[1])
+
+
+def test_count_margin_hand_worked():
+    """The n_h decision's distance from tau: the two cumulative masses around
+    the cut (hand-worked)."""
+    cum = np.array([0.5, 0.85, 0.95, 1.0])
+    assert O.count_margin(cum, 0.9, 3) == pytest.approx(0.05)   # 0.95 - 0.9 vs 0.9 - 0.85
+    assert O.count_margin(cum, 0.88, 3) == pytest.approx(0.03)  # 0.88 - 0.85
+    assert O.count_margin(cum, 0.4, 1) == pytest.approx(0.1)    # cum[0] - tau; no token below
+    assert O.count_margin(cum, 0.02, 1) == pytest.approx(0.02)  # the empty prefix: tau - 0
+    # consistent with grouping_count on real weights: the cut sits where cum crosses tau
+    rng = np.random.default_rng(3)
+    for _ in range(20):
+        q, K = rng.normal(size=4), rng.normal(size=(30, 4)) * 3
+        n_h, cum = O.grouping_count(q, K, 0.9)
+        m = O.count_margin(cum, 0.9, n_h)
+        assert cum[n_h - 1] >= 0.9 and (n_h == 1 or cum[n_h - 2] < 0.9)
+        assert m == pytest.approx(min(cum[n_h - 1] - 0.9, 0.9 - (cum[n_h - 2] if n_h > 1 else 0)))
