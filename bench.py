@@ -570,26 +570,74 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
-def run_strategies(args):
-    """--strategies: decode attention over one steady-state cache (every
-    layer, right after the period's update) three ways, as the paper's
-    alternatives for heads of different lengths: the ragged split-K kernel of
-    this library (hkv_decode_attention), padding every head to the longest
-    capacity with a key mask, and one dense batch per head group (local,
-    global). The two baselines run PyTorch's scaled_dot_product_attention on
-    padded tensors built once (the cache as it would be stored in that
-    layout); the outputs of all three are cross-checked."""
-    import numpy as np
+def padded_gather(cache, o, l, width):
+    """K, V [..., width, D] and the key mask [..., width] of heads at arena
+    offsets o with live lengths l, as a padded layout would store them (rows
+    past a head's length repeat its row 0 and are masked)."""
     import torch
-    import torch.nn.functional as F
+    ar = torch.arange(width, device=o.device)
+    mask = ar < l[..., None]
+    idx = torch.where(mask, o[..., None] + ar, o[..., None])
+    return cache.k[idx], cache.v[idx], mask
 
+
+def strategy_padding(q, cache, off, ln, width, dtype):
+    """The paper's padding strategy for heads of different lengths: every head
+    padded to `width` keys and masked, one batched attention per layer
+    (PyTorch's scaled_dot_product_attention, computed in `dtype`).
+    q [L, n, D]; off, ln [L, n]. Returns a closure filling out [L, n, D] and
+    the padded tensors' bytes read per layer."""
+    import torch.nn.functional as F
+    L, n, D = q.shape
+    Kp, Vp, Mp = padded_gather(cache, off, ln, width)
+    Kp, Vp, qd = Kp.to(dtype), Vp.to(dtype), q.to(dtype)
+
+    def run(out):
+        for layer in range(L):
+            o = F.scaled_dot_product_attention(
+                qd[layer].reshape(1, n, 1, D), Kp[layer].reshape(1, n, width, D),
+                Vp[layer].reshape(1, n, width, D), attn_mask=Mp[layer].reshape(1, n, 1, width))
+            out[layer] = o.reshape(n, D)
+    return run, n * width * D * 2 * Kp.element_size()
+
+
+def strategy_per_group(q, cache, off, ln, cap, lab, dtype):
+    """The paper's per-group strategy: one dense batch per (layer, head
+    group: local, global), each padded to its group's capacity and masked
+    (scaled_dot_product_attention in `dtype`). Returns a closure filling
+    out [L, n, D] and the bytes read per layer."""
+    import torch.nn.functional as F
+    L, n, D = q.shape
+    batches = []
+    for layer in range(L):
+        for g in (0, 1):   # local, global
+            h = (lab[layer] == g).nonzero().flatten()
+            if len(h) == 0:
+                continue
+            width = int(cap[layer][h].max())
+            Kg, Vg, Mg = padded_gather(cache, off[layer][h], ln[layer][h], width)
+            batches.append((layer, h, q[layer][h].contiguous().to(dtype), Kg.to(dtype),
+                            Vg.to(dtype), Mg, width))
+
+    def run(out):
+        for layer, h, qg, Kg, Vg, Mg, width in batches:
+            m = len(h)
+            o = F.scaled_dot_product_attention(
+                qg.reshape(1, m, 1, D), Kg.reshape(1, m, width, D), Vg.reshape(1, m, width, D),
+                attn_mask=Mg.reshape(1, m, 1, width))
+            out[layer].index_copy_(0, h, o.reshape(m, D).to(out.dtype))
+    es = batches[0][3].element_size() if batches else 2
+    return run, sum(len(b[1]) * b[6] * D * 2 * es for b in batches) / L
+
+
+def strategies_setup(w, dev):
+    """A steady-state cache of workload w (every layer right after the
+    period's update) and the next step's queries."""
+    import torch
     from paper_2605_20600_gb300 import hkv as H
     from paper_2605_20600_gb300.engine import Engine, torch_dtype
     from paper_2605_20600_gb300.runner import generate
     from synth.gpu import DeviceSynth
-
-    dev = torch.device("cuda", 0)
-    w = workload(args)
     L, S, Hh, D, P = w.n_layers, w.n_seqs, w.n_heads, w.head_dim, w.period
     t0 = steady_start(w)
     cfg = H.make_config(n_layers=L, n_seqs=S, n_heads=Hh, head_dim=D, dtype=w.dtype,
@@ -604,28 +652,34 @@ def run_strategies(args):
         eng.evict(layer)
     torch.cuda.synchronize()
     eng.check()
-    dt = torch_dtype(cfg)
-    q = torch.empty(1, L, S, Hh, D, dtype=dt, device=dev)
+    q = torch.empty(1, L, S, Hh, D, dtype=torch_dtype(cfg), device=dev)
     kk, vv = torch.empty_like(q), torch.empty_like(q)
     synth.image(q, kk, vv, 0, L, t0, 1)
-    q = q[0]
-    c = eng.cache
     n = S * Hh
-    off = c.off.view(L, n).long()
-    ln = c.len.view(L, n).long()
-    cap = c.cap.view(L, n).long()
-    lab = eng.labels.view(L, n)
-    es = 2 if cfg.dtype == 1 else 4
-    lmax = int(cap.max())
+    c = eng.cache
+    return (eng, q[0].reshape(L, n, D), c.off.view(L, n).long(), c.len.view(L, n).long(),
+            c.cap.view(L, n).long(), eng.labels.view(L, n))
 
-    def padded(o, l, width):
-        """K, V [..., width, D] and mask [..., width] for heads at offsets o with
-        live lengths l (rows past the length repeat row 0 and are masked)."""
-        ar = torch.arange(width, device=dev)
-        mask = ar < l[..., None]
-        idx = torch.where(mask, o[..., None] + ar, o[..., None])
-        return c.k[idx], c.v[idx], mask
 
+def run_strategies(args):
+    """--strategies: decode attention over one steady-state cache (every
+    layer, right after the period's update) three ways, as the paper's
+    alternatives for heads of different lengths: the ragged split-K kernel of
+    this library (hkv_decode_attention), padding every head to the longest
+    capacity with a key mask, and one dense batch per head group (local,
+    global). The two baselines run PyTorch's scaled_dot_product_attention on
+    padded tensors built once (the cache as it would be stored in that
+    layout), in the cache's dtype; the outputs of all three are
+    cross-checked."""
+    import torch
+
+    dev = torch.device("cuda", 0)
+    w = workload(args)
+    L, D, P = w.n_layers, w.head_dim, w.period
+    eng, q, off, ln, cap, lab = strategies_setup(w, dev)
+    n = q.shape[1]
+    dt = q.dtype
+    es = q.element_size()
     reps = max(3, args.steps)
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
 
@@ -650,42 +704,13 @@ def run_strategies(args):
     eng.check()
     bytes_ours = float((ln.sum() * D * 2 * es).item()) / L
 
-    Kp, Vp, Mp = padded(off, ln, lmax)
     out_pad = torch.empty(L, n, D, dtype=dt, device=dev)
-
-    def pad():
-        for layer in range(L):
-            o = F.scaled_dot_product_attention(
-                q[layer].reshape(1, n, 1, D), Kp[layer].reshape(1, n, lmax, D),
-                Vp[layer].reshape(1, n, lmax, D), attn_mask=Mp[layer].reshape(1, n, 1, lmax))
-            out_pad[layer] = o.reshape(n, D)
-
-    us_pad = timed(pad)
-    bytes_pad = n * lmax * D * 2 * es
-    del Kp, Vp, Mp
-    # one dense batch per (layer, head group), each padded to its group's
-    # capacity, gathered before timing
-    batches = []
-    for layer in range(L):
-        for g in (0, 1):   # local, global
-            h = (lab[layer] == g).nonzero().flatten()
-            if len(h) == 0:
-                continue
-            width = int(cap[layer][h].max())
-            Kg, Vg, Mg = padded(off[layer][h], ln[layer][h], width)
-            batches.append((layer, h, q[layer].reshape(n, D)[h].contiguous(), Kg, Vg, Mg, width))
+    pad, bytes_pad = strategy_padding(q, eng.cache, off, ln, int(cap.max()), dt)
+    us_pad = timed(lambda: pad(out_pad))
+    del pad
     out_grp = torch.empty(L, n, D, dtype=dt, device=dev)
-
-    def grp():
-        for layer, h, qg, Kg, Vg, Mg, width in batches:
-            m = len(h)
-            o = F.scaled_dot_product_attention(
-                qg.reshape(1, m, 1, D), Kg.reshape(1, m, width, D), Vg.reshape(1, m, width, D),
-                attn_mask=Mg.reshape(1, m, 1, width))
-            out_grp[layer].index_copy_(0, h, o.reshape(m, D))
-
-    us_grp = timed(grp)
-    bytes_grp = sum(len(b[1]) * b[6] * D * 2 * es for b in batches) / L
+    grp, bytes_grp = strategy_per_group(q, eng.cache, off, ln, cap, lab, dt)
+    us_grp = timed(lambda: grp(out_grp))
     err_pad = float((out_pad.float() - out_ours).abs().max())
     err_grp = float((out_grp.float() - out_ours).abs().max())
     peak, peak_kind = load_peaks()
@@ -700,6 +725,113 @@ def run_strategies(args):
             "note": "baselines: torch.nn.functional.scaled_dot_product_attention on padded "
                     "tensors (library kernels); their padded tensors are built before timing"}
     print(json.dumps(line), flush=True)
+
+
+def run_phases(args):
+    """--phases: the one-off kernels of one generation, each timed per launch
+    with CUDA events and set against its algorithmic bytes: the conditioning
+    prefill (Step 1), the grouping token's decode step with the head types
+    decided in it (hkv_decode_step_identify), identification from the
+    current query and from the ring's recent queries (Step 2), the budgets
+    (Sec. 5.1) and the repack with its first update (Step 3). Layer 0 of
+    every phase (and the single budgets call) runs inside the NVTX range
+    "hkv_profiled", the profiler's target; the other layers outside it."""
+    import numpy as np
+    import torch
+
+    from paper_2605_20600_gb300 import hkv as H
+    from paper_2605_20600_gb300.engine import CacheBuffers, Engine, torch_dtype
+    from paper_2605_20600_gb300.runner import generate
+    from synth.gpu import DeviceSynth
+
+    dev = torch.device("cuda", 0)
+    w = workload(args)
+    L, S, Hh, D, C, E, P = (w.n_layers, w.n_seqs, w.n_heads, w.head_dim, w.n_cond, w.group_at,
+                            w.period)
+    cfg = H.make_config(n_layers=L, n_seqs=S, n_heads=Hh, head_dim=D, dtype=w.dtype,
+                        n_cond=C, n_image=w.n_image, row_len=w.row_len, recent_w=w.recent_w,
+                        local_w=w.w_loc, period=P, group_at=E, rho=w.rho, tau=w.tau, r_s=w.r_s)
+    es = 2 if cfg.dtype == 1 else 4
+    n = S * Hh
+    eng = Engine(cfg, dev)
+    synth = DeviceSynth(w, dev)
+    st = eng.stream()
+    res = {}
+
+    def timed(name, fn, calls, bytes_per_call):
+        """fn(i) for i in calls, the first inside "hkv_profiled"; us per call."""
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in calls]
+        torch.cuda.synchronize()
+        for j, (i, (e0, e1)) in enumerate(zip(calls, evs)):
+            if j == 0:
+                torch.cuda.nvtx.range_push("hkv_profiled")
+            e0.record()
+            fn(i)
+            e1.record()
+            if j == 0:
+                torch.cuda.nvtx.range_pop()
+        torch.cuda.synchronize()
+        us = statistics.mean(e0.elapsed_time(e1) * 1e3 for e0, e1 in evs)
+        res[name] = {"calls": len(calls), "us_per_call": us, "bytes_per_call": bytes_per_call,
+                     "GBps": bytes_per_call / us / 1e3}
+
+    # Step 1: conditioning K/V of every head written into the dense cache
+    # (read kc, vc; write K, V rows and positions)
+    # (on an engine of its own: the generation below prefills its layers)
+    if C > 0:
+        pre = Engine(cfg, dev)
+        kc = torch.empty(L, S, Hh, C, D, dtype=torch_dtype(cfg), device=dev)
+        vc = torch.empty_like(kc)
+        for l in range(L):
+            synth.cond(kc[l], vc[l], l, st)
+        timed("prefill", lambda l: pre.prefill(l, kc[l], vc[l]), range(L), n * C * (4 * D * es + 4))
+        pre.check()
+        del pre, kc, vc
+        torch.cuda.empty_cache()
+    generate(eng, synth, first_step=0, last_step=E - 2)    # the dense phase up to E - 2
+    q = torch.empty(L, S, Hh, D, dtype=torch_dtype(cfg), device=dev)
+    k, v = torch.empty_like(q), torch.empty_like(q)
+    synth.image(q, k, v, 0, L, E - 1, 1)
+    out = torch.empty(L, S, Hh, D, dtype=torch.float32, device=dev)
+    # the grouping token's step: a decode step over every head's C + E - 1
+    # dense rows (+ the new one), the head types decided in the same pass
+    step_bytes = n * (C + E - 1) * D * 2 * es + n * D * (6 * es + 4)
+    timed("grouping_step_identify",
+          lambda l: eng.step_identify(l, q[l], k[l], v[l], out[l]), range(L), step_bytes)
+    # Step 2 on the cache as it stands after that step (C + E rows): the keys
+    # once and the query; the multi-query variant also reads min(P, E)
+    # queries of the ring
+    timed("identify", lambda l: eng.identify(l, q[l]), range(L), n * (C + E + 1) * D * es)
+    pe = min(P, E)
+    timed("identify_multi", lambda l: eng.identify_multi(l), range(L), n * (C + E + pe) * D * es)
+    eng.check()
+    labels = eng.labels.clone()
+    # Sec. 5.1: labels in, budget, cap, off out (1 + 4 + 4 + 8 bytes a head)
+    nt = L * n
+    budget = torch.empty(nt, dtype=torch.int32, device=dev)
+    cap = torch.empty(nt, dtype=torch.int32, device=dev)
+    off = torch.empty(nt, dtype=torch.int64, device=dev)
+    total = [0]
+
+    def budgets(_):
+        total[0] = H.hkv_allocate_budgets(cfg, labels, budget, cap, off, st)
+    timed("budgets", budgets, [0], nt * 17)
+    rag = CacheBuffers(cfg, total[0], dev, qbuf=eng.dense.qbuf, label=labels, off=off, cap=cap)
+    timed("repack", lambda l: H.hkv_repack(cfg, eng.dense.c, rag.c, l, st), range(L), 0)
+    H.hkv_check(rag.c, st)
+    # repack: the kept rows read from the dense cache and written to the
+    # ragged one (K and V), the history keys of global heads read for the
+    # scores (E - w image tokens) and their P buffered queries
+    kept = rag.len.view(L, n).long().sum(1).double().mean().item()
+    glob = float((labels.view(L, n) == 1).sum(1).double().mean().item())
+    rb = kept * D * es * 4 + glob * (max(0, E - w.recent_w) + P) * D * es
+    res["repack"]["bytes_per_call"] = rb
+    res["repack"]["GBps"] = rb / res["repack"]["us_per_call"] / 1e3
+    peak, peak_kind = load_peaks()
+    print(json.dumps({"phases": describe(w, P), "heads_per_layer": n,
+                      "global_head_fraction": float((labels == 1).float().mean().item()),
+                      "results": res, "peak_GBps": peak, "peak_kind": peak_kind}), flush=True)
 
 
 def run_grouping(args):
@@ -905,9 +1037,15 @@ def main():
                          "stays the raster oracle)")
     ap.add_argument("--grouping", action="store_true",
                     help="time the grouping step with identification separate and fused")
+    ap.add_argument("--phases", action="store_true",
+                    help="time the one-off kernels of a generation (prefill, grouping, "
+                         "identification, budgets, repack)")
     ap.add_argument("--labels", action="store_true",
                     help="head-type shares and stability over tau and early/late grouping")
     args = ap.parse_args()
+    if args.phases:
+        run_phases(args)
+        return
     if args.labels:
         run_labels(args)
         return
