@@ -48,7 +48,8 @@
 //    that wait (HKV_ATTN_PRE_TILES of them: tiles in flight then delay the
 //    previous finishing kernel, whose few loads are on the critical path);
 //  * every wait on an mbarrier is bounded; one that runs out flags the
-//    error and lets the CTA finish its control flow without the data.
+//    error and lets the CTA finish its control flow without the data, the
+//    producer first waiting (bounded) for the bulk copies it armed.
 #include <math.h>
 #include <stdlib.h>
 
@@ -376,6 +377,7 @@ __global__ void __launch_bounds__(AttnShape<D, T>::kThreads, 2) attn_kernel(cons
 #pragma unroll
       for (int j = 0; j < NS; ++j)
         if (j < n_pre) issue_extra(pre[j], j);
+      int armed = n_pre;  // tiles whose stage the producer has arrived on
       while (!pit.done()) {
         const int stage = issued % NS;
         // the consumers are done with the tile that used this stage before
@@ -390,6 +392,7 @@ __global__ void __launch_bounds__(AttnShape<D, T>::kThreads, 2) attn_kernel(cons
         Pending pd;
         issue_old(pd);
         issue_extra(pd, stage);
+        armed = issued;
       }
       if (!s_abort) {  // no more tiles: a closing record for the consumers
         const int stage = issued % NS;
@@ -400,6 +403,13 @@ __global__ void __launch_bounds__(AttnShape<D, T>::kThreads, 2) attn_kernel(cons
           meta[stage].flags = kDone;
           mbar_arrive(&full[stage]);
         }
+      }
+      if (s_abort) {
+        // No bulk copy may land in shared memory after the CTA exits: wait
+        // (bounded) for every armed stage that may still be in flight; a
+        // stage reused after an empty-barrier wait is complete already.
+        const int first = armed - NS > 0 ? armed - NS : 0;
+        for (int t = first; t < armed; ++t) mbar_wait(&full[t % NS], (uint32_t)(t / NS) & 1u);
       }
       HKV_TRACE_ADD(13, t_wait);
     }
@@ -539,11 +549,6 @@ __global__ void __launch_bounds__(AttnShape<D, T>::kThreads, 2) attn_kernel(cons
     if (cw == 0 && lane == 0) seg.h = -1;
     __syncwarp();
     if (lane == 0) mbar_arrive(&epi_full);
-    if (s_abort && ctid == 0)  // drain what may still be in flight (bounded)
-      for (int s = 0; s < NS; ++s) {
-        mbar_wait(&full[s], 0);
-        mbar_wait(&full[s], 1);
-      }
   } else {
     // ---- epilogue: finish each head segment the consumers hand over --------
     // A lane owns CPL consecutive output channels, so each of its stores of
