@@ -198,7 +198,7 @@ hkv_status hkv_update_due(const hkv_config *cfg, int32_t t, int32_t *due_out);
 /* Bytes of device workspace hkv_decode_attention and hkv_decode_step need
  * for this config (split-K partial results, records of the heads split
  * between CTAs, a small control block, ready flags of the partial results
- * and two barrier words per layer). The workspace must be zero-filled before
+ * and four barrier words per layer). The workspace must be zero-filled before
  * its first use; every call leaves it ready for the next one (after a call
  * that reported an error, zero it again). Concurrent calls must not share a
  * workspace. Host only. */

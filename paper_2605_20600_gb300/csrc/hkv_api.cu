@@ -182,7 +182,7 @@ WsLayout ws_layout(const hkv_config *c) {
   w.ctl = w.rec + align256((size_t)kAttnMaxGrid * sizeof(int4));
   w.pslot = w.ctl + kCtlBytes;
   w.bar = w.pslot + align256((size_t)kAttnMaxGrid * 2 * (c->head_dim + 2) * 8);
-  w.total = w.bar + align256((size_t)c->n_layers * 2 * sizeof(uint32_t));
+  w.total = w.bar + align256((size_t)c->n_layers * 4 * sizeof(uint32_t));
   return w;
 }
 
@@ -208,7 +208,7 @@ AttnArgs attn_args(const hkv_config *cfg, const hkv_cache *cache, int layer, con
   a.rec = reinterpret_cast<int4 *>(ws + w.rec);
   a.ctl = reinterpret_cast<AttnCtl *>(ws + w.ctl);
   a.pslot = reinterpret_cast<unsigned long long *>(ws + w.pslot);
-  a.bar = reinterpret_cast<uint32_t *>(ws + w.bar) + (size_t)layer * 2;
+  a.bar = reinterpret_cast<uint32_t *>(ws + w.bar) + (size_t)layer * 4;
   a.n_layers = cfg->n_layers;
   a.err = cache->err;
   a.pos = cache->pos;
@@ -273,21 +273,17 @@ hkv_status attn_grid(const hkv_config *cfg, int *grid) {
 // kernel's head table: a range of c tiles holds at most c + 1 heads (a head
 // has at least one tile in a step, its new token), and c is at most the
 // layer's tile count over the grid, bounded by every head at the longest
-// segment the config allows. Measured on GB300 (each shape A/B in one
-// process): one launch is faster while a layer has at most one head per CTA
-// (Lumina-mGPT-1024: 256 heads on 304 CTAs, 2-3 % per step), the two-kernel
-// design from about two heads per CTA on (Lumina-mGPT-768, Janus-Pro-7B,
-// LlamaGen-XL: 1-3 %). HKV_STEP_TWO_KERNELS / HKV_STEP_ONE_LAUNCH in the
-// environment force either design (tests of both).
+// segment the config allows. Where it fits, one launch is the faster design
+// on every model shape measured (each shape A/B in one process on GB300).
+// HKV_STEP_TWO_KERNELS in the environment forces the two-kernel design
+// (tests of both).
 bool one_launch_step(const hkv_config *cfg, int grid) {
   if (getenv("HKV_STEP_TWO_KERNELS")) return false;
   const long long tt = step_tile_rows(cfg->head_dim, cfg->dtype);
   const long long tiles = (long long)heads_per_layer(cfg) * ((max_segment(cfg) + tt - 1) / tt);
   long long chunk = (tiles + grid - 1) / grid;
   if (chunk < 2) chunk = 2;
-  if (chunk + 1 > kStepTable) return false;
-  if (getenv("HKV_STEP_ONE_LAUNCH")) return true;
-  return heads_per_layer(cfg) <= grid;
+  return chunk + 1 <= kStepTable;
 }
 
 #define HKV_TRY(x)                 \

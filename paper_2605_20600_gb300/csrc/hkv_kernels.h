@@ -57,8 +57,9 @@ struct AttnArgs {
   uint8_t *label_out;         // [L*S*H]
   int w_loc;
   float tau;
-  // one-launch step (hkv_step.cu): the layer's barrier word pair {arrivals,
-  // generation}, zero between launches; the partial results of split heads
+  // one-launch step (hkv_step.cu): the layer's barrier words {arrivals,
+  // generation, worst status of a bad step, unused}, the arrivals and the
+  // status zero between launches; the partial results of split heads
   // as (value, launch epoch) pairs, two slots per CTA (the piece at the end
   // of its range, the piece at its start), [grid][2][D + 2]
   uint32_t *bar;

@@ -22,14 +22,18 @@
 //    every pair carries this launch's epoch, while its consumers stream.
 //    Pieces are combined in index order and the CTA's own piece last, so the
 //    result does not depend on timing;
-//  * appends and counters: the merge warp copies the new token of every head
-//    whose last row is in the CTA's range into the cache as soon as the
-//    step's inputs are visible (nothing in the launch reads those rows).
-//    Every CTA reads the layer's lengths in its prologue and arrives on a
-//    per-layer barrier word when it is done reading them; the merge warp
-//    advances len, ntok and nbuf of its heads once the whole grid has
-//    arrived. The next launch of the same layer starts after this one
-//    completes, so the barrier word is free again by then;
+//  * prologue: every CTA loads the lengths of all the layer's heads
+//    (coalesced, into shared memory) to place the ranges, but reads and
+//    checks the other counters only for the heads of its own range;
+//  * appends and counters: every CTA arrives on a per-layer barrier word
+//    once it is done reading the layer's counters (a CTA that found a bad
+//    head marks its arrival); once the whole grid has arrived, and unless
+//    one was marked, the merge warp copies the new token of every head
+//    whose last row is in the CTA's range into the cache (nothing in the
+//    launch reads those rows) and advances len, ntok and nbuf of those
+//    heads, while the consumers stream. The next launch of the same layer
+//    starts after this one completes, so the barrier word is free again by
+//    then;
 //  * programmatic dependent launch: with the prefetch flag the prologue and
 //    the first tiles of old K/V rows go ahead of the wait for the previous
 //    kernel; the step's inputs (q, the new k and v) are read after it;
@@ -60,7 +64,9 @@ __device__ unsigned long long *g_step_trace = nullptr;  // [layer][kAttnMaxGrid]
   do {                                          \
     if (g_step_trace) STEP_TRACE_AT(slot) = (v); \
   } while (0)
+#define STEP_CLK() clock64()
 #else
+#define STEP_CLK() 0ll
 #define STEP_TRACE(slot) \
   do {                   \
   } while (0)
@@ -71,10 +77,10 @@ __device__ unsigned long long *g_step_trace = nullptr;  // [layer][kAttnMaxGrid]
 #endif
 
 // Tuning knobs (compile time) of the one-launch step, per head dimension:
-// consumer warps, bytes of K per stage, stages, tiles loaded before the wait;
-// CTAs per SM in the grid (kStepActivePerSm) and CTAs per SM the kernel is
-// built to be resident with (kStepResidentPerSm: with one more than the
-// grid uses, the next layer's CTAs can start while this layer streams).
+// consumer warps, bytes of K per stage, stages, tiles loaded before the wait
+// (measured at both head dimensions: 3 stages with 2 loaded before the wait
+// beat 2, 4 and 5 stages), and the CTAs per SM the kernel is built to be
+// resident with (the grid uses kStepActivePerSm).
 #ifndef HKV_STEP_CW_D128
 #define HKV_STEP_CW_D128 HKV_ATTN_CW_D128
 #endif
@@ -94,17 +100,13 @@ __device__ unsigned long long *g_step_trace = nullptr;  // [layer][kAttnMaxGrid]
 #define HKV_STEP_TILE_BYTES_D64 HKV_ATTN_TILE_BYTES_D64
 #endif
 #ifndef HKV_STEP_STAGES_D64
-#define HKV_STEP_STAGES_D64 HKV_ATTN_STAGES_D64
+#define HKV_STEP_STAGES_D64 3
 #endif
 #ifndef HKV_STEP_PRE_D64
-#define HKV_STEP_PRE_D64 HKV_ATTN_PRE_TILES
+#define HKV_STEP_PRE_D64 2
 #endif
 #ifndef HKV_STEP_RESIDENT_PER_SM
 #define HKV_STEP_RESIDENT_PER_SM 2
-#endif
-// heads of a thread's prologue slice kept in registers (more: reloaded)
-#ifndef HKV_STEP_SLICE_REGS
-#define HKV_STEP_SLICE_REGS 1
 #endif
 
 template <int D, typename T>
@@ -235,6 +237,7 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
   constexpr int NST = kCW * RPW;  // row-group states per segment
   constexpr int CPL = D / 32;     // output channels per epilogue lane
   static_assert(NST <= 32, "a lane of the epilogue per state");
+  static_assert(kStepTable <= kThr, "a thread per table entry");
   using V = Vec<CPL>;
 
   extern __shared__ __align__(128) unsigned char stages[];
@@ -295,57 +298,60 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
   if (!p.prefetch) pdl_wait();
 
   // ---- prologue: the layer's lengths, one round of loads -------------------
-  // Every thread takes a contiguous slice of the layer's heads and checks
-  // them (all loads of a head issued before any check); a block scan gives
-  // each slice its first index. Every CTA checks every head, so all CTAs take
-  // the same decision.
+  // Every thread takes a contiguous slice of the layer's heads and sums
+  // their slots; a block scan gives each slice its first index, so every
+  // CTA computes the same ranges, and a negative length stops every CTA.
+  // Offsets, capacities, labels and buffer counts are checked only for the
+  // heads of the CTA's own range: a CTA that finds a bad one streams nothing
+  // and flags the step on the layer's barrier word, and no CTA then appends
+  // or advances a counter. All of it takes one round of loads: a slice of
+  // one head is read whole into registers; with longer slices only the
+  // lengths are, and the same round reads the other counters of a window of
+  // kThr heads around the range's expected place (heads of equal length). A
+  // range outside the window reads them once it is known.
   const int per = (nheads + kThr - 1) / kThr;
   const int h_lo = tid * per < nheads ? tid * per : nheads;
   const int h_hi = h_lo + per < nheads ? h_lo + per : nheads;
+  const bool in_regs = per <= 1;
   long long mine = 0;
   int bad = 0;
-  auto check = [&](int l, long long o, int cp, int lab, int nb) {
-    if (l < 0 || o < 0 || o + cp > p.arena_tokens) bad = HKV_ERR_BOUNDS;
-    else if (l + 1 > cp) bad = bad ? bad : HKV_ERR_CAPACITY;
-    else if (lab != HKV_DENSE && nb >= p.period)
-      bad = bad ? bad : HKV_ERR_STATE;  // the periodic update is due first
+  auto count = [&](int l) {
+    if (l < 0) bad = HKV_ERR_BOUNDS;
     mine += slot_len<TT>(l + 1);
   };
-  // A slice of up to KR heads stays in registers for the whole prologue (one
-  // round of loads); a longer one is read again where needed.
-  constexpr int KR = HKV_STEP_SLICE_REGS;
-  const bool in_regs = per <= KR;
-  int rl[KR], rnb[KR];
-  long long ro[KR];
-  unsigned char rlb[KR];
+  // the counters of one head in registers: this thread's slice (in_regs) or
+  // its head of the window
+  int rl = 0, rcp = 0, rnb = 0, rlb = 0;
+  long long ro = 0;
+  int win_lo = 0;
   if (in_regs) {
-    int rcp[KR];
-#pragma unroll
-    for (int u = 0; u < KR; ++u) {  // every load issued before any use
-      const int h = h_lo + u;
-      rl[u] = rnb[u] = rcp[u] = 0;
-      ro[u] = 0;
-      rlb[u] = 0;
-      if (h < h_hi) {
-        rl[u] = p.len[h];
-        ro[u] = p.off[h];
-        rcp[u] = p.cap[h];
-        rlb[u] = p.label[p.layer_base + h];
-        rnb[u] = p.nbuf[p.layer_base + h];
-      }
+    if (h_lo < h_hi) {  // every load issued before any use
+      rl = p.len[h_lo];
+      ro = p.off[h_lo];
+      rcp = p.cap[h_lo];
+      rlb = p.label[p.layer_base + h_lo];
+      rnb = p.nbuf[p.layer_base + h_lo];
+      count(rl);
     }
-#pragma unroll
-    for (int u = 0; u < KR; ++u)
-      if (h_lo + u < h_hi) check(rl[u], ro[u], rcp[u], rlb[u], rnb[u]);
   } else {
+    const int guess = (int)((float)bx * ((float)nheads / (float)G));
+    win_lo = guess - kThr / 2;
+    win_lo = win_lo < nheads - kThr ? win_lo : nheads - kThr;
+    win_lo = win_lo > 0 ? win_lo : 0;
+    const int wh = win_lo + tid;
+    if (wh < nheads) {
+      ro = p.off[wh];
+      rcp = p.cap[wh];
+      rlb = p.label[p.layer_base + wh];
+      rnb = p.nbuf[p.layer_base + wh];
+    }
 #pragma unroll 4
-    for (int h = h_lo; h < h_hi; ++h)
-      check(p.len[h], p.off[h], p.cap[h], p.label[p.layer_base + h], p.nbuf[p.layer_base + h]);
+    for (int h = h_lo; h < h_hi; ++h) count(p.len[h]);
   }
   long long total;
   const long long slice_start = block_excl_scan<long long>(mine, scan_scratch, &total);
   if (tid == 0) STEP_TRACE(10);
-  if (bad) atomicMax(&s_bad, bad);
+  if (bad) s_bad = bad;
   if (tid == 0) {  // this CTA's range (a 64-bit division: one thread)
     Ranges<TT> r0;
     r0.total = total;
@@ -360,7 +366,7 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
   rg.total = total;
   rg.G = G;
   rg.chunk = s_chunk;
-  if (s_bad) {  // no CTA reads further or arrives: the step is not taken
+  if (s_bad) {  // every CTA sees it: none reads further or arrives
     pdl_wait();
     if (bx == 0 && tid == 0) set_err(p.err, (uint32_t)s_bad);
     return;
@@ -382,9 +388,7 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
         st += L;
       };
       if (in_regs) {
-#pragma unroll
-        for (int u = 0; u < KR; ++u)
-          if (h_lo + u < h_hi) visit(h_lo + u, rl[u]);
+        visit(h_lo, rl);
       } else {
         for (int h = h_lo; h < h_hi; ++h) visit(h, p.len[h]);
       }
@@ -393,33 +397,55 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
   __syncthreads();
   if (tid == 0) STEP_TRACE(11);
   int n = active ? s_h1 - s_h0 + 1 : 0;
-  if (n > kStepTable) {  // excluded by the host; reported, range skipped
-    if (tid == 0) set_err(p.err, HKV_ERR_CAPACITY);
+  int own_bad = 0;
+  if (n > kStepTable) {  // excluded by the host; the step is not taken
+    own_bad = HKV_ERR_CAPACITY;
     n = 0;
     active = false;
   }
   const int h0 = s_h0;
-  // the table: every thread fills the entries of its slice
-  if (active && h_lo <= h0 + n - 1 && h_hi > h0) {
-    long long st = slice_start;
-    auto fill = [&](int h, int l, long long o, int nb, int lab) {
-      if (h >= h0 && h < h0 + n) {
-        const int j = h - h0;
-        tab.start[j] = st;
-        tab.off[j] = o;
-        tab.vlen[j] = l + 1;
-        tab.nbuf[j] = nb;
-        tab.label[j] = (unsigned char)lab;
+  // the table entry of head h with its checks
+  auto enter = [&](int h, long long st, int l, long long o, int cp, int lab, int nb) {
+    const int j = h - h0;
+    int e = 0;
+    if (o < 0 || o + cp > p.arena_tokens) e = HKV_ERR_BOUNDS;
+    else if (l + 1 > cp) e = HKV_ERR_CAPACITY;
+    else if (lab != HKV_DENSE && nb >= p.period) e = HKV_ERR_STATE;  // the update is due first
+    if (e) atomicMax(&s_bad, e);
+    if (st >= 0) {
+      tab.start[j] = st;
+      tab.vlen[j] = l + 1;
+    }
+    tab.off[j] = o;
+    tab.nbuf[j] = nb;
+    tab.label[j] = (unsigned char)lab;
+  };
+  if (in_regs) {  // the slice owner enters its head
+    if (active && h_lo < h_hi && h_lo >= h0 && h_lo < h0 + n)
+      enter(h_lo, slice_start, rl, ro, rcp, rlb, rnb);
+  } else {
+    // the slice owners place the range's heads in the index space ...
+    if (active && h_lo <= h0 + n - 1 && h_hi > h0) {
+      long long st = slice_start;
+      for (int h = h_lo; h < h_hi && h < h0 + n; ++h) {
+        const int l = p.len[h];
+        if (h >= h0) {
+          tab.start[h - h0] = st;
+          tab.vlen[h - h0] = l + 1;
+        }
+        st += slot_len<TT>(l + 1);
       }
-      st += slot_len<TT>(l + 1);
-    };
-    if (in_regs) {
-#pragma unroll
-      for (int u = 0; u < KR; ++u)
-        if (h_lo + u < h_hi) fill(h_lo + u, rl[u], ro[u], rnb[u], rlb[u]);
-    } else {
-      for (int h = h_lo; h < h_hi; ++h)
-        fill(h, p.len[h], p.off[h], p.nbuf[p.layer_base + h], p.label[p.layer_base + h]);
+    }
+    // ... and a thread per head checks the rest: from registers when the
+    // window holds the whole range, else from one more round of loads
+    const bool in_win = h0 >= win_lo && h0 + n <= win_lo + kThr;
+    const int jt = in_win ? win_lo + tid - h0 : tid;
+    if (active && jt >= 0 && jt < n) {
+      const int h = h0 + jt, i = p.layer_base + h;
+      if (in_win)
+        enter(h, -1, p.len[h], ro, rcp, rlb, rnb);
+      else
+        enter(h, -1, p.len[h], p.off[h], p.cap[h], p.label[i], p.nbuf[i]);
     }
   }
   if (tid == 0) {
@@ -427,8 +453,12 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
     tab.n = n;
   }
   __syncthreads();
+  if (s_bad) {  // a bad head in this range: stream nothing
+    own_bad = own_bad > s_bad ? own_bad : s_bad;
+    active = false;
+  }
   // From here on nothing reads the layer's counters in global memory: the
-  // epilogue warp arrives on the layer's barrier word below.
+  // merge warp arrives on the layer's barrier word below.
   if (tid == 0) STEP_TRACE(1);
 
   // ---- the range's sub-ranges, in streaming order --------------------------
@@ -459,6 +489,8 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
       ++nsub;
     }
   }
+
+  if (tid == 0) STEP_TRACE(12);
 
   // ---- producer state (warp 0, lane 0) ------------------------------------
   const bool producer = tid == 0;
@@ -537,6 +569,7 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
   int n_pre = 0;
   if (producer)
     for (; n_pre < (p.prefetch ? S::kPre : NS) && more(); ++n_pre) issue_old(pre[n_pre]);
+  if (tid == 0) STEP_TRACE(7);
 
   if (p.prefetch) pdl_wait();  // the step's inputs are visible from here on
   if (tid == 0) STEP_TRACE(2);
@@ -545,6 +578,7 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
   if (warp == 0) {
     // ---- producer ----------------------------------------------------------
     if (producer) {
+      long long w_empty = 0;  // cycles waiting for free stages (tracer)
       int armed = 0;  // stages whose producer arrival is done (issued order)
 #pragma unroll
       for (int j = 0; j < NS; ++j)
@@ -552,12 +586,14 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
       armed = n_pre;
       while (more()) {
         const int stage = issued % NS;
+        const long long c0 = STEP_CLK();
         if (s_abort ||
             (issued >= NS && !mbar_wait(&empty[stage], (uint32_t)(issued / NS - 1) & 1u))) {
           s_abort = 1;
           set_err(p.err, HKV_ERR_TIMEOUT);
           break;
         }
+        w_empty += STEP_CLK() - c0;
         Pending pd;
         issue_old(pd);
         issue_extra(pd, stage);
@@ -573,6 +609,7 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
           mbar_arrive(&full[stage]);
         }
       }
+      STEP_TRACE_SET(20, w_empty);
       if (s_abort) {
         // No bulk copy may land in shared memory after the CTA exits: wait
         // (bounded) for every armed stage that may still be in flight. A
@@ -594,14 +631,17 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
 #pragma unroll
     for (int e = 0; e < EPL / 2; ++e) acc[e] = make_float2(0.f, 0.f);
     int n_tiles = 0;
+    long long w_full = 0, w_hand = 0;  // cycles waiting for tiles, for the epilogue (tracer)
     // hands one segment's state (or the closing record) to the epilogue
     auto hand_over = [&](const SegMeta *sm) {
       const int bb = nseg & 1;
+      const long long c0 = STEP_CLK();
       if (nseg >= 2 && !s_abort &&
           !mbar_wait(&epi_free[bb], (uint32_t)((nseg >> 1) - 1) & 1u)) {
         s_abort = 1;
         set_err(p.err, HKV_ERR_TIMEOUT);
       }
+      w_hand += STEP_CLK() - c0;
       if (sm) {
         const int si = cw * RPW + grp;
         float2 *dst = reinterpret_cast<float2 *>(&red_acc[bb][si][col * EPL]);
@@ -621,10 +661,12 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
     };
     for (int tile = 0;; ++tile) {
       const int stage = tile % NS;
+      const long long c0 = STEP_CLK();
       if (!s_abort && !mbar_wait(&full[stage], (uint32_t)(tile / NS) & 1u)) {
         s_abort = 1;
         set_err(p.err, HKV_ERR_TIMEOUT);
       }
+      if (tile > 0) w_full += STEP_CLK() - c0;
       if (s_abort) break;
       const int flags = meta[stage].flags;
       if (flags & kDone) break;
@@ -686,16 +728,21 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
     if (ctid == 0) STEP_TRACE(4);
     if (ctid == 0) STEP_TRACE_SET(17, n_tiles);
     hand_over(nullptr);  // nothing more
+    if (ctid == 0) STEP_TRACE_SET(21, w_full);
+    if (ctid == 0) STEP_TRACE_SET(22, w_hand);
   } else if (warp == kCW + 1) {
     // ---- epilogue: combine each segment's row-group states ----------------
     bool have_ep = false;  // the epoch and the merge head (merge warp)
+    long long w_epi = 0;   // cycles waiting for segments (tracer)
     int k = 0;
     for (;; ++k) {
       const int bb = k & 1;
+      const long long c0 = STEP_CLK();
       if (!s_abort && !mbar_wait(&epi_full[bb], (uint32_t)(k >> 1) & 1u)) {
         s_abort = 1;
         set_err(p.err, HKV_ERR_TIMEOUT);
       }
+      if (k > 0) w_epi += STEP_CLK() - c0;
       if (s_abort) break;
       const SegMeta sg = seg[bb];
       if (sg.h < 0) break;
@@ -770,6 +817,7 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
     }
     if (lane == 0) STEP_TRACE(5);
     STEP_TRACE_SET(9, k);
+    if (lane == 0) STEP_TRACE_SET(23, w_epi);
   } else {
     // ---- merge warp: barrier, appends, counters, the combined split head ---
     // The split head this CTA combines, if any: the head of its range's
@@ -778,6 +826,7 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
     // row. Then the launch's epoch, unique per (layer, launch of that
     // layer), from the generation of the layer's barrier word; the epilogue
     // waits for both only when it meets a split head.
+    constexpr uint32_t kBadStep = 0x80000000u;  // in the generation: step not taken
     uint32_t gen0 = 0;
     if (lane == 0) {
       if (active && tab.start[0] < a) {
@@ -792,19 +841,35 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
         }
       }
       gen0 = ld_acquire(p.bar + 1);
-      s_ep = (gen0 + 1u) * (uint32_t)p.n_layers + (uint32_t)(p.layer_base / nheads);
+      s_ep = ((gen0 & ~kBadStep) + 1u) * (uint32_t)p.n_layers + (uint32_t)(p.layer_base / nheads);
     }
     __syncwarp();
     mbar_arrive(&ep_bar);  // all 32 lanes: the epilogue may read s_ep, s_mg_*
-    // Arrive on the layer's barrier word: this CTA is done reading counters.
-    // The last of the grid to arrive resets the count and bumps the
-    // generation, which the others watch.
+    // Arrive on the layer's barrier words {arrivals, generation, worst
+    // status}: this CTA is done reading counters. The last of the grid to
+    // arrive resets the count and publishes the next generation, which the
+    // others watch. A CTA with a bad head raises the worst status and adds
+    // 1 << 16 more; the last arriver then marks the generation (the step is
+    // not taken) and reports the worst status, the same whichever CTAs found
+    // bad heads first.
+    const uint32_t inc = own_bad ? 0x10001u : 1u;
+    uint32_t gen1 = 0;
     int bar_done = 0;
     if (lane == 0) {
-      const uint32_t old = atomicAdd(p.bar, 1u);
-      if (old == (uint32_t)G - 1) {
+      if (own_bad) {
+        atomicMax(p.bar + 2, (uint32_t)own_bad);
+        __threadfence();  // the status before the arrival
+      }
+      const uint32_t old = atomicAdd(p.bar, inc);
+      if ((old & 0xFFFFu) == (uint32_t)G - 1) {
+        const bool bad_step = ((old + inc) >> 16) != 0;
+        if (bad_step) {
+          __threadfence();  // the bad CTAs' statuses after their arrivals
+          set_err(p.err, atomicExch(p.bar + 2, 0u));
+        }
         p.bar[0] = 0;
-        st_release(p.bar + 1, gen0 + 1);
+        gen1 = (((gen0 & ~kBadStep) + 1u) & ~kBadStep) | (bad_step ? kBadStep : 0u);
+        st_release(p.bar + 1, gen1);
         bar_done = 1;
       }
     }
@@ -819,12 +884,38 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
       }
       return true;
     };
+    if (own_bad) {
+      // empty pieces in both of this CTA's slots, so that no combining CTA
+      // waits for them (the step is not taken; the outputs are not defined)
+      for (int sl = 0; sl < 2; ++sl) {
+        unsigned long long *ps = p.pslot + ((size_t)bx * 2 + sl) * (D + 2);
+        for (int c = lane; c < D; c += 32) st_pair(ps + c, 0.f, s_ep);
+        if (lane == 0) {
+          st_pair(ps + D, -INFINITY, s_ep);
+          st_pair(ps + D + 1, 0.f, s_ep);
+        }
+      }
+    }
+
+    while (!s_abort && !bar_done) {
+      if (lane == 0) {
+        gen1 = ld_acquire(p.bar + 1);
+        bar_done = gen1 != gen0;
+      }
+      bar_done = __shfl_sync(0xFFFFFFFFu, bar_done, 0);
+      if (!bar_done && timed_out()) break;
+    }
+    gen1 = __shfl_sync(0xFFFFFFFFu, gen1, 0);
+    __syncwarp();
+    STEP_TRACE_SET(19, globaltimer());
+    const bool taken = !s_abort && bar_done && !(gen1 & kBadStep) && active;
 
     // Appends: the CTA holding a head's last row writes the new token (K/V
     // row at index len, its position, q into the ring of the periodic
-    // update). Nothing in this launch reads them, so they go first, while
-    // the consumers stream. The inputs are visible (after the wait above).
-    if (active) {
+    // update), then advances that head's counters. Nothing in this launch
+    // reads them; they wait for the barrier only to learn whether the step
+    // is taken, which it is by then long before the consumers finish.
+    if (taken) {
       for (int j0 = 0; j0 < n; j0 += 32) {  // ntok of 32 heads per round
         const int j = j0 + lane;
         if (j < n && tab.start[j] + tab.vlen[j] > a && tab.start[j] + tab.vlen[j] <= b)
@@ -871,16 +962,7 @@ __global__ void __launch_bounds__(step_threads<D, T>(), HKV_STEP_RESIDENT_PER_SM
         p.pos[tab.off[jj] + tab.vlen[jj] - 1] = p.n_cond + tab.ntok[jj];
     }
     STEP_TRACE_SET(8, globaltimer());
-
-    // counters of the heads this CTA appended, once every CTA has read them
-    while (!s_abort && !bar_done) {
-      if (lane == 0) bar_done = ld_acquire(p.bar + 1) != gen0;
-      bar_done = __shfl_sync(0xFFFFFFFFu, bar_done, 0);
-      if (!bar_done && timed_out()) break;
-    }
-    __syncwarp();
-    STEP_TRACE_SET(19, globaltimer());
-    if (!s_abort && active) {
+    if (taken) {
       for (int j = lane; j < n; j += 32) {
         const long long hs = tab.start[j], he = hs + tab.vlen[j];
         if (he > a && he <= b) {

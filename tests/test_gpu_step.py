@@ -1,0 +1,82 @@
+"""The one-launch decode step (hkv_decode_step when the layer fits its head
+table) on layers whose head lengths are far from equal: a few very long
+heads and many short ones, so that most CTA ranges lie far from where equal
+heads would put them and the prologue reads the range's counters in a
+second round. Every output against Eq. 1 (the oracle's fp64 attention), and
+the append and counters exact."""
+import numpy as np
+import pytest
+
+pytestmark = pytest.mark.gpu
+
+
+def _skewed(H, D, dtype, seed, long_len):
+    import torch
+    from paper_2605_20600_gb300.engine import CacheBuffers, torch_dtype
+    rng = np.random.default_rng(seed)
+    nh_seq, S, L = 100, 4, 2
+    cfg = H.make_config(n_layers=L, n_seqs=S, n_heads=nh_seq, head_dim=D, dtype=dtype,
+                        n_cond=1, n_image=4096, row_len=64, recent_w=128, local_w=8, period=8,
+                        group_at=long_len + 100, global_budget=512)
+    nh = S * nh_seq
+    lens = rng.integers(10, 60, size=(L, nh))
+    lens[:, :40] = rng.integers(long_len - 500, long_len, size=(L, 40))  # the long heads first
+    lens = lens.reshape(-1)
+    caps = lens + 3
+    off = np.zeros_like(caps)
+    off[1:] = np.cumsum(caps)[:-1]
+    total = int(caps.sum())
+    cb = CacheBuffers(cfg, total, "cuda")
+    dt = torch_dtype(cfg)
+    cb.k.copy_(torch.from_numpy(rng.normal(size=(total, D)).astype(np.float32)).to(dt))
+    cb.v.copy_(torch.from_numpy(rng.normal(size=(total, D)).astype(np.float32)).to(dt))
+    cb.off.copy_(torch.from_numpy(off))
+    cb.cap.copy_(torch.from_numpy(caps.astype(np.int32)))
+    cb.len.copy_(torch.from_numpy(lens.astype(np.int32)))
+    cb.ntok.copy_(torch.from_numpy(rng.integers(100, 200, size=L * nh).astype(np.int32)))
+    return cfg, cb, rng, nh
+
+
+@pytest.mark.parametrize("D,dtype,tol,long_len", [(128, "bf16", 2e-3, 3000), (64, "bf16", 2e-3, 3000),
+                                                  (128, "fp32", 1e-5, 1500)])
+def test_skewed_lengths_one_launch(D, dtype, tol, long_len):
+    import torch
+    from oracle import headkv as O
+    from paper_2605_20600_gb300 import hkv as H
+    from paper_2605_20600_gb300.engine import torch_dtype
+    cfg, cb, rng, nh = _skewed(H, D, dtype, D + len(dtype), long_len)
+    assert H.hkv_decode_step_launches(cfg) == 1
+    dt = torch_dtype(cfg)
+    ws = torch.zeros(H.hkv_workspace_size(cfg), dtype=torch.uint8, device="cuda")
+    st = torch.cuda.current_stream().cuda_stream
+    K0 = cb.k.float().cpu().numpy()
+    V0 = cb.v.float().cpu().numpy()
+    off = cb.off.cpu().numpy()
+    for step, layer in enumerate((1, 0, 1)):   # two calls on one layer: the barrier word again
+        ln0 = cb.len.cpu().numpy()
+        nt0 = cb.ntok.cpu().numpy()
+        q, k, v = (torch.from_numpy(rng.normal(size=(cfg.n_seqs, cfg.n_heads, D)).astype(np.float32))
+                   .to(dt).cuda() for _ in range(3))
+        out = torch.full((cfg.n_seqs, cfg.n_heads, D), float("nan"), dtype=torch.float32, device="cuda")
+        H.hkv_decode_step(cfg, cb.c, layer, q, k, v, out, ws, ws.numel(), 0, st)
+        torch.cuda.synchronize()
+        H.hkv_check(cb.c)
+        ln1 = cb.len.cpu().numpy()
+        sl = np.arange(layer * nh, (layer + 1) * nh)
+        assert (ln1[sl] == ln0[sl] + 1).all()
+        assert (np.delete(ln1, sl) == np.delete(ln0, sl)).all()
+        assert (cb.ntok.cpu().numpy()[sl] == nt0[sl] + 1).all()
+        qn, kn, vn = (x.float().cpu().numpy().reshape(nh, D) for x in (q, k, v))
+        got = out.cpu().numpy().reshape(nh, D)
+        Kc = cb.k.float().cpu().numpy()
+        Vc = cb.v.float().cpu().numpy()
+        pos = cb.pos.cpu().numpy()
+        for h in range(nh):
+            i = layer * nh + h
+            o, n_ = int(off[i]), int(ln0[i])
+            assert np.array_equal(Kc[o + n_], kn[h]) and np.array_equal(Vc[o + n_], vn[h])
+            assert pos[o + n_] == cfg.n_cond + nt0[i]
+            Kh = np.vstack([K0[o:o + n_], kn[h]]) if step < 2 else Kc[o:o + n_ + 1]
+            Vh = np.vstack([V0[o:o + n_], vn[h]]) if step < 2 else Vc[o:o + n_ + 1]
+            exp = O.attention(qn[h], Kh, Vh)
+            assert np.abs(got[h] - exp).max() <= tol, (layer, h)
