@@ -123,6 +123,15 @@ __device__ __forceinline__ bool mbar_test_wait(uint64_t *bar, uint32_t parity) {
   return ok != 0;
 }
 
+// 2^x with the hardware base-2 exponential (PTX ex2.approx.ftz.f32): a few
+// ulp; a subnormal result flushes to zero, which in a softmax only drops
+// weights below 2^-126 of the row's maximum
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 __device__ __forceinline__ uint64_t globaltimer() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
