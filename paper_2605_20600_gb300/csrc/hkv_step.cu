@@ -77,33 +77,39 @@ __device__ unsigned long long *g_step_trace = nullptr;  // [layer][kAttnMaxGrid]
 #endif
 
 // Tuning knobs (compile time) of the one-launch step, per head dimension:
-// consumer warps, bytes of K per stage, stages, tiles loaded before the wait
-// (measured at both head dimensions: 3 stages with 2 loaded before the wait
-// beat 2, 4 and 5 stages), and the CTAs per SM the kernel is built to be
-// resident with (the grid uses kStepActivePerSm).
+// consumer warps, bytes of K per stage, stages, tiles loaded before the wait,
+// and the CTAs per SM the kernel is built to be resident with (the grid uses
+// kStepActivePerSm). Measured per layer step (A/B in one process): rows of
+// 256 B stream best with 8 consumer warps over 48-row tiles in 3 stages, all
+// loaded before the wait (Lumina-mGPT 1024 at rho = 1/8: 13.01 us with 7
+// warps over 42 rows and 2 before the wait, 12.77 with 8 over 48, 12.63
+// with all 3 before it; 56-row tiles 13.06, 64-row tiles in 2 stages 13.10);
+// rows of 128 B (LlamaGen-XL's short heads, many to a CTA) with 128-row
+// tiles in 2 stages (15.26 us against 16.06 with 64-row tiles in 3 stages
+// and 17.42 with 96-row tiles in 3).
 #ifndef HKV_STEP_CW_D128
-#define HKV_STEP_CW_D128 HKV_ATTN_CW_D128
+#define HKV_STEP_CW_D128 8
 #endif
 #ifndef HKV_STEP_TILE_BYTES_D128
-#define HKV_STEP_TILE_BYTES_D128 HKV_ATTN_TILE_BYTES_D128
+#define HKV_STEP_TILE_BYTES_D128 12288
 #endif
 #ifndef HKV_STEP_STAGES_D128
 #define HKV_STEP_STAGES_D128 3
 #endif
 #ifndef HKV_STEP_PRE_D128
-#define HKV_STEP_PRE_D128 2
+#define HKV_STEP_PRE_D128 3
 #endif
 #ifndef HKV_STEP_CW_D64
-#define HKV_STEP_CW_D64 HKV_ATTN_CW_D64
+#define HKV_STEP_CW_D64 8
 #endif
 #ifndef HKV_STEP_TILE_BYTES_D64
-#define HKV_STEP_TILE_BYTES_D64 HKV_ATTN_TILE_BYTES_D64
+#define HKV_STEP_TILE_BYTES_D64 16384
 #endif
 #ifndef HKV_STEP_STAGES_D64
-#define HKV_STEP_STAGES_D64 3
+#define HKV_STEP_STAGES_D64 2
 #endif
 #ifndef HKV_STEP_PRE_D64
-#define HKV_STEP_PRE_D64 2
+#define HKV_STEP_PRE_D64 1
 #endif
 #ifndef HKV_STEP_RESIDENT_PER_SM
 #define HKV_STEP_RESIDENT_PER_SM 2
