@@ -22,9 +22,9 @@
 //    every pair carries this launch's epoch, while its consumers stream.
 //    Pieces are combined in index order and the CTA's own piece last, so the
 //    result does not depend on timing;
-//  * prologue: every CTA loads the lengths of all the layer's heads
-//    (coalesced, into shared memory) to place the ranges, but reads and
-//    checks the other counters only for the heads of its own range;
+//  * prologue: every CTA reads the lengths of all the layer's heads to place
+//    the ranges, but checks the other counters only for the heads of its own
+//    range, in the same round of loads;
 //  * appends and counters: every CTA arrives on a per-layer barrier word
 //    once it is done reading the layer's counters (a CTA that found a bad
 //    head marks its arrival); once the whole grid has arrived, and unless
