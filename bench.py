@@ -339,13 +339,22 @@ def measure_period(args, w, dev, world, K, W, *, e2e: bool):
     staging = torch.empty(3, P, L, S, Hh, D, dtype=dt, device=dev)
     out = torch.empty(P, L, S, Hh, D, dtype=torch.float32, device=dev)
 
+    per_layer = args.update == "per-layer"
+
     def period_calls(events=None, staging=staging, out=out):
-        # the period starts with the update of every layer (its buffer is full);
-        # events (instrumented copy only): [step_begin, step_end] per decode
-        # step, then [evict_begin, evict_end] per layer
+        # the period starts with the update of every layer (every buffer is
+        # full): one launch for all layers, or one before each layer's first
+        # step; events (instrumented copy only): [step_begin, step_end] per
+        # decode step, then [update_begin, update_end] per update launch
         for p in range(P):
+            if p == 0 and not per_layer:
+                if events is not None:
+                    events[P * L][0].record()
+                eng.evict_all()
+                if events is not None:
+                    events[P * L][1].record()
             for layer in range(L):
-                if p == 0:
+                if p == 0 and per_layer:
                     if events is not None:
                         events[P * L + layer][0].record()
                     eng.evict(layer)
@@ -363,9 +372,9 @@ def measure_period(args, w, dev, world, K, W, *, e2e: bool):
         period_calls()
     stream = torch.cuda.current_stream()
     # per period: the kernels of every decode step (one launch, or an
-    # attention and a finishing kernel) and every layer's update kernel
+    # attention and a finishing kernel) and the update of every layer (one)
     step_launches = H.hkv_decode_step_launches(cfg)
-    launches_per_step = step_launches * P * L + L
+    launches_per_step = step_launches * P * L + (L if per_layer else 1)
 
     def barrier():
         if world > 1:
@@ -406,7 +415,7 @@ def measure_period(args, w, dev, world, K, W, *, e2e: bool):
                   for p in range(P) for layer in range(L)]
     bytes_per_launch = statistics.mean(per_launch)
     events = [(torch.cuda.Event(enable_timing=True, external=True),
-               torch.cuda.Event(enable_timing=True, external=True)) for _ in range(P * L + L)]
+               torch.cuda.Event(enable_timing=True, external=True)) for _ in range(P * L + (L if per_layer else 1))]
     igraph = torch.cuda.CUDAGraph()
     with torch.cuda.graph(igraph):
         period_calls(events)
@@ -542,7 +551,9 @@ def run_ours(args):
                           if args.budget == "redistribute" else {}),
                        **({"distance": "grid (identification and Eq. 5 strata by squared "
                                        "distance on the image grid)"}
-                          if args.distance == "grid2d" else {})},
+                          if args.distance == "grid2d" else {}),
+                       "update": ("every layer in one launch (hkv_evict_all)" if args.update == "all"
+                                  else "one launch per layer (hkv_evict)")},
             "global_head_fraction": float((r["labels"] == 1).mean()),
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak,
@@ -648,8 +659,7 @@ def strategies_setup(w, dev):
     synth = DeviceSynth(w, dev)
     generate(eng, synth, last_step=t0 - 1)
     eng.release_dense()
-    for layer in range(L):
-        eng.evict(layer)
+    eng.evict_all()
     torch.cuda.synchronize()
     eng.check()
     q = torch.empty(1, L, S, Hh, D, dtype=torch_dtype(cfg), device=dev)
@@ -1029,6 +1039,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--strategies", action="store_true",
                     help="compare decode attention with the padding and per-group strategies")
+    ap.add_argument("--update", default="all", choices=["all", "per-layer"],
+                    help="the periodic update of every layer in one launch (hkv_evict_all) "
+                         "or one launch per layer (hkv_evict)")
     ap.add_argument("--budget", default="paper", choices=["paper", "redistribute"],
                     help="budget rule: the paper's, or local heads' unused tokens to global heads")
     ap.add_argument("--distance", default="raster", choices=["raster", "grid2d"],

@@ -247,6 +247,14 @@ hkv_status hkv_append_evict(const hkv_config *cfg, const hkv_cache *cache, int l
  * HKV_ERR_CAPACITY (also for hkv_append_evict and hkv_repack). */
 hkv_status hkv_evict(const hkv_config *cfg, const hkv_cache *cache, int layer, hkv_stream_t stream);
 
+/* hkv_evict for every layer in one launch (one CTA per head of the model):
+ * the same update of every head whose buffer holds P tokens, the same
+ * results, the same checks and errors. All heads fill their buffers at the
+ * same token, so one call before the first layer's step replaces a call
+ * per layer; the per-head updates are independent and latency-bound, and
+ * one launch keeps the GPU full with them. Asynchronous on `stream`. */
+hkv_status hkv_evict_all(const hkv_config *cfg, const hkv_cache *cache, hkv_stream_t stream);
+
 /* One decode step of one layer: the append of the new token (Sec. 3, KV
  * Cache) fused with the attention of Eq. 1 over the cache including that
  * token. One kernel launch when every CTA's share of the layer spans at

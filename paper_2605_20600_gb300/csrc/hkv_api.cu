@@ -490,19 +490,38 @@ hkv_status hkv_decode_step_identify(const hkv_config *cfg, const hkv_cache *cach
                      workspace, ws_bytes, flags, stream);
 }
 
+namespace {
+
+// the periodic update of the layers [first, first + count) in one launch
+hkv_status evict_layers(const hkv_config *cfg, const hkv_cache *cache, int first, int count,
+                        hkv_stream_t stream) {
+  DeviceState *st;
+  HKV_TRY(device_state(&st));
+  const size_t smem = update_smem_bytes(max_segment(cfg), cfg->head_dim, cfg->period, cfg->dtype);
+  HKV_TRY(update_ready(st, cfg->head_dim, cfg->dtype, smem));
+  const long long hpl = heads_per_layer(cfg);
+  if (hpl * count > 0x7FFFFFFFLL) return HKV_ERR_SHAPE;  // one CTA per head
+  return cuda_status(launch_evict(cache_args(cache), method_args(cfg), (int)(first * hpl),
+                                  (int)(count * hpl), cfg->head_dim, cfg->dtype, smem,
+                                  (cudaStream_t)stream));
+}
+
+}  // namespace
+
 hkv_status hkv_evict(const hkv_config *cfg, const hkv_cache *cache, int layer,
                      hkv_stream_t stream) {
   HKV_TRY(injected("evict"));
   HKV_TRY(hkv_validate_config(cfg));
   HKV_TRY(check_cache(cache));
   if (layer < 0 || layer >= cfg->n_layers) return HKV_ERR_INVALID_ARG;
-  DeviceState *st;
-  HKV_TRY(device_state(&st));
-  const size_t smem = update_smem_bytes(max_segment(cfg), cfg->head_dim, cfg->period, cfg->dtype);
-  HKV_TRY(update_ready(st, cfg->head_dim, cfg->dtype, smem));
-  const int hpl = heads_per_layer(cfg);
-  return cuda_status(launch_evict(cache_args(cache), method_args(cfg), layer * hpl, hpl,
-                                  cfg->head_dim, cfg->dtype, smem, (cudaStream_t)stream));
+  return evict_layers(cfg, cache, layer, 1, stream);
+}
+
+hkv_status hkv_evict_all(const hkv_config *cfg, const hkv_cache *cache, hkv_stream_t stream) {
+  HKV_TRY(injected("evict_all"));
+  HKV_TRY(hkv_validate_config(cfg));
+  HKV_TRY(check_cache(cache));
+  return evict_layers(cfg, cache, 0, cfg->n_layers, stream);
 }
 
 hkv_status hkv_identify_heads(const hkv_config *cfg, const hkv_cache *cache, int layer,

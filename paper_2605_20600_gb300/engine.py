@@ -86,6 +86,10 @@ class Engine:
     def evict(self, layer: int) -> None:
         H.hkv_evict(self.cfg, self.cache.c, layer, self.stream())
 
+    def evict_all(self) -> None:
+        """The periodic update of every layer in one launch."""
+        H.hkv_evict_all(self.cfg, self.cache.c, self.stream())
+
     def step(self, layer: int, q, k, v, out) -> None:
         # layers run in order, so with two or more layers the kernel before a
         # decode step belongs to another layer (or is hkv_evict, which never

@@ -79,6 +79,7 @@ _SIGNATURES = {
     "hkv_global_budget": ([c_int64, c_int64, c_int32, POINTER(c_int32)], c_int),
     "hkv_update_due": ([POINTER(hkv_config), c_int32, POINTER(c_int32)], c_int),
     "hkv_evict": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p], c_int),
+    "hkv_evict_all": ([POINTER(hkv_config), POINTER(hkv_cache), c_void_p], c_int),
     "hkv_identify_heads": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p, c_void_p, c_void_p,
                             c_void_p], c_int),
     "hkv_identify_heads_multi": ([POINTER(hkv_config), POINTER(hkv_cache), c_int, c_void_p, c_void_p,
@@ -203,6 +204,10 @@ def hkv_decode_step_identify(cfg, cache, layer, q, k, v, out, label_out, workspa
 
 def hkv_evict(cfg, cache, layer, stream=0) -> None:
     _call("evict", ctypes.byref(cfg), ctypes.byref(cache), layer, stream)
+
+
+def hkv_evict_all(cfg, cache, stream=0) -> None:
+    _call("evict_all", ctypes.byref(cfg), ctypes.byref(cache), stream)
 
 
 def hkv_identify_heads(cfg, cache, layer, q, label_out, nh_out=None, stream=0) -> None:

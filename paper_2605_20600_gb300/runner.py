@@ -18,8 +18,9 @@ def generate(engine: Engine, provider, *, last_step: int | None = None, on_step=
              identify: str | None = None) -> None:
     """Runs image tokens first_step..last_step (default N-1) for every layer.
 
-    fused: per layer and step, hkv_evict when the update is due and then
-    hkv_decode_step; otherwise hkv_append_evict then hkv_decode_attention.
+    fused: hkv_evict_all (every layer in one launch) when the update is due,
+    then hkv_decode_step per layer; otherwise hkv_append_evict then
+    hkv_decode_attention per layer.
     on_step(t, out) receives out [L][S][H][D] (fp32, device) after step t.
     before_compress(engine) runs after grouping, before budgets and repack.
     first_step > 0 continues a generation (the prefill is skipped).
@@ -54,10 +55,10 @@ def generate(engine: Engine, provider, *, last_step: int | None = None, on_step=
     for t in range(first_step, last + 1):
         provider.image(q, k, v, 0, L, t, 1, st)
         due = engine.update_due(t)
+        if fused and due:
+            engine.evict_all()       # every layer's buffer fills at the same token
         for layer in range(L):
             if fused:
-                if due:
-                    engine.evict(layer)
                 if t == E - 1 and identify == "fused":
                     engine.step_identify(layer, q[layer], k[layer], v[layer], out[layer])
                 else:

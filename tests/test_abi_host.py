@@ -47,7 +47,7 @@ def fake_cache(H, **kw):
 
 def test_every_declared_symbol_is_exported(H):
     names = declared_functions()
-    assert len(names) == 20
+    assert len(names) == 21
     for n in names:
         assert hasattr(H.lib(), n), n
     assert set(names) >= {"hkv_identify_heads", "hkv_allocate_budgets", "hkv_append_evict",
@@ -130,6 +130,9 @@ def test_null_and_misaligned_arguments(H):
     assert lib.hkv_decode_step(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 24, 16, 16, 16, 1 << 30, 0, None) == 8
     assert lib.hkv_decode_step(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, 16, 16, 16, 1 << 30, 6, None) == 1
     assert lib.hkv_evict(ctypes.byref(cfg), ctypes.byref(c), 5, None) == 1
+    assert lib.hkv_evict_all(ctypes.byref(cfg), None, None) == 1
+    assert lib.hkv_evict_all(None, ctypes.byref(c), None) == 1
+    assert lib.hkv_evict_all(ctypes.byref(tiny_cfg(H, head_dim=32)), ctypes.byref(c), None) == 2
     cnt = ctypes.c_int64(0)
     assert lib.hkv_export_state(ctypes.byref(cfg), None, 0, None, None, None, None, None, 0,
                                 ctypes.byref(cnt), None) == 1
@@ -153,8 +156,8 @@ def test_null_and_misaligned_arguments(H):
 
 @pytest.mark.parametrize("name", ["decode_attention", "append_evict", "identify_heads",
                                   "allocate_budgets", "repack", "prefill", "init_dense", "check",
-                                  "decode_step", "evict", "export_state", "decode_step_identify",
-                                  "identify_heads_multi"])
+                                  "decode_step", "evict", "evict_all", "export_state",
+                                  "decode_step_identify", "identify_heads_multi"])
 def test_fault_injection_returns_the_code(H, name, monkeypatch):
     cfg = tiny_cfg(H)
     c = fake_cache(H)
@@ -172,6 +175,7 @@ def test_fault_injection_returns_the_code(H, name, monkeypatch):
         "check": lambda: lib.hkv_check(ctypes.byref(c), None),
         "decode_step": lambda: lib.hkv_decode_step(ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, 16, 16, 16, 1 << 30, 0, None),
         "evict": lambda: lib.hkv_evict(ctypes.byref(cfg), ctypes.byref(c), 0, None),
+        "evict_all": lambda: lib.hkv_evict_all(ctypes.byref(cfg), ctypes.byref(c), None),
         "decode_step_identify": lambda: lib.hkv_decode_step_identify(
             ctypes.byref(cfg), ctypes.byref(c), 0, 16, 16, 16, 16, 16, 16, 1 << 30, 0, None),
         "export_state": lambda: lib.hkv_export_state(ctypes.byref(cfg), ctypes.byref(c), 0, None, None,

@@ -80,3 +80,47 @@ def test_skewed_lengths_one_launch(D, dtype, tol, long_len):
             Vh = np.vstack([V0[o:o + n_], vn[h]]) if step < 2 else Vc[o:o + n_ + 1]
             exp = O.attention(qn[h], Kh, Vh)
             assert np.abs(got[h] - exp).max() <= tol, (layer, h)
+
+
+@pytest.mark.parametrize("name", ["lumina1024", "llamagen_xl"])
+def test_update_of_every_layer_in_one_launch_equals_one_per_layer(name):
+    """hkv_evict_all runs the same update as hkv_evict on every layer: two
+    engines fed the same tokens up to a due update, one updated layer by
+    layer and one in one launch, hold the same cache bit for bit."""
+    import torch
+    from fractions import Fraction
+    from paper_2605_20600_gb300 import hkv as H
+    from paper_2605_20600_gb300.engine import Engine
+    from paper_2605_20600_gb300.runner import generate
+    from synth import configs
+    from synth.gpu import DeviceSynth
+    from _gpu_util import cfg_of
+    w = configs.ALL[name].with_(n_layers=3, n_seqs=2, rho=Fraction(1, 6))
+    t = w.group_at + 2 * w.period      # the second update after grouping is due
+    engines = []
+    for per_layer in (True, False):
+        eng = Engine(cfg_of(H, w), "cuda")
+        generate(eng, DeviceSynth(w, "cuda"), last_step=t - 1)
+        eng.release_dense()
+        assert eng.update_due(t)
+        nbuf0 = eng.cache.nbuf.clone()
+        if per_layer:
+            for layer in range(w.n_layers):
+                eng.evict(layer)
+        else:
+            eng.evict_all()
+        torch.cuda.synchronize()
+        eng.check()
+        engines.append((eng, nbuf0))
+    (a, nb_a), (b, nb_b) = engines
+    assert torch.equal(nb_a, nb_b) and int((nb_a == w.period).sum()) > 0
+    for nm in ("len", "nbuf", "ntok", "off", "cap", "label"):
+        assert torch.equal(getattr(a.cache, nm), getattr(b.cache, nm)), nm
+    # every retained row, position and buffered query
+    ln = a.cache.len.cpu().numpy()
+    off = a.cache.off.cpu().numpy()
+    for i in range(len(ln)):
+        o, n = int(off[i]), int(ln[i])
+        assert torch.equal(a.cache.k[o:o + n], b.cache.k[o:o + n]), i
+        assert torch.equal(a.cache.v[o:o + n], b.cache.v[o:o + n]), i
+        assert torch.equal(a.cache.pos[o:o + n], b.cache.pos[o:o + n]), i
