@@ -132,8 +132,8 @@ def oracle_labels(w, layers, seqs, multi=False, distance=0):
 
 
 # |fp64 mass - tau| below this: either decision is correct (the GPU sums the
-# same weights in fp32, whose rounding over a few thousand terms stays well
-# inside this band)
+# same weights in fp32; on every tested shape its rounding stays inside this
+# band)
 LABEL_TIE = 1e-5
 
 
