@@ -124,3 +124,60 @@ def test_update_of_every_layer_in_one_launch_equals_one_per_layer(name):
         assert torch.equal(a.cache.k[o:o + n], b.cache.k[o:o + n]), i
         assert torch.equal(a.cache.v[o:o + n], b.cache.v[o:o + n]), i
         assert torch.equal(a.cache.pos[o:o + n], b.cache.pos[o:o + n]), i
+
+
+@pytest.mark.parametrize("D,dtype,tol", [(128, "bf16", 2e-3), (64, "bf16", 2e-3), (128, "fp32", 1e-5),
+                                         (64, "fp32", 1e-5)])
+def test_lengths_at_tile_boundaries(D, dtype, tol):
+    """Empty heads (the new token only) and lengths one below, at and one
+    above every tile size the step uses (24, 48, 64 and 128 rows, by head
+    dimension and type), many heads per layer, one launch: every output
+    against Eq. 1, the appends and counters exact."""
+    import torch
+    from oracle import headkv as O
+    from paper_2605_20600_gb300 import hkv as H
+    from paper_2605_20600_gb300.engine import CacheBuffers, torch_dtype
+    rng = np.random.default_rng(31 + D)
+    base = [0, 1, 23, 24, 25, 47, 48, 49, 63, 64, 65, 127, 128, 129, 255, 256, 257]
+    S, nh_seq, L = 3, 68, 2
+    cfg = H.make_config(n_layers=L, n_seqs=S, n_heads=nh_seq, head_dim=D, dtype=dtype,
+                        n_cond=1, n_image=512, row_len=16, recent_w=32, local_w=8, period=8,
+                        group_at=300, global_budget=128)
+    nh = S * nh_seq
+    lens = np.array([base[(i * 7) % len(base)] for i in range(L * nh)], dtype=np.int64)
+    caps = lens + 2
+    off = np.zeros_like(caps)
+    off[1:] = np.cumsum(caps)[:-1]
+    total = int(caps.sum())
+    cb = CacheBuffers(cfg, total, "cuda")
+    dt = torch_dtype(cfg)
+    cb.k.copy_(torch.from_numpy(rng.normal(size=(total, D)).astype(np.float32)).to(dt))
+    cb.v.copy_(torch.from_numpy(rng.normal(size=(total, D)).astype(np.float32)).to(dt))
+    cb.off.copy_(torch.from_numpy(off))
+    cb.cap.copy_(torch.from_numpy(caps.astype(np.int32)))
+    cb.len.copy_(torch.from_numpy(lens.astype(np.int32)))
+    assert H.hkv_decode_step_launches(cfg) == 1
+    K0 = cb.k.float().cpu().numpy()
+    V0 = cb.v.float().cpu().numpy()
+    ws = torch.zeros(H.hkv_workspace_size(cfg), dtype=torch.uint8, device="cuda")
+    st = torch.cuda.current_stream().cuda_stream
+    layer = 1
+    q, k, v = (torch.from_numpy(rng.normal(size=(S, nh_seq, D)).astype(np.float32)).to(dt).cuda()
+               for _ in range(3))
+    out = torch.full((S, nh_seq, D), float("nan"), dtype=torch.float32, device="cuda")
+    H.hkv_decode_step(cfg, cb.c, layer, q, k, v, out, ws, ws.numel(), 0, st)
+    torch.cuda.synchronize()
+    H.hkv_check(cb.c)
+    ln1 = cb.len.cpu().numpy()
+    qn, kn, vn = (x.float().cpu().numpy().reshape(nh, D) for x in (q, k, v))
+    got = out.cpu().numpy().reshape(nh, D)
+    Kc = cb.k.float().cpu().numpy()
+    Vc = cb.v.float().cpu().numpy()
+    for h in range(nh):
+        i = layer * nh + h
+        o, n_ = int(off[i]), int(lens[i])
+        assert ln1[i] == n_ + 1
+        assert np.array_equal(Kc[o + n_], kn[h]) and np.array_equal(Vc[o + n_], vn[h])
+        exp = O.attention(qn[h], np.vstack([K0[o:o + n_], kn[h]]), np.vstack([V0[o:o + n_], vn[h]]))
+        assert np.abs(got[h] - exp).max() <= tol, (h, n_)
+    assert (ln1[:nh] == lens[:nh]).all()          # the other layer untouched
